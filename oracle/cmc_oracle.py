@@ -1,0 +1,218 @@
+"""Plain, slow fp64 CPU oracle of the CMC two-tier decode path.
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product imports this module; the
+CUDA library never calls it and it never calls the CUDA library.
+
+What it computes, following Section 2.5 of the paper ("Inference with Two-Tier
+KV Cache Policy"):
+
+* Tier-1 scoring: the cosine similarity between each decoder-ready CME m_j and
+  the mean-pooled question vector q_vec (the score_j equation of Section 2.5).
+* Tier-1 selection: keep the K highest-scoring CMEs, then re-order the kept
+  ones by original document position, i.e. by ascending index (Section 2.5,
+  text after the score_j equation).
+* Tier-2 window: a ring of W token slots per (sequence, layer, KV head) that
+  receives each generated token; the cache then stays bounded by K + W + |q|
+  tokens at every generation step (Section 2.5, "KV cache assembly").
+* Decode attention: for each query head, softmax(q . k_i * scale) over the
+  keys of [Tier-1 | Tier-2], applied to the values.  The MAC model of the
+  appendix ("Attention MACs Analysis", MACs_t = 2 n_h d_h n_l L_t) counts
+  exactly this per-step work over L_t cached keys.
+
+Readings where the paper is silent (each is also listed in the design notes):
+
+* A zero vector has no direction; its cosine score is taken as 0.
+* Ties in score go to the lower index, and the selection decision is taken on
+  the scores rounded to float32, the precision the kernels compute them in.
+  Scores themselves are computed in fp64.
+* The ring slot of token number p (counting from 0) is p mod W; once more than
+  W tokens have been appended the oldest is overwritten (sliding window).
+* Within a decode step the new token is appended before attention, so it
+  attends to itself (standard autoregressive decoding).
+* scale defaults to 1/sqrt(d); cached keys are taken as already position-
+  encoded, so no rotary embedding is applied here; nothing is masked.
+* Query head h reads KV head h // (Hq / Hkv) (grouped-query attention).
+* An empty cache (no Tier-1 rows and no ring tokens) yields a zero output.
+
+Parity status: every function here is pinned by the tests in
+tests/test_oracle_pins.py (closed forms, brute force, library routines,
+invariants); none is "parity unpinned".
+"""
+
+from __future__ import annotations
+
+import math
+from typing import Iterable, Optional, Tuple
+
+import numpy as np
+
+
+# ----------------------------------------------------------------------------
+# Inputs
+# ----------------------------------------------------------------------------
+
+def bf16_to_f64(a: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) -> float64, exact.  Float arrays pass
+    through as float64."""
+    a = np.asarray(a)
+    if a.dtype == np.uint16:
+        return (a.astype(np.uint32) << np.uint32(16)).view(np.float32).astype(np.float64)
+    return a.astype(np.float64)
+
+
+# ----------------------------------------------------------------------------
+# Tier-1: question-guided scoring and top-K selection (Section 2.5)
+# ----------------------------------------------------------------------------
+
+def cosine_scores(question_emb: np.ndarray, cme_bank: np.ndarray) -> np.ndarray:
+    """score[b, j] = (m_j . q_vec) / (||m_j|| ||q_vec||)  (Section 2.5, score_j).
+
+    question_emb: [B, D]; cme_bank: [B, N, D].  Returns float64 [B, N].
+    A zero-norm CME or question vector gives score 0.
+    """
+    q = np.asarray(question_emb, dtype=np.float64)
+    m = np.asarray(cme_bank, dtype=np.float64)
+    B, N, D = m.shape
+    out = np.zeros((B, N), dtype=np.float64)
+    for b in range(B):
+        qn = math.sqrt(float(q[b] @ q[b]))
+        for j0 in range(0, N, 4096):
+            rows = m[b, j0:j0 + 4096]
+            dots = rows @ q[b]
+            mn = np.sqrt(np.einsum("ij,ij->i", rows, rows))
+            den = mn * qn
+            s = np.zeros_like(dots)
+            nz = den > 0.0
+            s[nz] = dots[nz] / den[nz]
+            out[b, j0:j0 + 4096] = s
+    return out
+
+
+def select_top_k(scores: np.ndarray, k: int) -> np.ndarray:
+    """The k highest scores per row, returned as indices in ascending order
+    (Section 2.5: top-K, then re-ordered by original document position).
+
+    The decision is taken on the scores rounded to float32; equal scores go to
+    the lower index.  Returns int64 [B, k].
+    """
+    s = np.asarray(scores)
+    B, N = s.shape
+    if not 0 <= k <= N:
+        raise ValueError(f"k={k} outside [0, N={N}]")
+    s32 = s.astype(np.float32)
+    out = np.empty((B, k), dtype=np.int64)
+    j = np.arange(N)
+    for b in range(B):
+        # primary key: score descending; secondary: index ascending
+        ranked = np.lexsort((j, -s32[b]))
+        out[b] = np.sort(ranked[:k])
+    return out
+
+
+def score_select(question_emb: np.ndarray, cme_bank: np.ndarray, k: int
+                 ) -> Tuple[np.ndarray, np.ndarray]:
+    """Tier-1 selection M* = TopK(M, q, K) (Section 2.5).  Returns (idx, scores)."""
+    scores = cosine_scores(question_emb, cme_bank)
+    return select_top_k(scores, k), scores
+
+
+# ----------------------------------------------------------------------------
+# Tier-2: local-window ring (Section 2.5, Tier-2 and KV cache assembly)
+# ----------------------------------------------------------------------------
+
+def window_slots(pos: int, W: int) -> range:
+    """Ring slots that hold tokens after `pos` tokens have been appended."""
+    return range(min(int(pos), W))
+
+
+def window_append(ring_k: np.ndarray, ring_v: np.ndarray, pos: np.ndarray,
+                  k_new: np.ndarray, v_new: np.ndarray) -> None:
+    """Append one token per sequence, in place.
+
+    ring_k/ring_v: [B, L, Hkv, W, d]; pos: int64 [B] tokens appended so far;
+    k_new/v_new: [B, L, Hkv, d].  Token number pos[b] goes to slot pos[b] mod W,
+    overwriting the oldest token once the ring is full; pos[b] then grows by 1.
+    """
+    W = ring_k.shape[3]
+    for b in range(ring_k.shape[0]):
+        s = int(pos[b]) % W
+        ring_k[b, :, :, s, :] = k_new[b]
+        ring_v[b, :, :, s, :] = v_new[b]
+        pos[b] += 1
+
+
+# ----------------------------------------------------------------------------
+# Decode attention over [Tier-1 | Tier-2]
+# ----------------------------------------------------------------------------
+
+def default_scale(d: int) -> float:
+    return 1.0 / math.sqrt(d)
+
+
+def softmax_attention(q: np.ndarray, K: np.ndarray, V: np.ndarray, scale: float
+                      ) -> np.ndarray:
+    """sum_i softmax_i(scale * q . k_i) v_i for one query vector, in fp64.
+
+    q: [d]; K, V: [n, d].  n == 0 gives zeros.
+    """
+    q = np.asarray(q, dtype=np.float64)
+    if K.shape[0] == 0:
+        return np.zeros(V.shape[1], dtype=np.float64)
+    z = scale * (np.asarray(K, dtype=np.float64) @ q)
+    z = z - z.max()
+    p = np.exp(z)
+    return (p @ np.asarray(V, dtype=np.float64)) / p.sum()
+
+
+def two_tier_kv(tier1_k, tier1_v, idx_b: Iterable[int], ring_k, ring_v, pos_b: int,
+                b: int, l: int, g: int) -> Tuple[np.ndarray, np.ndarray]:
+    """Keys and values one KV head sees: the Tier-1 bank rows at the selected
+    indices, followed by the ring's occupied slots.  Returned as fp64 [n, d]."""
+    sel = np.asarray(list(idx_b), dtype=np.int64)
+    W = ring_k.shape[3]
+    slots = np.asarray(window_slots(pos_b, W), dtype=np.int64)
+    K = np.concatenate([bf16_to_f64(tier1_k[b, l, g][sel]),
+                        bf16_to_f64(ring_k[b, l, g][slots])], axis=0)
+    V = np.concatenate([bf16_to_f64(tier1_v[b, l, g][sel]),
+                        bf16_to_f64(ring_v[b, l, g][slots])], axis=0)
+    return K, V
+
+
+def two_tier_attention_head(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos,
+                            b: int, l: int, h: int, scale: Optional[float] = None
+                            ) -> np.ndarray:
+    """Output of query head h of layer l, sequence b: fp64 [d]."""
+    Hq = q.shape[2]
+    Hkv = ring_k.shape[2]
+    g = h // (Hq // Hkv)
+    d = q.shape[3]
+    sc = default_scale(d) if scale is None else scale
+    idx_b = [] if idx is None else idx[b]
+    K, V = two_tier_kv(tier1_k, tier1_v, idx_b, ring_k, ring_v, int(pos[b]), b, l, g)
+    return softmax_attention(bf16_to_f64(q[b, l, h]), K, V, sc)
+
+
+def two_tier_attention(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos,
+                       scale: Optional[float] = None) -> np.ndarray:
+    """Decode attention over [Tier-1 | Tier-2] for every (b, l, h).
+
+    q: [B, L, Hq, d]; tier1_k/v: [B, L, Hkv, N, d]; idx: [B, k] (or None for
+    k = 0); ring_k/v: [B, L, Hkv, W, d]; pos: [B] tokens appended so far.
+    Returns fp64 [B, L, Hq, d].
+    """
+    B, L, Hq, d = q.shape
+    out = np.zeros((B, L, Hq, d), dtype=np.float64)
+    for b in range(B):
+        for l in range(L):
+            for h in range(Hq):
+                out[b, l, h] = two_tier_attention_head(
+                    q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, b, l, h, scale)
+    return out
+
+
+def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new,
+                scale: Optional[float] = None) -> np.ndarray:
+    """One decode step: append the new token to the ring, then attend.
+    ring_k, ring_v and pos are updated in place."""
+    window_append(ring_k, ring_v, pos, k_new, v_new)
+    return two_tier_attention(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, scale)

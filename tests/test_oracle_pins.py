@@ -1,0 +1,381 @@
+"""Pins of the fp64 oracle against facts fixed outside it.
+
+Each test checks the oracle against something other than its own formula:
+closed forms, brute force over all candidate answers, library routines
+(scipy / torch fp64) on the special cases they cover, and invariants of the
+method (Section 2.5: cosine scoring, top-K with document-order re-ordering,
+the bounded two-tier cache).  A plausible slip in the oracle (a dropped norm,
+a wrong sign, a transposed operand, an off-by-one in the ring, the wrong GQA
+head mapping, a missing scale) fails at least one of them.
+"""
+
+import itertools
+import math
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import oracle
+from workloads import (WORKLOADS, selection_inputs, kv_inputs, step_inputs,
+                       f32_to_bf16_bits, bf16_bits_to_f32)
+from workloads.configs import Workload
+
+pytestmark = pytest.mark.filterwarnings("ignore::DeprecationWarning")
+
+
+# ----------------------------------------------------------------------------
+# Cosine scoring (Section 2.5, score_j)
+# ----------------------------------------------------------------------------
+
+def test_cosine_closed_forms():
+    q = np.array([[3.0, 4.0]])
+    bank = np.array([[[4.0, 3.0],     # 24 / 25
+                      [6.0, 8.0],     # parallel: 1
+                      [-3.0, -4.0],   # antiparallel: -1
+                      [-4.0, 3.0],    # orthogonal: 0
+                      [0.0, 0.0],     # zero vector: 0 (reading)
+                      [0.0, 5.0]]])   # 20 / 25
+    s = oracle.cosine_scores(q, bank)
+    assert s.shape == (1, 6)
+    np.testing.assert_allclose(s[0], [24 / 25, 1.0, -1.0, 0.0, 0.0, 0.8], rtol=0, atol=1e-15)
+
+
+def test_cosine_zero_question_gives_zero_scores():
+    s = oracle.cosine_scores(np.zeros((1, 8)), np.ones((1, 5, 8)))
+    assert np.all(s == 0.0)
+
+
+def test_cosine_against_scipy_and_torch():
+    rng = np.random.default_rng(11)
+    q = rng.standard_normal((3, 37))
+    bank = rng.standard_normal((3, 50, 37)) * rng.uniform(0.1, 10, size=(3, 50, 1))
+    s = oracle.cosine_scores(q, bank)
+    t = F.cosine_similarity(torch.from_numpy(bank), torch.from_numpy(q)[:, None, :], dim=-1)
+    np.testing.assert_allclose(s, t.numpy(), rtol=0, atol=1e-13)
+    spatial = pytest.importorskip("scipy.spatial.distance")
+    for b in range(3):
+        for j in range(0, 50, 7):
+            assert abs(s[b, j] - (1.0 - spatial.cosine(bank[b, j], q[b]))) < 1e-13
+
+
+def test_cosine_scale_invariance_and_sign():
+    rng = np.random.default_rng(12)
+    q = rng.standard_normal((1, 64))
+    bank = rng.standard_normal((1, 20, 64))
+    c = rng.uniform(0.01, 100.0, size=(1, 20, 1))
+    s = oracle.cosine_scores(q, bank)
+    np.testing.assert_allclose(oracle.cosine_scores(q, bank * c), s, rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(oracle.cosine_scores(q * 7.5, bank), s, rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(oracle.cosine_scores(q, -bank), -s, rtol=0, atol=0)
+    assert np.all(np.abs(s) <= 1.0)
+
+
+# ----------------------------------------------------------------------------
+# Top-K selection, re-ordered by document position (Section 2.5)
+# ----------------------------------------------------------------------------
+
+def _brute_force_topk(s: np.ndarray, k: int):
+    """The unique k-subset S such that every kept j beats every dropped i:
+    s_j > s_i, or s_j == s_i and j < i (ties to the lower index)."""
+    N = len(s)
+    found = []
+    for S in itertools.combinations(range(N), k):
+        inside = set(S)
+        ok = all((s[j] > s[i]) or (s[j] == s[i] and j < i)
+                 for j in inside for i in range(N) if i not in inside)
+        if ok:
+            found.append(S)
+    assert len(found) == 1
+    return list(found[0])
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_select_brute_force(seed):
+    rng = np.random.default_rng(seed)
+    N = 7
+    # few distinct values, so ties straddle the cut often
+    s = rng.integers(-2, 3, size=(1, N)).astype(np.float64) / 4.0
+    for k in range(N + 1):
+        got = oracle.select_top_k(s, k)[0].tolist()
+        assert got == _brute_force_topk(s[0].astype(np.float32), k)
+        assert got == sorted(got)
+
+
+def test_select_ties_go_to_lower_index():
+    s = np.full((2, 10), 0.25)
+    np.testing.assert_array_equal(oracle.select_top_k(s, 4), [[0, 1, 2, 3]] * 2)
+    s = np.array([[0.1, 0.5, 0.3, 0.5, 0.5, 0.2]])
+    np.testing.assert_array_equal(oracle.select_top_k(s, 2), [[1, 3]])
+    np.testing.assert_array_equal(oracle.select_top_k(s, 4), [[1, 2, 3, 4]])
+
+
+def test_select_decides_in_float32():
+    # 0.5 and 0.5 + 1e-12 are the same float32: a tie, so the lower index wins.
+    s = np.array([[0.5, 0.5 + 1e-12, 0.1]])
+    np.testing.assert_array_equal(oracle.select_top_k(s, 1), [[0]])
+    # 0.5 and 0.5 + 1e-6 differ in float32: the larger wins.
+    s = np.array([[0.5, 0.5 + 1e-6, 0.1]])
+    np.testing.assert_array_equal(oracle.select_top_k(s, 1), [[1]])
+
+
+def test_select_edges():
+    s = np.random.default_rng(3).standard_normal((2, 9))
+    assert oracle.select_top_k(s, 0).shape == (2, 0)
+    np.testing.assert_array_equal(oracle.select_top_k(s, 9), [list(range(9))] * 2)
+    with pytest.raises(ValueError):
+        oracle.select_top_k(s, 10)
+
+
+def test_select_recovers_rows_parallel_to_question():
+    # rows built as a positive multiple of q plus tiny noise outrank all others
+    rng = np.random.default_rng(5)
+    D, N, k = 64, 40, 6
+    q = rng.standard_normal((1, D))
+    bank = rng.standard_normal((1, N, D))
+    chosen = [3, 9, 17, 18, 30, 39]
+    for j in chosen:
+        bank[0, j] = rng.uniform(0.5, 3.0) * q[0] + 1e-3 * rng.standard_normal(D)
+    idx, _ = oracle.score_select(q, bank, k)
+    assert idx[0].tolist() == chosen
+
+
+@pytest.mark.parametrize("name", ["tiny", "llama3_8b"])
+def test_selection_matches_planted_set(name):
+    w = WORKLOADS[name]
+    si = selection_inputs(w)
+    idx, scores = oracle.score_select(si.question_emb, si.cme_bank, w.k)
+    np.testing.assert_array_equal(idx, si.planted_idx)
+    # the planted gap at the cut survives float32 rounding of the inputs
+    for b in range(w.B):
+        srt = np.sort(scores[b])[::-1]
+        assert srt[w.k - 1] - srt[w.k] >= 1e-4
+
+
+# ----------------------------------------------------------------------------
+# Tier-2 ring (Section 2.5, bounded two-tier cache)
+# ----------------------------------------------------------------------------
+
+def test_ring_equals_last_w_tokens():
+    rng = np.random.default_rng(21)
+    B, L, H, W, d = 2, 2, 3, 5, 4
+    fill = [2, 5]
+    ring_k = np.zeros((B, L, H, W, d))
+    ring_v = np.zeros((B, L, H, W, d))
+    hist_k = [[] for _ in range(B)]
+    hist_v = [[] for _ in range(B)]
+    pos = np.zeros(B, dtype=np.int64)
+    for b in range(B):
+        for t in range(fill[b]):
+            kt = rng.standard_normal((L, H, d))
+            vt = rng.standard_normal((L, H, d))
+            ring_k[b, :, :, t] = kt
+            ring_v[b, :, :, t] = vt
+            hist_k[b].append(kt)
+            hist_v[b].append(vt)
+        pos[b] = fill[b]
+    for step in range(13):
+        kn = rng.standard_normal((B, L, H, d))
+        vn = rng.standard_normal((B, L, H, d))
+        before = pos.copy()
+        oracle.window_append(ring_k, ring_v, pos, kn, vn)
+        np.testing.assert_array_equal(pos, before + 1)
+        for b in range(B):
+            hist_k[b].append(kn[b])
+            hist_v[b].append(vn[b])
+            slots = list(oracle.window_slots(pos[b], W))
+            assert len(slots) == min(len(hist_k[b]), W)
+            got = sorted(ring_k[b, 0, 0, s, 0] for s in slots)
+            want = sorted(x[0, 0, 0] for x in hist_k[b][-W:])
+            assert got == want
+            # token number p sits in slot p mod W
+            p = int(pos[b]) - 1
+            np.testing.assert_array_equal(ring_k[b, :, :, p % W], kn[b])
+
+
+# ----------------------------------------------------------------------------
+# Decode attention over [Tier-1 | Tier-2]
+# ----------------------------------------------------------------------------
+
+def test_attention_closed_forms():
+    d = 2
+    v1 = np.array([1.0, -2.0])
+    v2 = np.array([4.0, 8.0])
+    # logits ln 3 and 0 -> weights 3/4 and 1/4
+    q = np.array([1.0, 0.0])
+    K = np.array([[math.log(3.0), 0.0], [0.0, 0.0]])
+    out = oracle.softmax_attention(q, K, np.stack([v1, v2]), scale=1.0)
+    np.testing.assert_allclose(out, 0.75 * v1 + 0.25 * v2, rtol=0, atol=1e-15)
+    # one key: its value
+    out = oracle.softmax_attention(q, K[:1], v1[None], scale=3.0)
+    np.testing.assert_allclose(out, v1, rtol=0, atol=0)
+    # zero query: the mean of the values
+    rng = np.random.default_rng(2)
+    V = rng.standard_normal((9, d))
+    out = oracle.softmax_attention(np.zeros(d), rng.standard_normal((9, d)), V, scale=1.0)
+    np.testing.assert_allclose(out, V.mean(0), rtol=0, atol=1e-15)
+    # empty cache: zeros
+    assert np.all(oracle.softmax_attention(q, np.zeros((0, d)), np.zeros((0, d)), 1.0) == 0)
+
+
+def test_attention_is_stable_for_large_logits():
+    q = np.array([1.0, 0.0])
+    K = np.array([[2000.0, 0.0], [1000.0, 0.0], [-5.0, 0.0]])
+    V = np.array([[1.0, 2.0], [3.0, 4.0], [5.0, 6.0]])
+    out = oracle.softmax_attention(q, K, V, scale=1.0)
+    np.testing.assert_allclose(out, V[0], rtol=0, atol=0)
+
+
+def _small_problem(seed, B=2, L=2, Hq=6, Hkv=2, d=8, N=11, k=4, W=5, fill=(3, 5)):
+    rng = np.random.default_rng(seed)
+    t1k = rng.standard_normal((B, L, Hkv, N, d))
+    t1v = rng.standard_normal((B, L, Hkv, N, d))
+    q = rng.standard_normal((B, L, Hq, d))
+    idx = np.stack([np.sort(rng.choice(N, size=k, replace=False)) for _ in range(B)])
+    ring_k = np.zeros((B, L, Hkv, W, d))
+    ring_v = np.zeros((B, L, Hkv, W, d))
+    hist = []
+    pos = np.zeros(B, dtype=np.int64)
+    for b in range(B):
+        hk = rng.standard_normal((fill[b], L, Hkv, d))
+        hv = rng.standard_normal((fill[b], L, Hkv, d))
+        ring_k[b, :, :, : fill[b]] = hk.transpose(1, 2, 0, 3)
+        ring_v[b, :, :, : fill[b]] = hv.transpose(1, 2, 0, 3)
+        hist.append(([*hk], [*hv]))
+        pos[b] = fill[b]
+    return dict(q=q, t1k=t1k, t1v=t1v, idx=idx, ring_k=ring_k, ring_v=ring_v, pos=pos,
+                hist=hist, rng=rng)
+
+
+def _sdpa(q, K, V, scale=None):
+    """torch fp64 scaled_dot_product_attention of one query over K, V."""
+    out = F.scaled_dot_product_attention(
+        torch.from_numpy(q)[None, None, None, :], torch.from_numpy(K)[None, None],
+        torch.from_numpy(V)[None, None], scale=scale)
+    return out[0, 0, 0].numpy()
+
+
+def test_two_tier_attention_against_sdpa_with_history():
+    """Keys assembled independently (selected bank rows + the last W tokens of
+    the linear token history, GQA head h -> h // (Hq/Hkv)) and attended by the
+    library routine."""
+    P = _small_problem(31)
+    q, t1k, t1v, idx = P["q"], P["t1k"], P["t1v"], P["idx"]
+    ring_k, ring_v, pos, hist, rng = P["ring_k"], P["ring_v"], P["pos"], P["hist"], P["rng"]
+    B, L, Hq, d = q.shape
+    Hkv, W = ring_k.shape[2], ring_k.shape[3]
+    G = Hq // Hkv
+    for step in range(9):   # crosses the wrap of both sequences
+        kn = rng.standard_normal((B, L, Hkv, d))
+        vn = rng.standard_normal((B, L, Hkv, d))
+        qs = rng.standard_normal((B, L, Hq, d))
+        out = oracle.decode_step(qs, t1k, t1v, idx, ring_k, ring_v, pos, kn, vn)
+        for b in range(B):
+            hist[b][0].append(kn[b])
+            hist[b][1].append(vn[b])
+            lastk = np.stack(hist[b][0][-W:])
+            lastv = np.stack(hist[b][1][-W:])
+            for l in range(L):
+                kv_k = torch.from_numpy(t1k[b, l]).repeat_interleave(G, dim=0).numpy()
+                kv_v = torch.from_numpy(t1v[b, l]).repeat_interleave(G, dim=0).numpy()
+                wk = torch.from_numpy(lastk[:, l]).repeat_interleave(G, dim=1).numpy()
+                wv = torch.from_numpy(lastv[:, l]).repeat_interleave(G, dim=1).numpy()
+                for h in range(Hq):
+                    K = np.concatenate([kv_k[h][idx[b]], wk[:, h]])
+                    V = np.concatenate([kv_v[h][idx[b]], wv[:, h]])
+                    np.testing.assert_allclose(out[b, l, h], _sdpa(qs[b, l, h], K, V),
+                                               rtol=1e-12, atol=1e-12)
+
+
+def test_all_cmes_and_unbounded_window_equal_plain_attention():
+    """k = N and a window that never evicts: the two-tier cache holds every
+    token, so the result is plain attention over [bank | all tokens]."""
+    rng = np.random.default_rng(41)
+    B, L, Hq, Hkv, d, N, W = 1, 1, 4, 2, 16, 9, 32
+    t1k = rng.standard_normal((B, L, Hkv, N, d))
+    t1v = rng.standard_normal((B, L, Hkv, N, d))
+    ring_k = np.zeros((B, L, Hkv, W, d))
+    ring_v = np.zeros((B, L, Hkv, W, d))
+    pos = np.zeros(B, dtype=np.int64)
+    toks_k, toks_v = [], []
+    scores = rng.standard_normal((B, N))
+    idx = oracle.select_top_k(scores, N)
+    np.testing.assert_array_equal(idx[0], np.arange(N))
+    for step in range(20):
+        kn = rng.standard_normal((B, L, Hkv, d))
+        vn = rng.standard_normal((B, L, Hkv, d))
+        qs = rng.standard_normal((B, L, Hq, d)) * 2.0
+        out = oracle.decode_step(qs, t1k, t1v, idx, ring_k, ring_v, pos, kn, vn)
+        toks_k.append(kn[0, 0])
+        toks_v.append(vn[0, 0])
+        for h in range(Hq):
+            g = h // (Hq // Hkv)
+            K = np.concatenate([t1k[0, 0, g], np.stack(toks_k)[:, g]])
+            V = np.concatenate([t1v[0, 0, g], np.stack(toks_v)[:, g]])
+            np.testing.assert_allclose(out[0, 0, h], _sdpa(qs[0, 0, h], K, V),
+                                       rtol=1e-12, atol=1e-12)
+
+
+def test_k_zero_is_window_only_attention():
+    P = _small_problem(51, k=0)
+    q, ring_k, ring_v, pos = P["q"], P["ring_k"], P["ring_v"], P["pos"]
+    out = oracle.two_tier_attention(q, P["t1k"], P["t1v"], None, ring_k, ring_v, pos)
+    out2 = oracle.two_tier_attention(q, P["t1k"], P["t1v"], np.zeros((2, 0), np.int64),
+                                     ring_k, ring_v, pos)
+    np.testing.assert_array_equal(out, out2)
+    B, L, Hq, d = q.shape
+    G = Hq // ring_k.shape[2]
+    for b in range(B):
+        n = int(pos[b])
+        for l in range(L):
+            for h in range(Hq):
+                K = ring_k[b, l, h // G, :n]
+                V = ring_v[b, l, h // G, :n]
+                np.testing.assert_allclose(out[b, l, h], _sdpa(q[b, l, h], K, V),
+                                           rtol=1e-12, atol=1e-12)
+
+
+def test_attention_key_order_and_scale():
+    P = _small_problem(61)
+    q, t1k, t1v, idx = P["q"], P["t1k"], P["t1v"], P["idx"]
+    base = oracle.two_tier_attention(q, t1k, t1v, idx, P["ring_k"], P["ring_v"], P["pos"])
+    # permuting the selected rows or the ring slots leaves the output unchanged
+    rev = idx[:, ::-1].copy()
+    perm_ring_k = P["ring_k"][:, :, :, ::-1].copy()
+    perm_ring_v = P["ring_v"][:, :, :, ::-1].copy()
+    W = P["ring_k"].shape[3]
+    full = np.full_like(P["pos"], W)  # both sequences: all slots visible after reversal
+    out = oracle.two_tier_attention(q, t1k, t1v, rev, P["ring_k"], P["ring_v"], P["pos"])
+    np.testing.assert_allclose(out, base, rtol=1e-13, atol=1e-13)
+    # sequence 1 is full: reversed slots hold the same tokens
+    out = oracle.two_tier_attention(q, t1k, t1v, idx, perm_ring_k, perm_ring_v, full)
+    np.testing.assert_allclose(out[1], base[1], rtol=1e-13, atol=1e-13)
+    # default scale is 1/sqrt(d); an explicit scale s equals the query scaled by s*sqrt(d)
+    d = q.shape[-1]
+    s = 0.37
+    out = oracle.two_tier_attention(q, t1k, t1v, idx, P["ring_k"], P["ring_v"], P["pos"], scale=s)
+    out2 = oracle.two_tier_attention(q * s * math.sqrt(d), t1k, t1v, idx, P["ring_k"],
+                                     P["ring_v"], P["pos"])
+    np.testing.assert_allclose(out, out2, rtol=1e-12, atol=1e-12)
+
+
+def test_new_token_attends_to_itself():
+    B, L, Hq, Hkv, d, W = 1, 1, 2, 1, 4, 3
+    rng = np.random.default_rng(71)
+    ring_k = rng.standard_normal((B, L, Hkv, W, d))
+    ring_v = rng.standard_normal((B, L, Hkv, W, d))
+    pos = np.array([W], dtype=np.int64)
+    kn = np.zeros((B, L, Hkv, d)); kn[..., 0] = 50.0
+    vn = np.full((B, L, Hkv, d), 7.0)
+    q = np.zeros((B, L, Hq, d)); q[..., 0] = 50.0
+    out = oracle.decode_step(q, np.zeros((B, L, Hkv, 1, d)), np.zeros((B, L, Hkv, 1, d)),
+                             None, ring_k, ring_v, pos, kn, vn, scale=1.0)
+    np.testing.assert_allclose(out, 7.0, rtol=0, atol=1e-12)
+
+
+def test_bf16_inputs_are_read_exactly():
+    x = np.array([1.0, -2.5, 3.140625, 1e-3, -65504.0], dtype=np.float32)
+    bits = f32_to_bf16_bits(x)
+    t = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(oracle.bf16_to_f64(bits), t)
