@@ -1,0 +1,532 @@
+#!/usr/bin/env python3
+"""Throughput benchmark of the CMC two-tier decode path on GB300.
+
+Workload: the Llama-3-8B-shaped configuration -- batch 1, 32 layers, 32 query
+/ 8 KV heads, head_dim 128, a bank of 1,024 CMEs of dimension 4,096, top-k 128,
+a 512-token window, 3,000 decode steps.
+
+One benchmark step is one generation round over R independent requests of
+that shape (R = --requests, default 4): each request first runs the Tier-1
+scoring + top-k selection on its own CME bank, then the R requests run their
+3,000 fused decode steps (ring append + two-tier attention over all 32
+layers, one launch per request per step) round-robin.  Each request's KV
+state (84.5 MB read per step) fits in the 129 MB L2 by itself; interleaving R
+requests puts (R-1) x 84.5 MB of other traffic between two steps of the same
+request, so every launch reads its K/V from HBM, as it would inside a real
+decoder whose weights stream through L2 between attention layers.
+
+Reported (one JSON line on rank 0):
+  value          decode tokens/s over the whole job (all ranks), selection
+                 included in the timed region;
+  roofline       the fused decode-step kernel: algorithmic bytes per launch
+                 / average launch time, against the measured HBM copy peak;
+  select_us      Tier-1 score + select per request (two launches), L2-cold;
+  e2e            the same metric through the Python API with host buffers
+                 (question vector, CME bank and every step's q / new K,V
+                 copied in from pinned memory, every step's output copied out);
+  cpu_baseline   the fp64 oracle on the host, on a bounded sample.
+
+`--impl reference` times the fp64 oracle alone on the host cores (the
+reference arm; rank 0 only).
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+# The CPU oracle legs run single-threaded and say so.
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from workloads import WORKLOADS, kv_inputs, selection_inputs, step_inputs  # noqa: E402
+
+METRIC = ("two-tier decode-attn tokens/s and % of 8 TB/s HBM; CME top-k select µs")
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+PROFILE_FILE = os.path.join(ROOT, "profiles", "decode_step_llama3_8b.md")
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2609_25537_gb300", "csrc", f)
+                  for f in ("cmc_attn.cu", "cmc_internal.cuh")]
+
+
+# ----------------------------------------------------------------------------
+# Accounting
+# ----------------------------------------------------------------------------
+
+def decode_step_bytes(B, L, Hq, Hkv, d, k, W) -> int:
+    """Algorithmic HBM bytes of one fused decode step with a full ring:
+    k selected Tier-1 rows and W - 1 old ring rows of K and V read, the new
+    token's K,V read once and written once, q read, out written, idx read."""
+    kv_row = d * 2
+    return (B * L * Hkv * 2 * kv_row * (k + W + 1)
+            + B * L * Hq * d * 2 * 2
+            + B * k * 4)
+
+
+def decode_step_flops(B, L, Hq, d, k, W) -> int:
+    """2 flops per MAC; the paper's MACs_t = 2 n_h d_h n_l L_t (appendix,
+    Attention MACs Analysis) with L_t = k + W cached keys."""
+    return 2 * (2 * B * Hq * d * L * (k + W))
+
+
+def select_bytes(B, N, D, k) -> int:
+    return 4 * B * N * D + 4 * B * D + 4 * B * k
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def profiled_traffic():
+    """DRAM bytes per launch of the fused decode kernel from the committed ncu
+    summary, if it was taken on the current kernel source; else None."""
+    try:
+        txt = open(PROFILE_FILE).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", txt)
+    h = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", txt)
+    if not m or not h or h.group(1) != kernel_source_hash():
+        return None
+    return int(m.group(1))
+
+
+# ----------------------------------------------------------------------------
+# Clock sampling (nvidia-smi during the timed region)
+# ----------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, device: torch.device, interval_ms: int = 100):
+        self.proc = None
+        try:
+            uuid = str(torch.cuda.get_device_properties(device).uuid)
+            if not uuid.startswith("GPU-"):
+                uuid = "GPU-" + uuid
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", uuid, f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", str(interval_ms)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(self.NAMES, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------
+# Distributed plumbing (one process per GPU; replicas only)
+# ----------------------------------------------------------------------------
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------
+# The CPU oracle legs
+# ----------------------------------------------------------------------------
+
+def oracle_sample(w, host_state, seconds: float, min_steps: int = 1):
+    """Times the oracle: one Tier-1 selection, then decode steps until
+    `seconds` have passed.  Returns (decode tokens/s, steps, elapsed)."""
+    import oracle
+    qemb, bank, t1k, t1v, ring_k, ring_v, pos = host_state
+    ring_k, ring_v, pos = ring_k.copy(), ring_v.copy(), pos.copy()
+    t0 = time.perf_counter()
+    idx, _ = oracle.score_select(qemb, bank, w.k)
+    steps = 0
+    while True:
+        st = step_inputs(w, steps)
+        oracle.decode_step(st.q, t1k, t1v, idx, ring_k, ring_v, pos, st.k_new, st.v_new)
+        steps += 1
+        el = time.perf_counter() - t0
+        if steps >= min_steps and el >= seconds:
+            break
+    return steps * w.B / el, steps, el
+
+
+def host_state_for(w):
+    si = selection_inputs(w)
+    kv = kv_inputs(w)
+    return (si.question_emb, si.cme_bank, kv.tier1_k, kv.tier1_v, kv.ring_k, kv.ring_v,
+            kv.pos0)
+
+
+def run_reference(args, w, world, rank):
+    """The reference arm: the fp64 oracle on the host cores, rank 0 only."""
+    if rank != 0:
+        return 0
+    state = host_state_for(w)
+    per_step = args.ref_step_seconds
+    for _ in range(args.warmup):
+        oracle_sample(w, state, 0.0, min_steps=1)
+    t0 = time.perf_counter()
+    tokens = 0
+    for _ in range(args.steps):
+        tps, steps, el = oracle_sample(w, state, per_step, min_steps=1)
+        tokens += steps * w.B
+    elapsed = time.perf_counter() - t0
+    value = tokens / elapsed
+    sample = (f"per step: one Tier-1 selection + ~{per_step:g}s of fused decode steps "
+              f"(all {w.L} layers) of {w.name}; fp64 numpy, 1 thread")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * elapsed / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(w, args.requests),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(w, R):
+    return {
+        "workload": (f"{w.name}: B={w.B} L={w.L} Hq={w.Hq} Hkv={w.Hkv} d={w.d} "
+                     f"N={w.N} D={w.D} k={w.k} W={w.W} T={w.T}"),
+        "requests_round_robin": R,
+        "l2": (f"inputs larger than L2: {R} independent requests interleaved, "
+               f"{R * decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W) / 1e6:.0f} MB "
+               "of KV read per round vs 129 MB L2"),
+        "accumulate": "fp32",
+        "parallelism": "replicas",
+    }
+
+
+# ----------------------------------------------------------------------------
+# The GPU arm
+# ----------------------------------------------------------------------------
+
+class Request:
+    """Device state of one B=1 request of the workload."""
+
+    def __init__(self, w, dev, seed, pool, host_sel=None):
+        import paper_2609_25537_gb300 as cmc
+        g = torch.Generator(device=dev).manual_seed(seed)
+
+        def randn(shape, std):
+            return (torch.randn(shape, generator=g, device=dev, dtype=torch.float32)
+                    * std).to(torch.bfloat16)
+
+        B, L, Hq, Hkv, d = w.B, w.L, w.Hq, w.Hkv, w.d
+        sel = host_sel if host_sel is not None else selection_inputs(w.with_(seed=seed))
+        self.qemb = torch.from_numpy(sel.question_emb).to(dev)
+        self.bank = torch.from_numpy(sel.cme_bank).to(dev)
+        self.host_qemb = sel.question_emb
+        self.host_bank = sel.cme_bank
+        self.t1k = randn((B, L, Hkv, w.N, d), w.kv_std)
+        self.t1v = randn((B, L, Hkv, w.N, d), w.kv_std)
+        self.ring_k = randn((B, L, Hkv, w.W, d), w.kv_std)
+        self.ring_v = randn((B, L, Hkv, w.W, d), w.kv_std)
+        self.pos = torch.full((B,), w.W, dtype=torch.int64, device=dev)
+        self.q = randn((pool, B, L, Hq, d), w.q_std)
+        self.k_new = randn((pool, B, L, Hkv, d), w.kv_std)
+        self.v_new = randn((pool, B, L, Hkv, d), w.kv_std)
+        self.idx = torch.empty((B, w.k), dtype=torch.int32, device=dev)
+        self.out = torch.empty((B, L, Hq, d), dtype=torch.bfloat16, device=dev)
+        self.sel_ws = torch.empty(cmc.score_select_workspace_size(B, w.N), dtype=torch.uint8,
+                                  device=dev)
+        dims = cmc.dims_of(self.out, self.t1k, self.idx, self.ring_k)
+        self.ws = cmc.DecodeWorkspace(dims, dev)
+
+    def select(self):
+        import paper_2609_25537_gb300 as cmc
+        cmc.score_select(self.qemb, self.bank, self.idx.shape[1], idx_out=self.idx,
+                         workspace=self.sel_ws)
+
+    def decode(self, p):
+        import paper_2609_25537_gb300 as cmc
+        cmc.decode_step(self.q[p], self.t1k, self.t1v, self.idx, self.ring_k, self.ring_v,
+                        self.pos, self.k_new[p], self.v_new[p], out=self.out,
+                        workspace=self.ws)
+
+    def host_state(self):
+        def bits(t):
+            return t.view(torch.int16).cpu().numpy().view(np.uint16)
+        return (self.host_qemb, self.host_bank, bits(self.t1k), bits(self.t1v),
+                bits(self.ring_k), bits(self.ring_v), self.pos.cpu().numpy().copy())
+
+
+def run_gpu(args, w, world, rank, local):
+    import paper_2609_25537_gb300 as cmc
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    cmc.lib()  # fails loudly when the library is not built
+
+    R, T, P = args.requests, args.decode_steps, args.pool
+    if T % P:
+        raise SystemExit(f"--decode-steps {T} must be a multiple of --pool {P}")
+    sel0 = selection_inputs(w)
+    reqs = [Request(w, dev, 1000 * w.seed + 100 * rank + r, P,
+                    host_sel=sel0 if r == 0 else None) for r in range(R)]
+    torch.cuda.synchronize(dev)  # state was created on the default stream
+    want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
+    # the oracle's copy of request 0, taken before any kernel of ours touches it
+    cpu_state = reqs[0].host_state() if want_cpu else None
+    stream = torch.cuda.Stream(device=dev)
+
+    # eager warm-up of every kernel before graph capture
+    with torch.cuda.stream(stream):
+        for r in reqs:
+            r.select()
+            r.decode(0)
+    stream.synchronize()
+
+    # one graph = P rounds of R decode launches; replayed T / P times per step
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for p in range(P):
+            for r in reqs:
+                r.decode(p)
+    replays = T // P
+
+    def one_step(ev=None):
+        with torch.cuda.stream(stream):
+            if ev is not None:
+                ev[0].record(stream)
+            for r in reqs:
+                r.select()
+            if ev is not None:
+                ev[1].record(stream)
+            for _ in range(replays):
+                graph.replay()
+            if ev is not None:
+                ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        one_step()
+    stream.synchronize()
+
+    K = args.steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    clocks = ClockSampler(dev) if rank == 0 else None
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for s in range(K):
+        one_step(evs[s])
+    t_end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier(world)
+    clk = clocks.stop() if clocks is not None else None
+
+    elapsed_ms = t_start.elapsed_time(t_end)
+    sel_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    max_ms = max_over_ranks(elapsed_ms, world, dev)
+    tokens = world * K * R * w.B * T
+    value = tokens / (max_ms / 1000.0)
+
+    launches_dec = K * R * T
+    launch_us = 1000.0 * sum(dec_ms) / launches_dec
+    nbytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W)
+    achieved = nbytes / (launch_us * 1e-6) / 1e9
+    peak, peak_kind = measured_peaks()
+    select_us = 1000.0 * statistics.median(sel_ms) / R
+
+    # e2e through the Python API with pinned host buffers
+    e2e = run_e2e(args, w, reqs, dev, stream, world) if not args.no_e2e else None
+
+    # CPU oracle baseline (rank 0, N = 1)
+    cpu = None
+    if want_cpu:
+        tps, steps, el = oracle_sample(w, cpu_state, args.cpu_seconds)
+        cpu = {"value": tps, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": (f"one Tier-1 selection + {steps} fused decode steps (all {w.L} "
+                          f"layers) of {w.name} in {el:.1f}s; fp64 numpy, 1 thread")}
+
+    if rank != 0:
+        return 0
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": K, "warmup": args.warmup, "ms_per_step": max_ms / K,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic", "config": workload_config(w, R),
+        "decode_us_per_launch": launch_us,
+        "hbm_pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
+        "select_us": select_us,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
+                     "kernel": "two_tier_attn_kernel<128,4,fused>",
+                     "bytes_per_launch": nbytes, "traffic": profiled_traffic(),
+                     "flops_per_launch": decode_step_flops(w.B, w.L, w.Hq, w.d, w.k, w.W)},
+        "select_roofline": {"bound": "hbm", "bytes": select_bytes(w.B, w.N, w.D, w.k),
+                            "achieved": select_bytes(w.B, w.N, w.D, w.k) / (select_us * 1e-6)
+                            / 1e9, "unit": "GB/s"},
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "gpu_launches": K * R * (T + 2),
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_e2e(args, w, reqs, dev, stream, world):
+    """Same metric through the public Python API with host buffers: the
+    question vector and CME bank of each request and, every decode step, q and
+    the new token's K,V are copied in from pinned host memory and the output
+    copied back to pinned host memory."""
+    import paper_2609_25537_gb300 as cmc
+    R, T, P = args.requests, args.decode_steps, args.pool
+    steps = max(1, min(args.steps, args.e2e_steps))
+    host = []
+    for r in reqs:
+        h = {
+            "qemb": r.qemb.cpu().pin_memory(), "bank": r.bank.cpu().pin_memory(),
+            "q": r.q.cpu().pin_memory(), "k": r.k_new.cpu().pin_memory(),
+            "v": r.v_new.cpu().pin_memory(),
+            "out": torch.empty((P,) + tuple(r.out.shape), dtype=torch.bfloat16).pin_memory(),
+            "q_d": torch.empty_like(r.q[0]), "k_d": torch.empty_like(r.k_new[0]),
+            "v_d": torch.empty_like(r.v_new[0]),
+        }
+        host.append(h)
+
+    def step():
+        with torch.cuda.stream(stream):
+            for r, h in zip(reqs, host):
+                r.qemb.copy_(h["qemb"], non_blocking=True)
+                r.bank.copy_(h["bank"], non_blocking=True)
+                cmc.score_select(r.qemb, r.bank, w.k, idx_out=r.idx, workspace=r.sel_ws)
+            for t in range(T):
+                p = t % P
+                for r, h in zip(reqs, host):
+                    h["q_d"].copy_(h["q"][p], non_blocking=True)
+                    h["k_d"].copy_(h["k"][p], non_blocking=True)
+                    h["v_d"].copy_(h["v"][p], non_blocking=True)
+                    cmc.decode_step(h["q_d"], r.t1k, r.t1v, r.idx, r.ring_k, r.ring_v, r.pos,
+                                    h["k_d"], h["v_d"], out=r.out, workspace=r.ws)
+                    h["out"][p].copy_(r.out, non_blocking=True)
+        stream.synchronize()
+
+    step()  # warm-up
+    barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+    el = time.perf_counter() - t0
+    el = max_over_ranks(el, world, dev)
+    r0 = reqs[0]
+    h2d = R * (r0.qemb.numel() * 4 + r0.bank.numel() * 4
+               + T * 2 * (r0.q[0].numel() + r0.k_new[0].numel() + r0.v_new[0].numel()))
+    d2h = R * T * r0.out.numel() * 2
+    return {"value": world * steps * R * w.B * T / el, "unit": "tokens/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("cmc", "reference"), default="cmc")
+    ap.add_argument("--workload", default="llama3_8b", choices=sorted(WORKLOADS))
+    ap.add_argument("--requests", type=int, default=4)
+    ap.add_argument("--decode-steps", type=int, default=None)
+    ap.add_argument("--pool", type=int, default=8)
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--ref-step-seconds", type=float, default=2.0)
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    w = WORKLOADS[args.workload]
+    if args.decode_steps is None:
+        args.decode_steps = w.T
+    world, rank, local = dist_setup() if args.impl == "cmc" else (
+        int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")), 0)
+    if world != args.gpus and rank == 0:
+        print(f"warning: --gpus {args.gpus} but WORLD_SIZE {world}", file=sys.stderr)
+    if args.impl == "reference":
+        return run_reference(args, w, world, rank)
+    return run_gpu(args, w, world, rank, local)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,191 @@
+/*
+ * cmc.h -- C ABI of the CMC two-tier KV-cache decode path (GB300, sm_103a).
+ *
+ * The method (Section 2.5 of "Compressing Long Context into Answer-Aligned
+ * Memory Embeddings for LLM Inference", "Inference with Two-Tier KV Cache
+ * Policy") keeps, for every sequence, a KV cache of two tiers:
+ *
+ *   Tier-1  the K Context Memory Embeddings (CMEs) whose cosine similarity to
+ *           the mean-pooled question vector is highest, re-ordered by
+ *           document position (the score_j equation and the top-K text that
+ *           follows it);
+ *   Tier-2  a local window of W tokens at full resolution; generated tokens
+ *           enter it, so the cache never exceeds K + W + |q| tokens ("KV
+ *           cache assembly").
+ *
+ * Each decode step attends over [Tier-1 | Tier-2]; the appendix ("Attention
+ * MACs Analysis") costs it as MACs_t = 2 n_h d_h n_l L_t.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every tensor argument is a DEVICE pointer to memory the caller owns.  The
+ *    library allocates no memory and keeps no state between calls apart from
+ *    the thread-local last CUDA error and a per-device SM-count cache.
+ *  - All work is enqueued on `stream` (a cudaStream_t passed as void*; NULL is
+ *    the legacy default stream) and is asynchronous: a return of CMC_OK means
+ *    the launch was accepted, not that it has finished.
+ *  - Tensors are dense, row-major, with the shapes given below (last index
+ *    fastest).  bf16 tensors must be 16-byte aligned; so must fp32 tensors.
+ *  - Arguments are checked on the host before any launch; a failed check
+ *    launches nothing and returns the status below.  Kernels never trap.
+ *  - Calls that share a workspace must be ordered on one stream.
+ */
+#ifndef CMC_H_
+#define CMC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define CMC_API __attribute__((visibility("default")))
+#else
+#define CMC_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum cmc_status {
+  CMC_OK = 0,
+  CMC_ERR_NULL = 1,      /* a required pointer is NULL                              */
+  CMC_ERR_SHAPE = 2,     /* a size outside the supported range (see each call)      */
+  CMC_ERR_RANGE = 3,     /* an index-like argument out of range (k > N, W < 1, ...) */
+  CMC_ERR_ALIGN = 4,     /* a tensor pointer is not 16-byte aligned                 */
+  CMC_ERR_WORKSPACE = 5, /* workspace NULL or smaller than the size query returns   */
+  CMC_ERR_CUDA = 6       /* a CUDA call failed; cmc_last_cuda_error() has the code  */
+} cmc_status;
+
+/* Device-side status bits, accumulated in a workspace's status word (see
+ * cmc_read_status).  Kernels skip the offending element and carry on. */
+#define CMC_DEVFLAG_BAD_INDEX 1u /* an idx entry outside [0, N): that row was skipped   */
+#define CMC_DEVFLAG_BAD_POS 2u   /* a negative pos: that sequence was skipped            */
+
+/* Shapes of one decode problem. */
+typedef struct cmc_dims {
+  int32_t B;   /* sequences, >= 1                                                  */
+  int32_t L;   /* decoder layers handled by one call, >= 1                         */
+  int32_t Hq;  /* query heads, >= 1                                                */
+  int32_t Hkv; /* KV heads; Hq % Hkv == 0 and Hq / Hkv in {1, 2, 4, 8}             */
+  int32_t d;   /* head dimension: 64 or 128                                        */
+  int32_t N;   /* rows of the Tier-1 K/V bank per (sequence, layer, KV head), >= 1 */
+  int32_t k;   /* selected Tier-1 rows per sequence, 0 <= k <= N                   */
+  int32_t W;   /* Tier-2 ring capacity in tokens, >= 1                             */
+} cmc_dims;
+
+/* Human-readable name of a cmc_status value (static storage). */
+CMC_API const char* cmc_status_string(int status);
+
+/* cudaError_t of the most recent failed CUDA call made by this library on the
+ * calling thread; 0 if none.  Reading it clears it. */
+CMC_API int cmc_last_cuda_error(void);
+
+/* ------------------------------------------------------------------------ *
+ * Tier-1: question-guided scoring and top-K selection                       *
+ * (Section 2.5, the score_j equation and the top-K re-ordering after it)    *
+ * ------------------------------------------------------------------------ */
+
+/* Bytes of workspace cmc_score_select needs for B sequences of N CMEs. */
+CMC_API size_t cmc_score_select_workspace_size(int B, int N);
+
+/*
+ * For each sequence b, scores every CME j by cosine similarity
+ *     score[b, j] = (m_j . q_b) / (||m_j|| ||q_b||)
+ * and writes the k indices with the highest scores, in ascending index order
+ * (document order), to idx_out[b, 0..k).
+ *
+ *   question_emb  fp32 [B, D]       the question vectors q_vec
+ *   cme_bank      fp32 [B, N, D]    the decoder-ready CMEs m_j of each sequence
+ *   idx_out       int32 [B, k]      output, ascending within each row
+ *   scores_out    fp32 [B, N]       optional output (NULL: not written)
+ *   workspace     >= cmc_score_select_workspace_size(B, N) bytes, any content
+ *
+ * Scores are computed in fp32 with a fixed summation order, so equal rows get
+ * bit-identical scores.  Equal scores go to the lower index; -0 equals +0.  A
+ * zero-norm CME or question vector scores 0.  Non-finite inputs are outside
+ * the contract (no fault, unspecified selection).
+ * Limits: 1 <= B <= 65535, 1 <= N <= 1048576, 4 <= D <= 65536, D % 4 == 0,
+ * 0 <= k <= N.
+ */
+CMC_API int cmc_score_select(const float* question_emb, const float* cme_bank, int B, int N, int D,
+                             int k, int32_t* idx_out, float* scores_out, void* workspace,
+                             size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------ *
+ * Tier-2: local-window ring append (Section 2.5, Tier-2 and the K + W + |q| *
+ * bound of "KV cache assembly")                                             *
+ * ------------------------------------------------------------------------ */
+
+/*
+ * Appends one token per sequence to the ring.  Token number pos[b] (counting
+ * from 0) is written to slot pos[b] mod W of every (layer, KV head); once more
+ * than W tokens have been appended this overwrites the oldest one.  pos[b] is
+ * then incremented on the device.
+ *
+ *   ring_k, ring_v  bf16 [B, L, Hkv, W, d]   updated in place
+ *   pos             int64 [B]                tokens appended so far; updated
+ *   k_new, v_new    bf16 [B, L, Hkv, d]      the new token's keys and values
+ *
+ * dims->Hq, N and k are ignored.  A sequence with pos[b] < 0 is left unchanged.
+ */
+CMC_API int cmc_window_append(void* ring_k, void* ring_v, int64_t* pos, const void* k_new,
+                              const void* v_new, const cmc_dims* dims, void* stream);
+
+/* ------------------------------------------------------------------------ *
+ * Decode attention over [Tier-1 | Tier-2]                                   *
+ * (Section 2.5 "KV cache assembly"; cost model in "Attention MACs Analysis")*
+ * ------------------------------------------------------------------------ */
+
+/* Bytes of workspace the two attention entry points need for `dims`.  The
+ * workspace must be zero-filled once before its first use; every call leaves
+ * its counters at zero again. */
+CMC_API size_t cmc_decode_attn_workspace_size(const cmc_dims* dims);
+
+/*
+ * For every sequence b, layer l and query head h (KV head g = h / (Hq/Hkv)):
+ *     out[b,l,h] = sum_i softmax_i(scale * q[b,l,h] . key_i) value_i
+ * over the keys of
+ *     Tier-1: tier1_k[b,l,g, idx[b,i]] for i < k (gathered by index), then
+ *     Tier-2: ring_k[b,l,g, s] for the occupied slots s < min(pos[b], W).
+ * An empty cache gives a zero output.
+ *
+ *   q                 bf16 [B, L, Hq, d]
+ *   tier1_k, tier1_v  bf16 [B, L, Hkv, N, d]
+ *   idx               int32 [B, k]   (may be NULL when k == 0); any order
+ *   ring_k, ring_v    bf16 [B, L, Hkv, W, d]
+ *   pos               int64 [B]      tokens appended so far (read only)
+ *   scale             softmax scale; <= 0 selects 1/sqrt(d)
+ *   out               bf16 [B, L, Hq, d]  (round to nearest even)
+ *   workspace         see cmc_decode_attn_workspace_size
+ *
+ * Accumulation is fp32.  idx entries outside [0, N) are skipped and flagged
+ * with CMC_DEVFLAG_BAD_INDEX.  A sequence with pos[b] < 0 gets a zero output
+ * and sets CMC_DEVFLAG_BAD_POS.
+ */
+CMC_API int cmc_two_tier_decode_attn(const void* q, const void* tier1_k, const void* tier1_v,
+                                     const int32_t* idx, const void* ring_k, const void* ring_v,
+                                     const int64_t* pos, const cmc_dims* dims, float scale, void* out,
+                                     void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * One fused decode step: cmc_window_append followed by
+ * cmc_two_tier_decode_attn, in one launch.  The new token is appended before
+ * attention, so it attends to itself.  On return (in stream order) the ring
+ * holds the new token at slot pos[b] mod W and pos[b] has grown by one.
+ * Arguments are those of the two calls it fuses.  A sequence with pos[b] < 0
+ * is left unchanged, its output is zero and CMC_DEVFLAG_BAD_POS is set.
+ */
+CMC_API int cmc_decode_step(const void* q, const void* tier1_k, const void* tier1_v,
+                            const int32_t* idx, void* ring_k, void* ring_v, int64_t* pos,
+                            const void* k_new, const void* v_new, const cmc_dims* dims, float scale,
+                            void* out, void* workspace, size_t workspace_bytes, void* stream);
+
+/* Copies the device status word of an attention workspace (CMC_DEVFLAG_*
+ * bits) into *flags, waiting for `stream`, and clears it when `clear` != 0. */
+CMC_API int cmc_read_status(void* workspace, int clear, uint32_t* flags, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CMC_H_ */

@@ -71,13 +71,13 @@ def cosine_scores(question_emb: np.ndarray, cme_bank: np.ndarray) -> np.ndarray:
     A zero-norm CME or question vector gives score 0.
     """
     q = np.asarray(question_emb, dtype=np.float64)
-    m = np.asarray(cme_bank, dtype=np.float64)
+    m = np.asarray(cme_bank)
     B, N, D = m.shape
     out = np.zeros((B, N), dtype=np.float64)
     for b in range(B):
         qn = math.sqrt(float(q[b] @ q[b]))
         for j0 in range(0, N, 4096):
-            rows = m[b, j0:j0 + 4096]
+            rows = m[b, j0:j0 + 4096].astype(np.float64)
             dots = rows @ q[b]
             mn = np.sqrt(np.einsum("ij,ij->i", rows, rows))
             den = mn * qn

@@ -1,0 +1,247 @@
+"""Python binding of libcmc: the CMC two-tier decode path on GB300.
+
+Argument marshalling only.  Each function checks the tensors it is given
+(device, dtype, contiguity, shapes), derives the sizes, and calls the C ABI
+with raw device pointers and the current torch CUDA stream.  Every step of the
+computation runs in the library's CUDA kernels; there is no CPU path.
+
+Tensor layouts (row-major, last index fastest):
+
+  question_emb  fp32 [B, D]            cme_bank  fp32 [B, N, D]
+  q             bf16 [B, L, Hq, d]     out       bf16 [B, L, Hq, d]
+  tier1_k/v     bf16 [B, L, Hkv, N, d] idx       int32 [B, k]
+  ring_k/v      bf16 [B, L, Hkv, W, d] pos       int64 [B]
+  k_new/v_new   bf16 [B, L, Hkv, d]
+"""
+
+from __future__ import annotations
+
+import ctypes
+import math
+from typing import Dict, Optional, Tuple
+
+import torch
+
+from ._lib import CmcDims, check, lib, DEVFLAG_BAD_INDEX, DEVFLAG_BAD_POS
+
+__all__ = [
+    "CmcDims",
+    "DecodeWorkspace",
+    "score_select",
+    "score_select_workspace_size",
+    "window_append",
+    "two_tier_decode_attn",
+    "decode_step",
+    "decode_attn_workspace_size",
+    "dims_of",
+    "DEVFLAG_BAD_INDEX",
+    "DEVFLAG_BAD_POS",
+]
+
+
+def _p(t: Optional[torch.Tensor]) -> ctypes.c_void_p:
+    return ctypes.c_void_p(0 if t is None else t.data_ptr())
+
+
+def _stream(device: torch.device) -> ctypes.c_void_p:
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _need(t: torch.Tensor, name: str, dtype: torch.dtype, ndim: int, device=None) -> None:
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor (the library has no CPU path)")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got shape {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+
+
+# ----------------------------------------------------------------------------
+# Tier-1: scoring and selection
+# ----------------------------------------------------------------------------
+
+def score_select_workspace_size(B: int, N: int) -> int:
+    return int(lib().cmc_score_select_workspace_size(B, N))
+
+
+def score_select(question_emb: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
+                 idx_out: Optional[torch.Tensor] = None,
+                 scores_out: Optional[torch.Tensor] = None,
+                 workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Top-k CMEs by cosine similarity to the question vector, as int32 [B, k]
+    indices in ascending (document) order.  See cmc_score_select."""
+    _need(cme_bank, "cme_bank", torch.float32, 3)
+    dev = cme_bank.device
+    _need(question_emb, "question_emb", torch.float32, 2, dev)
+    B, N, D = cme_bank.shape
+    if tuple(question_emb.shape) != (B, D):
+        raise ValueError(f"question_emb shape {tuple(question_emb.shape)} != {(B, D)}")
+    if idx_out is None:
+        idx_out = torch.empty((B, k), dtype=torch.int32, device=dev)
+    _need(idx_out, "idx_out", torch.int32, 2, dev)
+    if tuple(idx_out.shape) != (B, k):
+        raise ValueError(f"idx_out shape {tuple(idx_out.shape)} != {(B, k)}")
+    if scores_out is not None:
+        _need(scores_out, "scores_out", torch.float32, 2, dev)
+        if tuple(scores_out.shape) != (B, N):
+            raise ValueError(f"scores_out shape {tuple(scores_out.shape)} != {(B, N)}")
+    ws_bytes = 0
+    if scores_out is None:
+        need = score_select_workspace_size(B, N)
+        if workspace is None:
+            workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+        ws_bytes = workspace.numel() * workspace.element_size()
+    st = lib().cmc_score_select(_p(question_emb), _p(cme_bank), B, N, D, k, _p(idx_out),
+                                _p(scores_out), _p(workspace), ws_bytes, _stream(dev))
+    check(st, "cmc_score_select")
+    return idx_out
+
+
+# ----------------------------------------------------------------------------
+# Decode attention
+# ----------------------------------------------------------------------------
+
+def dims_of(q: torch.Tensor, tier1_k: torch.Tensor, idx: Optional[torch.Tensor],
+            ring_k: torch.Tensor) -> CmcDims:
+    B, L, Hq, d = q.shape
+    Bk, Lk, Hkv, N, dk = tier1_k.shape
+    Br, Lr, Hr, W, dr = ring_k.shape
+    k = 0 if idx is None else int(idx.shape[1])
+    if (Bk, Lk, dk) != (B, L, d) or (Br, Lr, Hr, dr) != (B, L, Hkv, d):
+        raise ValueError(f"inconsistent shapes: q {tuple(q.shape)}, tier1 {tuple(tier1_k.shape)}, "
+                         f"ring {tuple(ring_k.shape)}")
+    if idx is not None and int(idx.shape[0]) != B:
+        raise ValueError(f"idx shape {tuple(idx.shape)} does not match batch {B}")
+    return CmcDims(B, L, Hq, Hkv, d, N, k, W)
+
+
+def decode_attn_workspace_size(dims: CmcDims) -> int:
+    return int(lib().cmc_decode_attn_workspace_size(ctypes.byref(dims)))
+
+
+class DecodeWorkspace:
+    """Zero-filled device workspace for the attention entry points.
+
+    Holds the split-K partials, the arrival tickets and the device status word.
+    Calls sharing one workspace must be ordered on one stream."""
+
+    def __init__(self, dims: CmcDims, device: torch.device):
+        n = decode_attn_workspace_size(dims)
+        if n == 0:
+            raise ValueError(f"unsupported dims {dims.key()}")
+        self.dims = dims
+        self.nbytes = n
+        self.buf = torch.zeros(n, dtype=torch.uint8, device=device)
+
+    def status(self, clear: bool = True) -> int:
+        """CMC_DEVFLAG_* bits raised by kernels since the last clear (synchronises)."""
+        flags = ctypes.c_uint32(0)
+        st = lib().cmc_read_status(_p(self.buf), 1 if clear else 0, ctypes.byref(flags),
+                                   _stream(self.buf.device))
+        check(st, "cmc_read_status")
+        return int(flags.value)
+
+
+_ws_cache: Dict[Tuple, DecodeWorkspace] = {}
+
+
+def _workspace_for(dims: CmcDims, device: torch.device) -> DecodeWorkspace:
+    key = (device.index, torch.cuda.current_stream(device).cuda_stream, dims.key())
+    ws = _ws_cache.get(key)
+    if ws is None:
+        ws = DecodeWorkspace(dims, device)
+        _ws_cache[key] = ws
+    return ws
+
+
+def _attn_args(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, out):
+    _need(q, "q", torch.bfloat16, 4)
+    dev = q.device
+    _need(tier1_k, "tier1_k", torch.bfloat16, 5, dev)
+    _need(tier1_v, "tier1_v", torch.bfloat16, 5, dev)
+    _need(ring_k, "ring_k", torch.bfloat16, 5, dev)
+    _need(ring_v, "ring_v", torch.bfloat16, 5, dev)
+    _need(pos, "pos", torch.int64, 1, dev)
+    if idx is not None:
+        _need(idx, "idx", torch.int32, 2, dev)
+    if tier1_v.shape != tier1_k.shape or ring_v.shape != ring_k.shape:
+        raise ValueError("K and V tensors must have the same shapes")
+    dims = dims_of(q, tier1_k, idx, ring_k)
+    if int(pos.shape[0]) != dims.B:
+        raise ValueError(f"pos shape {tuple(pos.shape)} does not match batch {dims.B}")
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16, 4, dev)
+    if out.shape != q.shape:
+        raise ValueError("out must have the shape of q")
+    return dims, dev, out
+
+
+def _scale(scale: Optional[float]) -> float:
+    return 0.0 if scale is None else float(scale)
+
+
+def two_tier_decode_attn(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, *,
+                         scale: Optional[float] = None, out: Optional[torch.Tensor] = None,
+                         workspace: Optional[DecodeWorkspace] = None) -> torch.Tensor:
+    """Decode attention over [Tier-1 rows at idx | occupied ring slots]; see
+    cmc_two_tier_decode_attn.  Returns bf16 [B, L, Hq, d]."""
+    dims, dev, out = _attn_args(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, out)
+    ws = workspace if workspace is not None else _workspace_for(dims, dev)
+    st = lib().cmc_two_tier_decode_attn(
+        _p(q), _p(tier1_k), _p(tier1_v), _p(idx), _p(ring_k), _p(ring_v), _p(pos),
+        ctypes.byref(dims), _scale(scale), _p(out), _p(ws.buf), ws.nbytes, _stream(dev))
+    check(st, "cmc_two_tier_decode_attn")
+    return out
+
+
+def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, *,
+                scale: Optional[float] = None, out: Optional[torch.Tensor] = None,
+                workspace: Optional[DecodeWorkspace] = None) -> torch.Tensor:
+    """Fused decode step: append (k_new, v_new) to the ring, then attend; see
+    cmc_decode_step.  Updates ring_k, ring_v and pos in place."""
+    dims, dev, out = _attn_args(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, out)
+    _need(k_new, "k_new", torch.bfloat16, 4, dev)
+    _need(v_new, "v_new", torch.bfloat16, 4, dev)
+    want = (dims.B, dims.L, dims.Hkv, dims.d)
+    if tuple(k_new.shape) != want or tuple(v_new.shape) != want:
+        raise ValueError(f"k_new/v_new must be {want}")
+    ws = workspace if workspace is not None else _workspace_for(dims, dev)
+    st = lib().cmc_decode_step(
+        _p(q), _p(tier1_k), _p(tier1_v), _p(idx), _p(ring_k), _p(ring_v), _p(pos),
+        _p(k_new), _p(v_new), ctypes.byref(dims), _scale(scale), _p(out), _p(ws.buf),
+        ws.nbytes, _stream(dev))
+    check(st, "cmc_decode_step")
+    return out
+
+
+def window_append(ring_k: torch.Tensor, ring_v: torch.Tensor, pos: torch.Tensor,
+                  k_new: torch.Tensor, v_new: torch.Tensor) -> None:
+    """Append one token per sequence to the Tier-2 ring; see cmc_window_append."""
+    _need(ring_k, "ring_k", torch.bfloat16, 5)
+    dev = ring_k.device
+    _need(ring_v, "ring_v", torch.bfloat16, 5, dev)
+    _need(pos, "pos", torch.int64, 1, dev)
+    _need(k_new, "k_new", torch.bfloat16, 4, dev)
+    _need(v_new, "v_new", torch.bfloat16, 4, dev)
+    B, L, Hkv, W, d = ring_k.shape
+    if ring_v.shape != ring_k.shape:
+        raise ValueError("ring_v must have the shape of ring_k")
+    if tuple(k_new.shape) != (B, L, Hkv, d) or tuple(v_new.shape) != (B, L, Hkv, d):
+        raise ValueError(f"k_new/v_new must be {(B, L, Hkv, d)}")
+    if int(pos.shape[0]) != B:
+        raise ValueError("pos must be [B]")
+    dims = CmcDims(B, L, Hkv, Hkv, d, 1, 0, W)
+    st = lib().cmc_window_append(_p(ring_k), _p(ring_v), _p(pos), _p(k_new), _p(v_new),
+                                 ctypes.byref(dims), _stream(dev))
+    check(st, "cmc_window_append")
+
+
+def default_scale(d: int) -> float:
+    return 1.0 / math.sqrt(d)

@@ -1,0 +1,154 @@
+"""The C ABI on the host: the library builds, loads and exports every symbol
+include/cmc.h declares; argument checks fail with the documented status
+before any CUDA call; workspace-size queries follow their formulas.  None of
+these tests launches a kernel, so they run without a GPU."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2609_25537_gb300 as cmc
+from paper_2609_25537_gb300 import _lib
+from paper_2609_25537_gb300.build import build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "cmc.h")
+
+OK, NULL, SHAPE, RANGE, ALIGN, WORKSPACE = 0, 1, 2, 3, 4, 5
+
+
+@pytest.fixture(scope="module")
+def L():
+    build()
+    return cmc.lib()
+
+
+def _declared():
+    src = open(HEADER).read()
+    return re.findall(r"CMC_API\s+[\w\s\*]+?\b(cmc_\w+)\s*\(", src)
+
+
+def test_header_and_binding_agree():
+    names = _declared()
+    assert len(names) == len(set(names)) and names
+    assert set(names) == set(_lib.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in _declared():
+        assert hasattr(L, name), name
+
+
+def test_status_strings(L):
+    for code in range(7):
+        s = L.cmc_status_string(code).decode()
+        assert s.startswith(_lib.STATUS[code])
+    assert L.cmc_last_cuda_error() == 0
+
+
+FAKE = 0x10000  # 16-byte aligned, never dereferenced: these calls fail before any launch
+
+# The fake-pointer checks run only where no GPU is visible, so that a bug in
+# the argument checks can never launch a kernel on fake pointers.
+import torch  # noqa: E402
+
+host_only = pytest.mark.skipif(torch.cuda.is_available(),
+                               reason="fake-pointer argument checks run only without a GPU")
+
+
+def _sel(L, qe=FAKE, bank=FAKE, B=2, N=64, D=16, k=8, idx=FAKE, scores=0, ws=FAKE, wsb=1 << 20):
+    return L.cmc_score_select(qe, bank, B, N, D, k, idx, scores, ws, wsb, None)
+
+
+@host_only
+def test_score_select_argument_checks(L):
+    assert _sel(L, B=0) == SHAPE
+    assert _sel(L, N=0) == SHAPE
+    assert _sel(L, D=6) == SHAPE
+    assert _sel(L, D=0) == SHAPE
+    assert _sel(L, k=65) == RANGE
+    assert _sel(L, k=-1) == RANGE
+    assert _sel(L, qe=0) == NULL
+    assert _sel(L, bank=0) == NULL
+    assert _sel(L, idx=0) == NULL
+    assert _sel(L, bank=FAKE + 4) == ALIGN
+    assert _sel(L, ws=0) == WORKSPACE
+    assert _sel(L, wsb=2 * 64 * 4 - 1) == WORKSPACE
+
+
+def test_score_select_workspace_size(L):
+    assert L.cmc_score_select_workspace_size(3, 100) == 1280  # 1200 rounded up to 256
+    assert L.cmc_score_select_workspace_size(0, 100) == 0
+
+
+def _dims(**kw):
+    base = dict(B=2, L=3, Hq=8, Hkv=2, d=128, N=100, k=10, W=16)
+    base.update(kw)
+    return cmc.CmcDims(*(base[f] for f, _ in cmc.CmcDims._fields_))
+
+
+def _attn(L, dims, q=FAKE, idx=FAKE, ws=FAKE, wsb=1 << 30, out=FAKE, pos=FAKE):
+    return L.cmc_two_tier_decode_attn(q, FAKE, FAKE, idx, FAKE, FAKE, pos, ctypes.byref(dims),
+                                      0.0, out, ws, wsb, None)
+
+
+def _step(L, dims, k_new=FAKE, ws=FAKE, wsb=1 << 30):
+    return L.cmc_decode_step(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, k_new, FAKE,
+                             ctypes.byref(dims), 0.0, FAKE, ws, wsb, None)
+
+
+@host_only
+def test_attention_argument_checks(L):
+    assert _attn(L, _dims(d=96)) == SHAPE
+    assert _attn(L, _dims(Hq=6)) == SHAPE          # Hq % Hkv != 0
+    assert _attn(L, _dims(Hq=32, Hkv=2)) == SHAPE  # G = 16 unsupported
+    assert _attn(L, _dims(B=0)) == SHAPE
+    assert _attn(L, _dims(W=0)) == SHAPE
+    assert _attn(L, _dims(k=101)) == RANGE
+    assert _attn(L, _dims(k=-1)) == RANGE
+    assert _attn(L, _dims(), q=0) == NULL
+    assert _attn(L, _dims(), idx=0) == NULL
+    assert _attn(L, _dims(), out=0) == NULL
+    assert _attn(L, _dims(), q=FAKE + 2) == ALIGN
+    assert _attn(L, _dims(), pos=FAKE + 4) == ALIGN
+    assert _attn(L, _dims(), ws=0) == WORKSPACE
+    assert _attn(L, _dims(), wsb=16) == WORKSPACE
+    assert _step(L, _dims(), k_new=0) == NULL
+    assert _step(L, _dims(), k_new=FAKE + 8) == ALIGN
+    assert _step(L, _dims(), wsb=16) == WORKSPACE
+    assert L.cmc_two_tier_decode_attn(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, 0.0, FAKE,
+                                      FAKE, 1 << 30, None) == NULL
+
+
+@host_only
+def test_window_append_argument_checks(L):
+    d = _dims()
+    assert L.cmc_window_append(0, FAKE, FAKE, FAKE, FAKE, ctypes.byref(d), None) == NULL
+    assert L.cmc_window_append(FAKE, FAKE, FAKE + 4, FAKE, FAKE, ctypes.byref(d), None) == ALIGN
+    assert L.cmc_window_append(FAKE, FAKE, FAKE, FAKE, FAKE, ctypes.byref(_dims(d=32)),
+                               None) == SHAPE
+
+
+def test_attention_workspace_size(L):
+    d = _dims()
+    n = L.cmc_decode_attn_workspace_size(ctypes.byref(d))
+    units = 2 * 3 * 2
+    smax = -(-(10 + 16) // 32)
+    G = 4
+    tickets = -(-(4 * (units + 2)) // 256) * 256
+    assert n == 256 + tickets + units * smax * G * (128 + 2) * 4
+    assert L.cmc_decode_attn_workspace_size(ctypes.byref(_dims(d=80))) == 0
+
+
+@host_only
+def test_read_status_checks(L):
+    flags = ctypes.c_uint32(0)
+    assert L.cmc_read_status(0, 0, ctypes.byref(flags), None) == NULL
+
+
+def test_binding_rejects_cpu_tensors():
+    import torch
+    with pytest.raises(ValueError, match="CUDA"):
+        cmc.score_select(torch.zeros(1, 8), torch.zeros(1, 4, 8), 2)

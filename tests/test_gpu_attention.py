@@ -1,0 +1,306 @@
+"""Two-tier decode attention (and the ring append) on the GPU against the fp64
+oracle, on the seeded workloads and on edge cases.
+
+Full-size workloads run every decode step on the GPU and compare every head
+of every layer at sampled steps (first steps, around the ring's wrap, middle,
+last), with the oracle replaying the same appends."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_25537_gb300 as cmc
+from workloads import (WORKLOADS, kv_inputs, random_tier1_indices, selection_inputs,
+                       step_inputs)
+from workloads.configs import ablation_workloads, full_window_workload
+from _gpu_helpers import assert_attn_close, dev_bf16, host_bits, to_f64
+
+pytestmark = pytest.mark.gpu
+
+
+class Problem:
+    """Device and host (oracle) copies of one decode problem."""
+
+    def __init__(self, w, dev, idx=None):
+        self.w = w
+        self.dev = dev
+        kv = kv_inputs(w)
+        self.kv = kv
+        if idx is None and w.k > 0:
+            idx = random_tier1_indices(w)
+        self.idx_host = None if w.k == 0 else np.asarray(idx, dtype=np.int64)
+        self.idx = None if w.k == 0 else torch.from_numpy(
+            np.asarray(idx, dtype=np.int32)).to(dev)
+        self.t1k, self.t1v = dev_bf16(kv.tier1_k, dev), dev_bf16(kv.tier1_v, dev)
+        self.ring_k, self.ring_v = dev_bf16(kv.ring_k, dev), dev_bf16(kv.ring_v, dev)
+        self.pos = torch.from_numpy(kv.pos0.copy()).to(dev)
+        self.o_ring_k, self.o_ring_v = kv.ring_k.copy(), kv.ring_v.copy()
+        self.o_pos = kv.pos0.copy()
+        dims = cmc.dims_of(torch.empty(w.B, w.L, w.Hq, w.d, dtype=torch.bfloat16),
+                           torch.empty(w.B, w.L, w.Hkv, w.N, w.d, dtype=torch.bfloat16),
+                           self.idx, torch.empty(w.B, w.L, w.Hkv, w.W, w.d,
+                                                 dtype=torch.bfloat16))
+        self.ws = cmc.DecodeWorkspace(dims, dev)
+
+    def step(self, st, q_dev=None, compare=True, scale=None):
+        q_dev = dev_bf16(st.q, self.dev) if q_dev is None else q_dev
+        out = cmc.decode_step(q_dev, self.t1k, self.t1v, self.idx, self.ring_k, self.ring_v,
+                              self.pos, dev_bf16(st.k_new, self.dev),
+                              dev_bf16(st.v_new, self.dev), workspace=self.ws, scale=scale)
+        if not compare:
+            oracle.window_append(self.o_ring_k, self.o_ring_v, self.o_pos, st.k_new, st.v_new)
+            return out, None
+        ref = oracle.decode_step(st.q, self.kv.tier1_k, self.kv.tier1_v, self.idx_host,
+                                 self.o_ring_k, self.o_ring_v, self.o_pos, st.k_new, st.v_new,
+                                 scale=scale)
+        return out, ref
+
+    def check_state(self):
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(self.pos.cpu().numpy(), self.o_pos)
+        np.testing.assert_array_equal(host_bits(self.ring_k), self.o_ring_k)
+        np.testing.assert_array_equal(host_bits(self.ring_v), self.o_ring_v)
+        assert self.ws.status() == 0
+
+
+def test_tiny_every_step(cuda_device):
+    w = WORKLOADS["tiny"]
+    si = selection_inputs(w)
+    idx_ref, _ = oracle.score_select(si.question_emb, si.cme_bank, w.k)
+    P = Problem(w, cuda_device, idx=idx_ref)
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t))
+        assert_attn_close(to_f64(out), ref, f"tiny step {t}")
+    P.check_state()
+
+
+@pytest.mark.parametrize("q_scale", [3.0])
+def test_tiny_peaked(cuda_device, q_scale):
+    """Unscaled-style queries: logits with std ~3, so the softmax is peaked."""
+    w = WORKLOADS["tiny"]
+    P = Problem(w, cuda_device)
+    for t in range(4):
+        out, ref = P.step(step_inputs(w, t, q_std=q_scale / w.kv_std))
+        assert_attn_close(to_f64(out), ref, f"tiny peaked step {t}")
+
+
+def _sampled_run(w, dev, sample_steps, idx=None, q_std=None):
+    P = Problem(w, dev, idx=idx)
+    q_fill = dev_bf16(step_inputs(w, 0, parts="q", q_std=q_std).q, dev)
+    sample_steps = set(sample_steps)
+    for t in range(w.T):
+        if t in sample_steps:
+            st = step_inputs(w, t, q_std=q_std)
+            out, ref = P.step(st)
+            assert_attn_close(to_f64(out), ref, f"{w.name} step {t}")
+        else:
+            st = step_inputs(w, t, parts="kv")
+            P.step(st, q_dev=q_fill, compare=False)
+    P.check_state()
+
+
+def _samples(w):
+    return sorted({0, 1, 2, w.W - 1, w.W, w.W + 1, w.T // 2, w.T - 1} & set(range(w.T)))
+
+
+def test_llama3_8b_full(cuda_device):
+    """The 32-layer Llama-3-8B-shaped workload, all 3,000 steps, with the
+    selection taken from the Tier-1 scoring of its own CME bank."""
+    w = WORKLOADS["llama3_8b"]
+    si = selection_inputs(w)
+    idx = cmc.score_select(torch.from_numpy(si.question_emb).to(cuda_device),
+                           torch.from_numpy(si.cme_bank).to(cuda_device), w.k)
+    idx_host = idx.cpu().numpy()
+    np.testing.assert_array_equal(idx_host, oracle.score_select(si.question_emb, si.cme_bank,
+                                                                w.k)[0])
+    _sampled_run(w, cuda_device, _samples(w), idx=idx_host)
+
+
+def test_llama3_8b_peaked(cuda_device):
+    w = WORKLOADS["llama3_8b"].with_(T=3, L=4)
+    _sampled_run(w, cuda_device, range(3), q_std=3.0 / w.kv_std)
+
+
+def test_mistral_batched_full(cuda_device):
+    w = WORKLOADS["mistral_batched"]
+    _sampled_run(w, cuda_device, _samples(w))
+
+
+def test_long_context_full(cuda_device):
+    w = WORKLOADS["long_context"]
+    _sampled_run(w, cuda_device, _samples(w))
+
+
+@pytest.mark.parametrize("w", ablation_workloads(L=1, T=3), ids=lambda w: w.name)
+def test_ablation_grid(cuda_device, w):
+    _sampled_run(w, cuda_device, [0, w.T - 1])
+
+
+def test_all_cmes_unbounded_window_is_plain_attention(cuda_device):
+    """k = N and a window that never evicts: GPU output equals the oracle and
+    plain softmax attention over [whole bank | every token so far]."""
+    w = full_window_workload(B=2, T=6)
+    P = Problem(w, cuda_device, idx=np.tile(np.arange(w.N), (w.B, 1)))
+    hist_k = [list(P.kv.ring_k[b, :, :, :P.kv.pos0[b]].transpose(2, 0, 1, 3))
+              for b in range(w.B)]
+    hist_v = [list(P.kv.ring_v[b, :, :, :P.kv.pos0[b]].transpose(2, 0, 1, 3))
+              for b in range(w.B)]
+    for t in range(w.T):
+        st = step_inputs(w, t)
+        out, ref = P.step(st)
+        got = to_f64(out)
+        assert_attn_close(got, ref, f"full-window step {t}")
+        for b in range(w.B):
+            hist_k[b].append(st.k_new[b])
+            hist_v[b].append(st.v_new[b])
+        # plain attention for a few heads
+        for b, l, h in [(0, 0, 0), (1, 0, 13), (1, 0, 31)]:
+            g = h // w.G
+            K = np.concatenate([oracle.bf16_to_f64(P.kv.tier1_k[b, l, g]),
+                                oracle.bf16_to_f64(np.stack(hist_k[b])[:, l, g])])
+            V = np.concatenate([oracle.bf16_to_f64(P.kv.tier1_v[b, l, g]),
+                                oracle.bf16_to_f64(np.stack(hist_v[b])[:, l, g])])
+            qv = oracle.bf16_to_f64(st.q[b, l, h])
+            z = K @ qv / np.sqrt(w.d)
+            p = np.exp(z - z.max())
+            plain = p @ V / p.sum()
+            np.testing.assert_allclose(ref[b, l, h], plain, rtol=1e-10, atol=1e-12)
+            assert_attn_close(got[b, l, h], plain, "plain attention")
+
+
+def test_fused_step_equals_append_then_attend(cuda_device):
+    """The fused step and the two separate calls give bit-identical results."""
+    for w in (WORKLOADS["tiny"], WORKLOADS["llama3_8b"].with_(L=2, T=3)):
+        A = Problem(w, cuda_device)
+        Bp = Problem(w, cuda_device)
+        for t in range(3):
+            st = step_inputs(w, t)
+            q = dev_bf16(st.q, cuda_device)
+            out_a = cmc.decode_step(q, A.t1k, A.t1v, A.idx, A.ring_k, A.ring_v, A.pos,
+                                    dev_bf16(st.k_new, cuda_device),
+                                    dev_bf16(st.v_new, cuda_device), workspace=A.ws)
+            cmc.window_append(Bp.ring_k, Bp.ring_v, Bp.pos, dev_bf16(st.k_new, cuda_device),
+                              dev_bf16(st.v_new, cuda_device))
+            out_b = cmc.two_tier_decode_attn(q, Bp.t1k, Bp.t1v, Bp.idx, Bp.ring_k, Bp.ring_v,
+                                             Bp.pos, workspace=Bp.ws)
+            torch.cuda.synchronize()
+            assert torch.equal(out_a.view(torch.int16), out_b.view(torch.int16))
+            assert torch.equal(A.ring_k, Bp.ring_k) and torch.equal(A.pos, Bp.pos)
+
+
+def test_deterministic(cuda_device):
+    w = WORKLOADS["llama3_8b"].with_(L=2)
+    outs = []
+    for _ in range(2):
+        P = Problem(w, cuda_device)
+        st = step_inputs(w, 0)
+        out, _ = P.step(st, compare=False)
+        outs.append(out.view(torch.int16).clone())
+    assert torch.equal(outs[0], outs[1])
+
+
+@pytest.mark.parametrize("G,d", [(1, 64), (2, 128), (8, 64), (8, 128), (4, 64)])
+def test_head_shapes(cuda_device, G, d):
+    Hkv = 2
+    w = WORKLOADS["tiny"].with_(B=2, L=3, Hq=G * Hkv, Hkv=Hkv, d=d, N=70, k=9, W=33, T=4,
+                                kv_std=1.0, q_std=1.0 / np.sqrt(d), W0=(33, 5))
+    P = Problem(w, cuda_device)
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t))
+        assert_attn_close(to_f64(out), ref, f"G={G} d={d} step {t}")
+    P.check_state()
+
+
+def test_ragged_fill_and_wrap(cuda_device):
+    """Sequences at different ring fills, including empty, crossing the wrap."""
+    w = WORKLOADS["tiny"].with_(B=5, W=16, k=7, T=20, W0=(0, 1, 9, 15, 16))
+    P = Problem(w, cuda_device)
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t))
+        assert_attn_close(to_f64(out), ref, f"ragged step {t}")
+    P.check_state()
+
+
+def test_window_of_one(cuda_device):
+    w = WORKLOADS["tiny"].with_(W=1, k=3, T=5)
+    P = Problem(w, cuda_device)
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t))
+        assert_attn_close(to_f64(out), ref, f"W=1 step {t}")
+    P.check_state()
+
+
+def test_k_zero_and_empty_cache(cuda_device):
+    w = WORKLOADS["tiny"].with_(k=0, B=2, W0=(0, 40), T=3)
+    P = Problem(w, cuda_device)
+    # attention without append on an empty ring: zero output for sequence 0
+    st = step_inputs(w, 0)
+    out = cmc.two_tier_decode_attn(dev_bf16(st.q, cuda_device), P.t1k, P.t1v, None, P.ring_k,
+                                   P.ring_v, P.pos, workspace=P.ws)
+    ref = oracle.two_tier_attention(st.q, P.kv.tier1_k, P.kv.tier1_v, None, P.o_ring_k,
+                                    P.o_ring_v, P.o_pos)
+    got = to_f64(out)
+    assert np.all(got[0] == 0.0)
+    assert_attn_close(got, ref, "k=0 attention-only")
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t))
+        assert_attn_close(to_f64(out), ref, f"k=0 step {t}")
+    P.check_state()
+
+
+def test_unsorted_idx_and_explicit_scale(cuda_device):
+    w = WORKLOADS["tiny"].with_(T=2)
+    idx = random_tier1_indices(w)
+    perm = np.random.default_rng(0).permutation(w.k)
+    P = Problem(w, cuda_device, idx=idx[:, perm])
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t), scale=0.05)
+        assert_attn_close(to_f64(out), ref, f"unsorted idx step {t}")
+
+
+def test_bad_index_and_bad_pos_are_flagged_and_skipped(cuda_device):
+    w = WORKLOADS["tiny"].with_(B=3, T=1)
+    idx = random_tier1_indices(w).astype(np.int64)
+    idx[1, 3] = -1
+    idx[1, 10] = w.N
+    P = Problem(w, cuda_device, idx=idx)
+    P.pos[2] = -5
+    st = step_inputs(w, 0)
+    out = cmc.decode_step(dev_bf16(st.q, cuda_device), P.t1k, P.t1v, P.idx, P.ring_k, P.ring_v,
+                          P.pos, dev_bf16(st.k_new, cuda_device),
+                          dev_bf16(st.v_new, cuda_device), workspace=P.ws)
+    flags = P.ws.status()
+    assert flags == cmc.DEVFLAG_BAD_INDEX | cmc.DEVFLAG_BAD_POS
+    got = to_f64(out)
+    # sequence 2: zero output, ring and pos untouched
+    assert np.all(got[2] == 0.0)
+    assert int(P.pos[2]) == -5
+    np.testing.assert_array_equal(host_bits(P.ring_k)[2], P.kv.ring_k[2])
+    # sequences 0 and 1: the oracle with the bad rows removed
+    keep = [np.array([i for i in row if 0 <= i < w.N]) for row in idx[:2]]
+    ring_k, ring_v = P.kv.ring_k[:2].copy(), P.kv.ring_v[:2].copy()
+    pos = P.kv.pos0[:2].copy()
+    oracle.window_append(ring_k, ring_v, pos, st.k_new[:2], st.v_new[:2])
+    for b in range(2):
+        for h in range(w.Hq):
+            ref = oracle.two_tier_attention_head(st.q, P.kv.tier1_k, P.kv.tier1_v,
+                                                 {b: keep[b]}, ring_k, ring_v, pos, b, 0, h)
+            assert_attn_close(got[b, 0, h], ref, f"bad idx b={b} h={h}")
+
+
+def test_large_unit_count(cuda_device):
+    """B * L * Hkv = 16,384 units in one launch (batch 64, 32 layers)."""
+    w = WORKLOADS["llama3_8b"].with_(B=64, L=32, N=40, k=8, W=24, T=1, W0=None)
+    P = Problem(w, cuda_device)
+    st = step_inputs(w, 0)
+    out, _ = P.step(st, compare=False)
+    got = to_f64(out)
+    rng = np.random.default_rng(0)
+    ring_k, ring_v, pos = P.o_ring_k, P.o_ring_v, P.o_pos
+    for _ in range(64):
+        b, l, h = int(rng.integers(w.B)), int(rng.integers(w.L)), int(rng.integers(w.Hq))
+        ref = oracle.two_tier_attention_head(st.q, P.kv.tier1_k, P.kv.tier1_v, P.idx_host,
+                                             ring_k, ring_v, pos, b, l, h)
+        assert_attn_close(got[b, l, h], ref, f"unit sample {(b, l, h)}")
+    P.check_state()

@@ -1,0 +1,125 @@
+"""Tier-1 scoring and selection on the GPU against the fp64 oracle.
+
+The selected index set is compared bit-exactly (as an ordered array); scores
+within 1e-5 absolute (fp32 accumulation over D <= 4096 terms of a cosine)."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_25537_gb300 as cmc
+from workloads import WORKLOADS, selection_inputs
+from workloads.configs import ablation_workload
+from _gpu_helpers import dev_f32
+
+pytestmark = pytest.mark.gpu
+
+SCORE_ATOL = 1e-5
+
+
+def _run(q, bank, k, dev):
+    qd, bd = dev_f32(q, dev), dev_f32(bank, dev)
+    scores = torch.empty(bank.shape[:2], dtype=torch.float32, device=dev)
+    idx = cmc.score_select(qd, bd, k, scores_out=scores)
+    # the workspace path (no scores_out) must select the same rows
+    idx2 = cmc.score_select(qd, bd, k)
+    torch.cuda.synchronize()
+    assert torch.equal(idx, idx2)
+    return idx.cpu().numpy(), scores.cpu().numpy()
+
+
+@pytest.mark.parametrize("name,batch", [
+    ("tiny", None), ("llama3_8b", None), ("mistral_batched", None),
+    ("long_context", range(0, 2)),
+])
+def test_select_workloads(cuda_device, name, batch):
+    w = WORKLOADS[name]
+    si = selection_inputs(w, batch=batch)
+    idx, scores = _run(si.question_emb, si.cme_bank, w.k, cuda_device)
+    ref_idx, ref_scores = oracle.score_select(si.question_emb, si.cme_bank, w.k)
+    np.testing.assert_array_equal(idx, ref_idx)
+    np.testing.assert_array_equal(idx, si.planted_idx)
+    assert np.abs(scores - ref_scores).max() <= SCORE_ATOL
+
+
+@pytest.mark.parametrize("k", [0, 64, 256, 1024])
+def test_select_ablation_k(cuda_device, k):
+    w = ablation_workload(k, 512, 16)
+    si = selection_inputs(w)
+    idx, _ = _run(si.question_emb, si.cme_bank, w.k, cuda_device)
+    ref_idx, _ = oracle.score_select(si.question_emb, si.cme_bank, w.k)
+    np.testing.assert_array_equal(idx, ref_idx)
+
+
+def test_select_ties_go_to_lower_index(cuda_device):
+    rng = np.random.default_rng(7)
+    B, N, D = 3, 700, 64
+    q = rng.standard_normal((B, D)).astype(np.float32)
+    bank = rng.standard_normal((B, N, D)).astype(np.float32)
+    # three bit-identical rows at the top; k = 2 must keep the two lowest indices
+    for b in range(B):
+        top = (q[b] * 3.0 + 0.01 * rng.standard_normal(D)).astype(np.float32)
+        for j in (5, 300, 650):
+            bank[b, j] = top
+    idx, scores = _run(q, bank, 2, cuda_device)
+    assert idx.tolist() == [[5, 300]] * B
+    assert np.all(scores[:, 5] == scores[:, 300]) and np.all(scores[:, 300] == scores[:, 650])
+    # duplicates straddling the cut deep in the ranking
+    k = 100
+    ref_scores = oracle.cosine_scores(q, bank)
+    for b in range(B):
+        order = np.argsort(-ref_scores[b], kind="stable")
+        cut_row = bank[b, order[k - 1]].copy()
+        for j in (order[k - 1], order[k + 5], 699):
+            bank[b, j] = cut_row
+    idx, _ = _run(q, bank, k, cuda_device)
+    ref_idx, _ = oracle.score_select(q, bank, k)
+    np.testing.assert_array_equal(idx, ref_idx)
+
+
+@pytest.mark.parametrize("N,D,k", [(1, 4, 1), (1, 4, 0), (5, 8, 5), (1000, 36, 999),
+                                   (1025, 512, 17), (3000, 4, 1500), (4096, 128, 4095)])
+def test_select_edge_shapes(cuda_device, N, D, k):
+    rng = np.random.default_rng(N + D + k)
+    B = 3
+    q = rng.standard_normal((B, D)).astype(np.float32)
+    bank = rng.standard_normal((B, N, D)).astype(np.float32)
+    idx, scores = _run(q, bank, k, cuda_device)
+    ref_idx, ref_scores = oracle.score_select(q, bank, k)
+    assert np.abs(scores - ref_scores).max() <= SCORE_ATOL
+    # without a planted margin, compare where the float32 decision is unambiguous
+    for b in range(B):
+        s = np.sort(ref_scores[b])[::-1]
+        if k in (0, N) or s[k - 1] - s[k] > 1e-5:
+            np.testing.assert_array_equal(idx[b], ref_idx[b])
+        assert idx[b].tolist() == sorted(set(idx[b].tolist()))
+        assert len(idx[b]) == k
+
+
+def test_select_zero_vectors(cuda_device):
+    B, N, D = 2, 40, 16
+    rng = np.random.default_rng(3)
+    q = rng.standard_normal((B, D)).astype(np.float32)
+    q[1] = 0.0                                    # zero question: every score 0
+    bank = rng.standard_normal((B, N, D)).astype(np.float32)
+    bank[0, 7] = 0.0                              # zero CME: score 0
+    idx, scores = _run(q, bank, 10, cuda_device)
+    assert scores[0, 7] == 0.0 and np.all(scores[1] == 0.0)
+    assert idx[1].tolist() == list(range(10))
+    ref_idx, _ = oracle.score_select(q, bank, 10)
+    np.testing.assert_array_equal(idx, ref_idx)
+
+
+def test_select_negative_and_signed_zero_scores(cuda_device):
+    # orthogonal rows give +-0 dot products; -0 and +0 must tie (lower index wins)
+    B, N, D = 1, 8, 4
+    q = np.array([[1.0, 0.0, 0.0, 0.0]], dtype=np.float32)
+    bank = np.zeros((B, N, D), dtype=np.float32)
+    bank[0, :, 1] = 1.0
+    bank[0, 0] = [-1.0, 0.0, 0.0, 0.0]   # score -1
+    bank[0, 3] = [-0.0, 2.0, 0.0, 0.0]   # dot -0
+    bank[0, 6] = [0.5, 0.5, 0.0, 0.0]    # positive
+    idx, scores = _run(q, bank, 3, cuda_device)
+    assert idx[0].tolist() == [1, 2, 6]
+    assert not np.signbit(scores[0, 3])

@@ -13,6 +13,7 @@ from .generate import (
     selection_inputs,
     kv_inputs,
     step_inputs,
+    random_tier1_indices,
     f32_to_bf16_bits,
     bf16_bits_to_f32,
 )
@@ -28,6 +29,7 @@ __all__ = [
     "selection_inputs",
     "kv_inputs",
     "step_inputs",
+    "random_tier1_indices",
     "f32_to_bf16_bits",
     "bf16_bits_to_f32",
 ]

@@ -45,6 +45,7 @@ _TAGS = {
     "step_q": 9,
     "step_k": 10,
     "step_v": 11,
+    "idx": 12,
 }
 
 
@@ -67,10 +68,19 @@ def bf16_bits_to_f32(bits: np.ndarray) -> np.ndarray:
             << np.uint32(16)).view(np.float32)
 
 
-def _gauss_bf16(rng: np.random.Generator, shape, std: float) -> np.ndarray:
-    x = rng.standard_normal(shape, dtype=np.float32)
-    x *= np.float32(std)
-    return f32_to_bf16_bits(x)
+def _torch_gen(seed: int, tag: str, *extra: int):
+    import torch
+    s = np.random.SeedSequence([seed, _TAGS[tag], *extra]).generate_state(1, np.uint64)[0]
+    return torch.Generator().manual_seed(int(s) & 0x7FFFFFFFFFFFFFFF)
+
+
+def _gauss_bf16(key, shape, std: float) -> np.ndarray:
+    """Gaussian bf16 bit patterns; torch's float32 -> bfloat16 cast rounds to
+    nearest even, like f32_to_bf16_bits."""
+    import torch
+    x = torch.randn(tuple(shape), generator=_torch_gen(*key), dtype=torch.float32)
+    x.mul_(float(std))
+    return x.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
 
 
 # ----------------------------------------------------------------------------
@@ -102,20 +112,29 @@ def _target_cosines(w: Workload, b: int, attempt: int):
 
 def _bank_rows(w: Workload, b: int, attempt: int, qhat: np.ndarray, c: np.ndarray,
                out: np.ndarray, chunk: int = 2048) -> None:
-    rng = _rng(w.seed, "bank", b, attempt)
+    import torch
+    qh = torch.from_numpy(qhat)
+    out_t = torch.from_numpy(out)
+    work = torch.empty((min(chunk, w.N), w.D), dtype=torch.float64)
     for r0 in range(0, w.N, chunk):
         r1 = min(w.N, r0 + chunk)
-        g = rng.standard_normal((r1 - r0, w.D), dtype=np.float32).astype(np.float64)
-        g *= w.emb_std
-        along = g @ qhat
-        perp = g - along[:, None] * qhat[None, :]
-        rho = np.sqrt(np.einsum("ij,ij->i", g, g))
-        pn = np.sqrt(np.einsum("ij,ij->i", perp, perp))
-        u = perp / pn[:, None]
-        cj = c[r0:r1]
-        rows = rho[:, None] * (cj[:, None] * qhat[None, :]
-                               + np.sqrt(1.0 - cj * cj)[:, None] * u)
-        out[r0:r1] = rows.astype(np.float32)
+        g = work[: r1 - r0]
+        g.copy_(torch.randn((r1 - r0, w.D), generator=_torch_gen(w.seed, "bank", b, attempt, r0),
+                            dtype=torch.float32))
+        g.mul_(float(w.emb_std))
+        # g = along * qhat + perp with perp orthogonal to qhat; the row keeps
+        # |g| and the direction of perp, and gets cosine c_j with q:
+        #   m = |g| (c_j qhat + sqrt(1 - c_j^2) perp / |perp|)
+        along = g @ qh
+        rho2 = torch.linalg.vector_norm(g, dim=1) ** 2
+        rho = rho2.sqrt()
+        pn = (rho2 - along * along).sqrt()
+        cj = torch.from_numpy(np.ascontiguousarray(c[r0:r1]))
+        coef_perp = rho * (1.0 - cj * cj).sqrt() / pn
+        coef_q = rho * cj - coef_perp * along
+        g.mul_(coef_perp[:, None])
+        g.addr_(coef_q, qh)
+        out_t[r0:r1].copy_(g)
 
 
 def selection_inputs(w: Workload, attempt: int = 0, batch: Optional[range] = None
@@ -166,13 +185,13 @@ def kv_inputs(w: Workload, batch: Optional[range] = None) -> KVInputs:
     rv = np.zeros((nb, w.L, w.Hkv, w.W, w.d), dtype=np.uint16)
     pos0 = np.empty(nb, dtype=np.int64)
     for i, b in enumerate(seqs):
-        t1k[i] = _gauss_bf16(_rng(w.seed, "tier1_k", b), shp_bank, w.kv_std)
-        t1v[i] = _gauss_bf16(_rng(w.seed, "tier1_v", b), shp_bank, w.kv_std)
+        t1k[i] = _gauss_bf16((w.seed, "tier1_k", b), shp_bank, w.kv_std)
+        t1v[i] = _gauss_bf16((w.seed, "tier1_v", b), shp_bank, w.kv_std)
         f = fill[b]
         assert 0 <= f <= w.W
         shp_ring = (w.L, w.Hkv, f, w.d)
-        rk[i, :, :, :f] = _gauss_bf16(_rng(w.seed, "ring_k", b), shp_ring, w.kv_std)
-        rv[i, :, :, :f] = _gauss_bf16(_rng(w.seed, "ring_v", b), shp_ring, w.kv_std)
+        rk[i, :, :, :f] = _gauss_bf16((w.seed, "ring_k", b), shp_ring, w.kv_std)
+        rv[i, :, :, :f] = _gauss_bf16((w.seed, "ring_v", b), shp_ring, w.kv_std)
         pos0[i] = f
     return KVInputs(t1k, t1v, rk, rv, pos0)
 
@@ -188,11 +207,29 @@ class StepInputs:
     v_new: np.ndarray  # bf16 bits [B, L, Hkv, d]
 
 
-def step_inputs(w: Workload, t: int, q_std: Optional[float] = None) -> StepInputs:
-    """Query and new-token K/V of decode step t (all sequences, all layers)."""
+def step_inputs(w: Workload, t: int, q_std: Optional[float] = None,
+                parts: str = "qkv") -> StepInputs:
+    """Query and new-token K/V of decode step t (all sequences, all layers).
+    `parts` picks which of q, k_new, v_new to draw (the others are None)."""
     qs = w.q_std if q_std is None else q_std
     return StepInputs(
-        q=_gauss_bf16(_rng(w.seed, "step_q", t), (w.B, w.L, w.Hq, w.d), qs),
-        k_new=_gauss_bf16(_rng(w.seed, "step_k", t), (w.B, w.L, w.Hkv, w.d), w.kv_std),
-        v_new=_gauss_bf16(_rng(w.seed, "step_v", t), (w.B, w.L, w.Hkv, w.d), w.kv_std),
+        q=_gauss_bf16((w.seed, "step_q", t), (w.B, w.L, w.Hq, w.d), qs)
+        if "q" in parts else None,
+        k_new=_gauss_bf16((w.seed, "step_k", t), (w.B, w.L, w.Hkv, w.d), w.kv_std)
+        if "k" in parts else None,
+        v_new=_gauss_bf16((w.seed, "step_v", t), (w.B, w.L, w.Hkv, w.d), w.kv_std)
+        if "v" in parts else None,
     )
+
+
+def random_tier1_indices(w: Workload, batch: Optional[range] = None) -> np.ndarray:
+    """A seeded, ascending k-subset of [0, N) per sequence: int32 [B, k].
+
+    Stands in for a selection result when the attention path is exercised
+    without generating the CME bank."""
+    seqs = range(w.B) if batch is None else batch
+    out = np.empty((len(seqs), w.k), dtype=np.int32)
+    for i, b in enumerate(seqs):
+        rng = _rng(w.seed, "idx", b)
+        out[i] = np.sort(rng.choice(w.N, size=w.k, replace=False))
+    return out
