@@ -184,6 +184,38 @@ CMC_API int cmc_decode_step(const void* q, const void* tier1_k, const void* tier
  * bits) into *flags, waiting for `stream`, and clears it when `clear` != 0. */
 CMC_API int cmc_read_status(void* workspace, int clear, uint32_t* flags, void* stream);
 
+/* ------------------------------------------------------------------------ *
+ * Allocation-free Tier-1 selection                                          *
+ * ------------------------------------------------------------------------ */
+
+/* Largest B * N that cmc_score_select_static accepts (1 MiB of fp32 scores). */
+#define CMC_STATIC_SCORES_MAX 262144
+
+/*
+ * cmc_score_select without a caller-provided workspace.  The paper has no
+ * counterpart: this is a deployment variant of the same computation.
+ *
+ * Some callers cannot hand the library a workspace: a serving engine that
+ * reserves all free HBM for its KV-cache pool at start-up and forbids any
+ * later allocation, or a plain C host program that links only this library
+ * and owns no device allocator.  This entry point allocates nothing and calls
+ * no allocating routine.  Its score scratch is one file-scope device array of
+ * CMC_STATIC_SCORES_MAX floats (1 MiB), which every GPU that loads the library
+ * holds until the process exits.
+ *
+ * Arguments, results and limits are those of cmc_score_select, except that
+ * there is no scores_out and no workspace, and B * N must not exceed
+ * CMC_STATIC_SCORES_MAX (otherwise CMC_ERR_SHAPE, nothing launched).
+ *
+ * The first call on a device looks up the array's device address (with that
+ * device current); make that first call before any stream capture.  All calls
+ * share the one array: each call overwrites the B * N scores it then reads,
+ * so nothing in it needs to start at zero, but calls whose kernels overlap on
+ * the GPU (different streams, no ordering between them) race on it.
+ */
+CMC_API int cmc_score_select_static(const float* question_emb, const float* cme_bank, int B,
+                                    int N, int D, int k, int32_t* idx_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -24,6 +24,7 @@ EXPORTS = (
     "cmc_two_tier_decode_attn",
     "cmc_decode_step",
     "cmc_read_status",
+    "cmc_score_select_static",
 )
 
 STATUS = {
@@ -78,7 +79,11 @@ _SIGNATURES = {
     "cmc_decode_step": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _dims_p,
                              ctypes.c_float, _vp, _vp, _sz, _vp]),
     "cmc_read_status": (_i, [_vp, _i, ctypes.POINTER(ctypes.c_uint32), _vp]),
+    "cmc_score_select_static": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
 }
+
+# Largest B * N accepted by cmc_score_select_static (CMC_STATIC_SCORES_MAX).
+STATIC_SCORES_MAX = 262144
 
 
 def lib() -> ctypes.CDLL:

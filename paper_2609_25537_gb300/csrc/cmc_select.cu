@@ -14,6 +14,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "cmc_internal.cuh"
 
 namespace cmc {
@@ -226,3 +228,65 @@ int cmc_score_select(const float* question_emb, const float* cme_bank, int B, in
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant: the score scratch is a file-scope device array.
+// ---------------------------------------------------------------------------
+
+// One copy per device that loads the library; shared by every call.
+static __device__ __align__(256) float g_static_scores[CMC_STATIC_SCORES_MAX];
+
+namespace cmc {
+
+constexpr int kStaticMaxDevices = 64;
+static std::mutex g_static_mu;
+static float* g_static_scores_dev[kStaticMaxDevices] = {};
+
+// Device address of g_static_scores on the current device; looked up once per
+// device (host code cannot use the symbol itself as a device pointer).
+static int static_scores_address(float** out) {
+  int dev = -1;
+  int st = record_cuda_error(cudaGetDevice(&dev));
+  if (st != CMC_OK) return st;
+  if (dev < 0 || dev >= kStaticMaxDevices) return CMC_ERR_SHAPE;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_scores_dev[dev]) {
+    void* p = nullptr;
+    st = record_cuda_error(cudaGetSymbolAddress(&p, g_static_scores));
+    if (st != CMC_OK) return st;
+    if (!p) return CMC_ERR_CUDA;
+    g_static_scores_dev[dev] = static_cast<float*>(p);
+  }
+  *out = g_static_scores_dev[dev];
+  return CMC_OK;
+}
+
+}  // namespace cmc
+
+extern "C" int cmc_score_select_static(const float* question_emb, const float* cme_bank, int B,
+                                       int N, int D, int k, int32_t* idx_out, void* stream) {
+  using namespace cmc;
+  if (B < 1 || B > 65535 || N < 1 || N > (1 << 20) || D < 4 || D > 65536 || (D & 3))
+    return CMC_ERR_SHAPE;
+  if (static_cast<long long>(B) * N > CMC_STATIC_SCORES_MAX) return CMC_ERR_SHAPE;
+  if (k < 0 || k > N) return CMC_ERR_RANGE;
+  if (!question_emb || !cme_bank) return CMC_ERR_NULL;
+  if (k > 0 && !idx_out) return CMC_ERR_NULL;
+  if (!aligned16(question_emb) || !aligned16(cme_bank)) return CMC_ERR_ALIGN;
+  if (idx_out && (reinterpret_cast<uintptr_t>(idx_out) & 3)) return CMC_ERR_ALIGN;
+  float* sc = nullptr;
+  int st = static_scores_address(&sc);
+  if (st != CMC_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const long long rows = static_cast<long long>(B) * N;
+  const long long warps_per_block = kScoreThreads / 32;
+  long long blocks = (rows + warps_per_block - 1) / warps_per_block;
+  const long long cap = static_cast<long long>(sm_count()) * 16;
+  if (blocks > cap) blocks = cap;
+  cosine_scores_kernel<<<static_cast<unsigned>(blocks), kScoreThreads, 0, s>>>(
+      question_emb, cme_bank, N, D, rows, sc);
+  st = check_launch();
+  if (st != CMC_OK || k == 0) return st;
+  topk_select_kernel<<<B, kSelectThreads, 0, s>>>(sc, N, k, idx_out);
+  return check_launch();
+}
