@@ -7,9 +7,12 @@ a 512-token window, 3,000 decode steps.
 
 One benchmark step is one generation round over R independent requests of
 that shape (R = --requests, default 4): each request first runs the Tier-1
-scoring + top-k selection on its own CME bank, then the R requests run their
-3,000 fused decode steps (ring append + two-tier attention over all 32
-layers, one launch per request per step) round-robin.  Each request's KV
+scoring + top-k selection on its own CME bank and compacts the selected K/V
+rows into its dense Tier-1 cache (cmc_tier1_gather: the cache the paper's
+prefill of the selected CMEs leaves), then the R requests run their 3,000
+fused decode steps (ring append + two-tier attention over all 32 layers, one
+launch per request per step) round-robin.  `--tier1 gather` instead passes the
+bank and idx to every decode step (the gather inside the attention kernel).  Each request's KV
 state (84.5 MB read per step) fits in the 129 MB L2 by itself; interleaving R
 requests puts (R-1) x 84.5 MB of other traffic between two steps of the same
 request, so every launch reads its K/V from HBM, as it would inside a real
@@ -21,6 +24,8 @@ Reported (one JSON line on rank 0):
   roofline       the fused decode-step kernel: algorithmic bytes per launch
                  / average launch time, against the measured HBM copy peak;
   select_us      Tier-1 score + select per request (two launches), L2-cold;
+  tier1_gather_us  the once-per-request Tier-1 compaction;
+  variant        the decode step with the other Tier-1 form, us per launch;
   e2e            the same metric through the Python API with host buffers
                  (question vector, CME bank and every step's q / new K,V
                  copied in from pinned memory, every step's output copied out);
@@ -67,14 +72,20 @@ KERNEL_SOURCES = [os.path.join(ROOT, "paper_2609_25537_gb300", "csrc", f)
 # Accounting
 # ----------------------------------------------------------------------------
 
-def decode_step_bytes(B, L, Hq, Hkv, d, k, W) -> int:
+def decode_step_bytes(B, L, Hq, Hkv, d, k, W, gather=False) -> int:
     """Algorithmic HBM bytes of one fused decode step with a full ring:
     k selected Tier-1 rows and W - 1 old ring rows of K and V read, the new
-    token's K,V read once and written once, q read, out written, idx read."""
+    token's K,V read once and written once, q read, out written, and idx
+    read when the step gathers the Tier-1 rows itself."""
     kv_row = d * 2
     return (B * L * Hkv * 2 * kv_row * (k + W + 1)
             + B * L * Hq * d * 2 * 2
-            + B * k * 4)
+            + (B * k * 4 if gather else 0))
+
+
+def tier1_gather_bytes(B, L, Hkv, d, k) -> int:
+    """The selected K and V rows read from the bank and written densely, idx read."""
+    return 2 * 2 * B * L * Hkv * k * d * 2 + B * k * 4
 
 
 def decode_step_flops(B, L, Hq, d, k, W) -> int:
@@ -305,22 +316,37 @@ class Request:
         self.k_new = randn((pool, B, L, Hkv, d), w.kv_std)
         self.v_new = randn((pool, B, L, Hkv, d), w.kv_std)
         self.idx = torch.empty((B, w.k), dtype=torch.int32, device=dev)
+        self.t1k_dense = torch.empty((B, L, Hkv, w.k, d), dtype=torch.bfloat16, device=dev)
+        self.t1v_dense = torch.empty((B, L, Hkv, w.k, d), dtype=torch.bfloat16, device=dev)
         self.out = torch.empty((B, L, Hq, d), dtype=torch.bfloat16, device=dev)
         self.sel_ws = torch.empty(cmc.score_select_workspace_size(B, w.N), dtype=torch.uint8,
                                   device=dev)
-        dims = cmc.dims_of(self.out, self.t1k, self.idx, self.ring_k)
-        self.ws = cmc.DecodeWorkspace(dims, dev)
+        self.ws = cmc.DecodeWorkspace(cmc.dims_of(self.out, self.t1k, self.idx, self.ring_k),
+                                      dev)
+        self.ws_dense = cmc.DecodeWorkspace(
+            cmc.dims_of(self.out, self.t1k_dense, None, self.ring_k), dev)
 
     def select(self):
         import paper_2609_25537_gb300 as cmc
         cmc.score_select(self.qemb, self.bank, self.idx.shape[1], idx_out=self.idx,
                          workspace=self.sel_ws)
 
-    def decode(self, p):
+    def gather(self):
         import paper_2609_25537_gb300 as cmc
-        cmc.decode_step(self.q[p], self.t1k, self.t1v, self.idx, self.ring_k, self.ring_v,
-                        self.pos, self.k_new[p], self.v_new[p], out=self.out,
-                        workspace=self.ws)
+        cmc.tier1_gather(self.t1k, self.t1v, self.idx, out_k=self.t1k_dense,
+                         out_v=self.t1v_dense, workspace=self.ws_dense)
+
+    def decode(self, p, q=None, k_new=None, v_new=None, mode="dense"):
+        import paper_2609_25537_gb300 as cmc
+        q = self.q[p] if q is None else q
+        k_new = self.k_new[p] if k_new is None else k_new
+        v_new = self.v_new[p] if v_new is None else v_new
+        if mode == "dense":
+            cmc.decode_step(q, self.t1k_dense, self.t1v_dense, None, self.ring_k, self.ring_v,
+                            self.pos, k_new, v_new, out=self.out, workspace=self.ws_dense)
+        else:
+            cmc.decode_step(q, self.t1k, self.t1v, self.idx, self.ring_k, self.ring_v,
+                            self.pos, k_new, v_new, out=self.out, workspace=self.ws)
 
     def host_state(self):
         def bits(t):
@@ -347,19 +373,26 @@ def run_gpu(args, w, world, rank, local):
     cpu_state = reqs[0].host_state() if want_cpu else None
     stream = torch.cuda.Stream(device=dev)
 
+    mode = args.tier1
+    other = "gather" if mode == "dense" else "dense"
     # eager warm-up of every kernel before graph capture
     with torch.cuda.stream(stream):
         for r in reqs:
             r.select()
-            r.decode(0)
+            r.gather()
+            r.decode(0, mode=mode)
+            r.decode(0, mode=other)
     stream.synchronize()
 
     # one graph = P rounds of R decode launches; replayed T / P times per step
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph, stream=stream):
-        for p in range(P):
-            for r in reqs:
-                r.decode(p)
+    def capture(m):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for p in range(P):
+                for r in reqs:
+                    r.decode(p, mode=m)
+        return g
+    graph = capture(mode)
     replays = T // P
 
     def one_step(ev=None):
@@ -370,17 +403,22 @@ def run_gpu(args, w, world, rank, local):
                 r.select()
             if ev is not None:
                 ev[1].record(stream)
+            if mode == "dense":
+                for r in reqs:
+                    r.gather()
+            if ev is not None:
+                ev[2].record(stream)
             for _ in range(replays):
                 graph.replay()
             if ev is not None:
-                ev[2].record(stream)
+                ev[3].record(stream)
 
     for _ in range(args.warmup):
         one_step()
     stream.synchronize()
 
     K = args.steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
     barrier(world)
     torch.cuda.synchronize(dev)
     clocks = ClockSampler(dev) if rank == 0 else None
@@ -396,17 +434,38 @@ def run_gpu(args, w, world, rank, local):
 
     elapsed_ms = t_start.elapsed_time(t_end)
     sel_ms = [e[0].elapsed_time(e[1]) for e in evs]
-    dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    gat_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    dec_ms = [e[2].elapsed_time(e[3]) for e in evs]
     max_ms = max_over_ranks(elapsed_ms, world, dev)
     tokens = world * K * R * w.B * T
     value = tokens / (max_ms / 1000.0)
 
     launches_dec = K * R * T
     launch_us = 1000.0 * sum(dec_ms) / launches_dec
-    nbytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W)
+    nbytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W, gather=mode == "gather")
     achieved = nbytes / (launch_us * 1e-6) / 1e9
     peak, peak_kind = measured_peaks()
     select_us = 1000.0 * statistics.median(sel_ms) / R
+    gather_us = 1000.0 * statistics.median(gat_ms) / R if mode == "dense" else 0.0
+
+    # the decode step with the other Tier-1 form (same state, same launch shape)
+    variant = None
+    if not args.no_variant:
+        g2 = capture(other)
+        with torch.cuda.stream(stream):
+            g2.replay()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(args.variant_replays):
+                g2.replay()
+            e1.record(stream)
+        stream.synchronize()
+        v_us = 1000.0 * e0.elapsed_time(e1) / (args.variant_replays * P * R)
+        v_bytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W,
+                                    gather=other == "gather")
+        variant = {"tier1": other, "us_per_launch": v_us,
+                   "achieved_gbs": v_bytes / (v_us * 1e-6) / 1e9}
+        del g2
 
     # e2e through the Python API with pinned host buffers
     e2e = run_e2e(args, w, reqs, dev, stream, world) if not args.no_e2e else None
@@ -425,13 +484,20 @@ def run_gpu(args, w, world, rank, local):
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": K, "warmup": args.warmup, "ms_per_step": max_ms / K,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "bf16", "data": "synthetic", "config": workload_config(w, R),
+        "dtype": "bf16", "data": "synthetic",
+        "config": dict(workload_config(w, R), tier1=mode),
+        "tier1": mode,
         "decode_us_per_launch": launch_us,
         "hbm_pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
         "select_us": select_us,
+        "tier1_gather_us": gather_us,
+        "tier1_gather_gbs": (tier1_gather_bytes(w.B, w.L, w.Hkv, w.d, w.k) / (gather_us * 1e-6)
+                             / 1e9 if gather_us > 0 else None),
+        "variant": variant,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
-                     "kernel": "two_tier_attn_kernel<128,4,fused>",
+                     "kernel": ("fused decode step: two_tier_attn_kernel<128,4,fused> + "
+                                "two_tier_combine_kernel"),
                      "bytes_per_launch": nbytes, "traffic": profiled_traffic(),
                      "flops_per_launch": decode_step_flops(w.B, w.L, w.Hq, w.d, w.k, w.W)},
         "select_roofline": {"bound": "hbm", "bytes": select_bytes(w.B, w.N, w.D, w.k),
@@ -439,7 +505,7 @@ def run_gpu(args, w, world, rank, local):
                             / 1e9, "unit": "GB/s"},
         "e2e": e2e,
         "cpu_baseline": cpu,
-        "gpu_launches": K * R * (T + 2),
+        "gpu_launches": K * R * (2 * T + (3 if mode == "dense" else 2)),
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)
@@ -472,14 +538,15 @@ def run_e2e(args, w, reqs, dev, stream, world):
                 r.qemb.copy_(h["qemb"], non_blocking=True)
                 r.bank.copy_(h["bank"], non_blocking=True)
                 cmc.score_select(r.qemb, r.bank, w.k, idx_out=r.idx, workspace=r.sel_ws)
+                if args.tier1 == "dense":
+                    r.gather()
             for t in range(T):
                 p = t % P
                 for r, h in zip(reqs, host):
                     h["q_d"].copy_(h["q"][p], non_blocking=True)
                     h["k_d"].copy_(h["k"][p], non_blocking=True)
                     h["v_d"].copy_(h["v"][p], non_blocking=True)
-                    cmc.decode_step(h["q_d"], r.t1k, r.t1v, r.idx, r.ring_k, r.ring_v, r.pos,
-                                    h["k_d"], h["v_d"], out=r.out, workspace=r.ws)
+                    r.decode(p, q=h["q_d"], k_new=h["k_d"], v_new=h["v_d"], mode=args.tier1)
                     h["out"][p].copy_(r.out, non_blocking=True)
         stream.synchronize()
 
@@ -511,6 +578,10 @@ def main(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tier1", choices=("dense", "gather"), default="dense",
+                    help="Tier-1 form of the timed decode steps")
+    ap.add_argument("--no-variant", action="store_true")
+    ap.add_argument("--variant-replays", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--ref-step-seconds", type=float, default=2.0)
     args = ap.parse_args(argv)

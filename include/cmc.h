@@ -60,6 +60,8 @@ typedef enum cmc_status {
  * cmc_read_status).  Kernels skip the offending element and carry on. */
 #define CMC_DEVFLAG_BAD_INDEX 1u /* an idx entry outside [0, N): that row was skipped   */
 #define CMC_DEVFLAG_BAD_POS 2u   /* a negative pos: that sequence was skipped            */
+#define CMC_DEVFLAG_TIMEOUT 4u   /* a pipeline wait hit its iteration limit: the call's
+                                    outputs are invalid (never expected in operation)     */
 
 /* Shapes of one decode problem. */
 typedef struct cmc_dims {
@@ -137,21 +139,27 @@ CMC_API int cmc_window_append(void* ring_k, void* ring_v, int64_t* pos, const vo
  * ------------------------------------------------------------------------ */
 
 /* Bytes of workspace the two attention entry points need for `dims`.  The
- * workspace must be zero-filled once before its first use; every call leaves
- * its counters at zero again. */
+ * workspace starts with the device status word (read by cmc_read_status),
+ * which must be zero before the first call: zero-fill the workspace once.
+ * The rest holds fp32 partial results that each call writes before reading. */
 CMC_API size_t cmc_decode_attn_workspace_size(const cmc_dims* dims);
 
 /*
  * For every sequence b, layer l and query head h (KV head g = h / (Hq/Hkv)):
  *     out[b,l,h] = sum_i softmax_i(scale * q[b,l,h] . key_i) value_i
  * over the keys of
- *     Tier-1: tier1_k[b,l,g, idx[b,i]] for i < k (gathered by index), then
+ *     Tier-1: tier1_k[b,l,g, idx[b,i]] for i < k (gathered by index), or,
+ *             when idx is NULL, tier1_k[b,l,g, i] for i < k (the selected
+ *             rows already stored in order, as cmc_tier1_gather or the
+ *             prefill of the selected CMEs leaves them), then
  *     Tier-2: ring_k[b,l,g, s] for the occupied slots s < min(pos[b], W).
  * An empty cache gives a zero output.
  *
  *   q                 bf16 [B, L, Hq, d]
- *   tier1_k, tier1_v  bf16 [B, L, Hkv, N, d]
- *   idx               int32 [B, k]   (may be NULL when k == 0); any order
+ *   tier1_k, tier1_v  bf16 [B, L, Hkv, N, d]   (N >= k)
+ *   idx               int32 [B, k] in any order, or NULL (identity selection;
+ *                     the Tier-1 tiles then stream as contiguous boxes, which
+ *                     is the fast path)
  *   ring_k, ring_v    bf16 [B, L, Hkv, W, d]
  *   pos               int64 [B]      tokens appended so far (read only)
  *   scale             softmax scale; <= 0 selects 1/sqrt(d)
@@ -179,6 +187,27 @@ CMC_API int cmc_decode_step(const void* q, const void* tier1_k, const void* tier
                             const int32_t* idx, void* ring_k, void* ring_v, int64_t* pos,
                             const void* k_new, const void* v_new, const cmc_dims* dims, float scale,
                             void* out, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Tier-1 compaction, once per question: copies the selected rows of the
+ * per-CME K/V bank into a dense Tier-1 cache,
+ *     tier1_k[b,l,g,i] = bank_k[b,l,g, idx[b,i]]   for i < k  (same for V),
+ * the cache that Section 2.5's prefill of the selected CMEs M* (re-ordered by
+ * document position) leaves.  Decode steps then pass tier1_k/v with N = k and
+ * idx = NULL.
+ *
+ *   bank_k, bank_v    bf16 [B, L, Hkv, N, d]
+ *   idx               int32 [B, k]   (from cmc_score_select)
+ *   tier1_k, tier1_v  bf16 [B, L, Hkv, k, d]   output; must not overlap the bank
+ *   status            NULL, or a device uint32 word (for example the start of an
+ *                     attention workspace) that receives CMC_DEVFLAG_BAD_INDEX
+ *                     when an idx entry is outside [0, N); that row is zeroed
+ *
+ * dims->Hq and W are ignored.  k == 0 launches nothing.
+ */
+CMC_API int cmc_tier1_gather(const void* bank_k, const void* bank_v, const int32_t* idx,
+                             const cmc_dims* dims, void* tier1_k, void* tier1_v, uint32_t* status,
+                             void* stream);
 
 /* Copies the device status word of an attention workspace (CMC_DEVFLAG_*
  * bits) into *flags, waiting for `stream`, and clears it when `clear` != 0. */

@@ -10,11 +10,13 @@ from .cmc import (  # noqa: F401
     DecodeWorkspace,
     DEVFLAG_BAD_INDEX,
     DEVFLAG_BAD_POS,
+    DEVFLAG_TIMEOUT,
     decode_attn_workspace_size,
     decode_step,
     dims_of,
     score_select,
     score_select_workspace_size,
+    tier1_gather,
     two_tier_decode_attn,
     window_append,
 )

@@ -23,6 +23,7 @@ EXPORTS = (
     "cmc_decode_attn_workspace_size",
     "cmc_two_tier_decode_attn",
     "cmc_decode_step",
+    "cmc_tier1_gather",
     "cmc_read_status",
     "cmc_score_select_static",
 )
@@ -39,6 +40,7 @@ STATUS = {
 
 DEVFLAG_BAD_INDEX = 1
 DEVFLAG_BAD_POS = 2
+DEVFLAG_TIMEOUT = 4
 
 
 class CmcDims(ctypes.Structure):
@@ -78,6 +80,7 @@ _SIGNATURES = {
                                       ctypes.c_float, _vp, _vp, _sz, _vp]),
     "cmc_decode_step": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _dims_p,
                              ctypes.c_float, _vp, _vp, _sz, _vp]),
+    "cmc_tier1_gather": (_i, [_vp, _vp, _vp, _dims_p, _vp, _vp, _vp, _vp]),
     "cmc_read_status": (_i, [_vp, _i, ctypes.POINTER(ctypes.c_uint32), _vp]),
     "cmc_score_select_static": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
 }

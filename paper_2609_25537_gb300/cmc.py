@@ -12,6 +12,11 @@ Tensor layouts (row-major, last index fastest):
   tier1_k/v     bf16 [B, L, Hkv, N, d] idx       int32 [B, k]
   ring_k/v      bf16 [B, L, Hkv, W, d] pos       int64 [B]
   k_new/v_new   bf16 [B, L, Hkv, d]
+
+Tier-1 selection in the attention calls: an ``idx`` tensor [B, k] gathers
+rows of the bank by index at every step; ``idx=None`` takes every row of
+``tier1_k``/``tier1_v`` in order (k = N), which is how the dense Tier-1 cache
+made once per question by :func:`tier1_gather` is passed.
 """
 
 from __future__ import annotations
@@ -22,7 +27,7 @@ from typing import Dict, Optional, Tuple
 
 import torch
 
-from ._lib import CmcDims, check, lib, DEVFLAG_BAD_INDEX, DEVFLAG_BAD_POS
+from ._lib import CmcDims, check, lib, DEVFLAG_BAD_INDEX, DEVFLAG_BAD_POS, DEVFLAG_TIMEOUT
 
 __all__ = [
     "CmcDims",
@@ -32,10 +37,12 @@ __all__ = [
     "window_append",
     "two_tier_decode_attn",
     "decode_step",
+    "tier1_gather",
     "decode_attn_workspace_size",
     "dims_of",
     "DEVFLAG_BAD_INDEX",
     "DEVFLAG_BAD_POS",
+    "DEVFLAG_TIMEOUT",
 ]
 
 
@@ -112,7 +119,7 @@ def dims_of(q: torch.Tensor, tier1_k: torch.Tensor, idx: Optional[torch.Tensor],
     B, L, Hq, d = q.shape
     Bk, Lk, Hkv, N, dk = tier1_k.shape
     Br, Lr, Hr, W, dr = ring_k.shape
-    k = 0 if idx is None else int(idx.shape[1])
+    k = N if idx is None else int(idx.shape[1])
     if (Bk, Lk, dk) != (B, L, d) or (Br, Lr, Hr, dr) != (B, L, Hkv, d):
         raise ValueError(f"inconsistent shapes: q {tuple(q.shape)}, tier1 {tuple(tier1_k.shape)}, "
                          f"ring {tuple(ring_k.shape)}")
@@ -128,8 +135,8 @@ def decode_attn_workspace_size(dims: CmcDims) -> int:
 class DecodeWorkspace:
     """Zero-filled device workspace for the attention entry points.
 
-    Holds the split-K partials, the arrival tickets and the device status word.
-    Calls sharing one workspace must be ordered on one stream."""
+    Holds the device status word and the fp32 partial results of keys split
+    between CTAs.  Calls sharing one workspace must be ordered on one stream."""
 
     def __init__(self, dims: CmcDims, device: torch.device):
         n = decode_attn_workspace_size(dims)
@@ -219,6 +226,40 @@ def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, *,
         ws.nbytes, _stream(dev))
     check(st, "cmc_decode_step")
     return out
+
+
+def tier1_gather(bank_k: torch.Tensor, bank_v: torch.Tensor, idx: torch.Tensor, *,
+                 out_k: Optional[torch.Tensor] = None, out_v: Optional[torch.Tensor] = None,
+                 workspace: Optional[DecodeWorkspace] = None
+                 ) -> Tuple[torch.Tensor, torch.Tensor]:
+    """Dense Tier-1 cache of the selected rows, bf16 [B, L, Hkv, k, d] each for
+    K and V; see cmc_tier1_gather.  Out-of-range indices raise
+    DEVFLAG_BAD_INDEX in ``workspace``'s status word when one is given."""
+    _need(bank_k, "bank_k", torch.bfloat16, 5)
+    dev = bank_k.device
+    _need(bank_v, "bank_v", torch.bfloat16, 5, dev)
+    _need(idx, "idx", torch.int32, 2, dev)
+    if bank_v.shape != bank_k.shape:
+        raise ValueError("bank_v must have the shape of bank_k")
+    B, L, Hkv, N, d = bank_k.shape
+    k = int(idx.shape[1])
+    if int(idx.shape[0]) != B:
+        raise ValueError(f"idx shape {tuple(idx.shape)} does not match batch {B}")
+    want = (B, L, Hkv, k, d)
+    if out_k is None:
+        out_k = torch.empty(want, dtype=torch.bfloat16, device=dev)
+    if out_v is None:
+        out_v = torch.empty(want, dtype=torch.bfloat16, device=dev)
+    for t, name in ((out_k, "out_k"), (out_v, "out_v")):
+        _need(t, name, torch.bfloat16, 5, dev)
+        if tuple(t.shape) != want:
+            raise ValueError(f"{name} must be {want}")
+    dims = CmcDims(B, L, Hkv, Hkv, d, N, k, 1)
+    status = None if workspace is None else workspace.buf
+    st = lib().cmc_tier1_gather(_p(bank_k), _p(bank_v), _p(idx), ctypes.byref(dims), _p(out_k),
+                                _p(out_v), _p(status), _stream(dev))
+    check(st, "cmc_tier1_gather")
+    return out_k, out_v
 
 
 def window_append(ring_k: torch.Tensor, ring_v: torch.Tensor, pos: torch.Tensor,

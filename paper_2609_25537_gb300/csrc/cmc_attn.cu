@@ -1,46 +1,77 @@
-// Tier-2 ring append and decode attention over the two-tier cache
-// (Section 2.5, "Tier-2: local context window" and "KV cache assembly"; cost
-// model in the appendix "Attention MACs Analysis").
+// Tier-2 ring append, Tier-1 gather and decode attention over the two-tier
+// cache (Section 2.5, "Tier-1", "Tier-2: local context window" and "KV cache
+// assembly"; cost model in the appendix "Attention MACs Analysis").
 //
-// Work decomposition: a unit is one (sequence b, layer l, KV head g).  Its
-// keys are the k Tier-1 rows gathered by idx followed by the occupied ring
-// slots; the key range is cut into `splits` chunks and one CTA handles one
-// (chunk, unit) pair (split-K / flash-decoding).  Inside a CTA each group of
-// d/8 lanes owns one key at a time and each lane one 16-byte slice of it
-// (8 bf16): keys of a warp step are adjacent rows, so a ring span is read as
-// contiguous 16-byte vectors and a gathered Tier-1 row as whole 256-byte
-// (d = 128) rows.  The G = Hq/Hkv query heads of the unit share every K/V
-// load.  Logits are reduced across the d/8 lanes with xor shuffles, the
-// softmax is an online (running max / sum) softmax in the log2 domain, and the
-// per-group (m, l, o) states are merged in shared memory.  With splits > 1 each
-// CTA writes its (m, l, o) partial to the workspace and the last CTA of the
-// unit to arrive (an atomic ticket, no waiting) merges the partials with a
-// log-sum-exp rescale and writes the bf16 output.
+// Work decomposition (stream-K over keys).  A unit is one (sequence b,
+// layer l, KV head g).  Its keys are cut into tiles of 64: ceil(k / 64)
+// Tier-1 tiles, then ceil(W / 64) tiles of ring slots; no tile mixes the two
+// tiers.  The flattened list of (unit, tile) pairs is split into equal
+// contiguous ranges, one per CTA, with the grid sized to the SMs that fit, so
+// every CTA streams the same number of bytes.  A CTA accumulates across the
+// tiles of a unit and writes the bf16 output of every unit it covers whole;
+// for a unit cut between CTAs each CTA writes an fp32 (max, sum, output)
+// partial record, and a small combine kernel that follows on the stream
+// merges the records with a log-sum-exp rescale.  The attention kernel has no
+// atomics, fences or inter-CTA waits.
 //
-// The fused decode step additionally appends the new token: every reader of
-// the ring slot being overwritten takes the new token's K/V from k_new/v_new
-// instead, the CTA whose chunk holds that slot stores it into the ring, and
-// the last CTA of the sequence to arrive (a second ticket) advances pos[b].
+// Inside a CTA one producer warp streams the tiles through a ring of shared-
+// memory stages.  Ring tiles, and Tier-1 tiles when the Tier-1 rows are the
+// first k rows of their tensor (the cache the prefill of M* leaves, or the
+// output of cmc_tier1_gather), are two 64-row x 64-column boxes per K and per
+// V loaded by the Tensor Memory Accelerator.  Tier-1 tiles gathered by an
+// index list are copied with 16-byte cp.async by the producer lanes.  Both
+// land in the 128-byte swizzled layout, which places 16-byte chunk c of a row
+// at position c ^ (row & 7) within its 128-byte line, so the consumers'
+// ldmatrix reads are conflict-free.  Rows that hold no key are masked, and
+// their V rows zeroed, so stale or unwritten memory never reaches the output.
+// The unit's query rows travel with each tile (1-D bulk copy) and a small
+// header written by the producer.  A stage is "full" when its TMA transaction
+// bytes (expect_tx / complete_tx) and its cp.async copies
+// (cp.async.mbarrier.arrive) have landed; four consumer warps, each owning 16
+// keys of a tile, compute
+//   S = Q K^T   with mma.sync m16n8k16 (query heads as the M rows: the G
+//               heads sharing the KV head, padded to 16),
+// an online softmax in the log2 domain (running max / sum per head), and
+//   O += P V    with mma.sync, P taken straight from the S accumulators,
+// reading K with ldmatrix and V with ldmatrix.trans, then hand the stage back
+// through an "empty" mbarrier.  Every mbarrier wait has an iteration limit.
+// Warps are merged in shared memory at the end of a unit.
+//
+// The fused decode step also appends the new token: the producer copies the
+// new token's K/V rows next to the tile that holds its ring slot, a consumer
+// warp patches them over the stale ring row in shared memory and stores them
+// into the ring, and the combine kernel advances pos[b] after the attention
+// kernel has finished.
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
+
+#include <cstring>
+#include <mutex>
 
 #include "cmc_internal.cuh"
 
 namespace cmc {
 
-constexpr int kAttnWarps = 4;
-constexpr int kAttnThreads = 32 * kAttnWarps;
-constexpr int kAttnUnroll = 4;
-constexpr int kMinChunk = 32;   // smallest chunk the split planner uses
-constexpr int kMaxChunk = 512;  // largest chunk (bounds the shared idx buffer)
+constexpr int kTileKeys = 64;  // keys per pipeline tile
+constexpr int kWarps = 4;      // consumer warps; each owns 16 keys of a tile
+constexpr int kThreads = 32 * kWarps;
 constexpr size_t kWsHeader = 256;
+constexpr int kHalfBytes = kTileKeys * 128;  // one 64-row x 128-byte swizzled box
+constexpr int kMetaSlots = 4;                // producer metadata prefetch distance (tiles)
+
+// Tensor maps of one launch (passed by value, in the kernel's parameter space).
+struct AttnMaps {
+  CUtensorMap rk_box, rv_box;      // ring [units * W, d], box 64 cols x 64 rows
+  CUtensorMap t1k_box, t1v_box;    // Tier-1 [units * N, d] (identity selection only)
+};
 
 struct AttnParams {
   const uint16_t* q;      // [B, L, Hq, d]
   const uint16_t* t1k;    // [B, L, Hkv, N, d]
   const uint16_t* t1v;    // [B, L, Hkv, N, d]
-  const int32_t* idx;     // [B, k]
+  const int32_t* idx;     // [B, k], or NULL: Tier-1 is rows 0 .. k-1 of t1k / t1v
   uint16_t* ring_k;       // [B, L, Hkv, W, d]
   uint16_t* ring_v;       // [B, L, Hkv, W, d]
   int64_t* pos;           // [B]
@@ -48,301 +79,746 @@ struct AttnParams {
   const uint16_t* v_new;  // [B, L, Hkv, d]
   uint16_t* out;          // [B, L, Hq, d]
   uint32_t* status;       // workspace status word
-  uint32_t* unit_ticket;  // [B * L * Hkv]
-  uint32_t* seq_ticket;   // [B]
-  float* partials;        // [units, splits, G * (d + 2)]
+  unsigned long long* tickets;  // [B] tiles whose pos read is done (fused step)
+  float* partials;        // [units, tpu, G * (d + 2)]
   int B, L, Hq, Hkv, N, k, W;
-  int splits, chunk;
+  int tpu;                // tiles per unit: t1_tiles Tier-1 tiles, then the ring tiles
+  int t1_tiles;           // ceil(k / 64)
+  int rot;                // in-unit processing order: tile (j + rot) % tpu at position j
+  long long base;         // tiles per CTA (CTAs below `rem` take one more)
+  long long rem;
   float scale_log2;       // softmax scale * log2(e)
 };
 
-// Split plan: number of chunks per unit and keys per chunk.
-struct SplitPlan {
-  int splits, chunk;
-};
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
 
-static int max_splits(int n_max) { return (n_max + kMinChunk - 1) / kMinChunk; }
-
-static SplitPlan plan_splits(long long units, int n_max) {
-  const long long target = 4LL * sm_count();
-  long long s = (target + units - 1) / units;
-  if (s < 1) s = 1;
-  if (s > max_splits(n_max)) s = max_splits(n_max);
-  int chunk = static_cast<int>((n_max + s - 1) / s);
-  chunk = (chunk + kMinChunk - 1) / kMinChunk * kMinChunk;
-  if (chunk > kMaxChunk) chunk = kMaxChunk;
-  if (chunk < kMinChunk) chunk = kMinChunk;
-  SplitPlan p;
-  p.chunk = chunk;
-  p.splits = (n_max + chunk - 1) / chunk;
-  if (p.splits < 1) p.splits = 1;
-  return p;
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+
+// C[16x8] += A[16x16] B[16x8], bf16 inputs, fp32 accumulators.  A rows 8..15
+// are the padding heads (always zero), so a1 = a3 = 0.
+__device__ __forceinline__ void mma_rows0to7(float (&c)[4], uint32_t a0, uint32_t a2, uint32_t b0,
+                                             uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+}
+
+// 2^x with the ex2.approx instruction (ex2(-inf) = +0).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Two fp32 -> bf16x2 (round to nearest even); `lo` lands in the low half.
+__device__ __forceinline__ uint32_t pack_bf16_rn(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;\n" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// --- mbarrier (shared::cta).  Every wait is bounded: after kMaxWaitSpins
+// failed polls the waiter reports CMC_DEVFLAG_TIMEOUT and gives up, so a
+// broken pipeline cannot hang the GPU.
+constexpr uint32_t kMaxWaitSpins = 1u << 22;
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(smem_addr(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}\n" ::"r"(
+                   smem_addr(bar))
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile(
+      "{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}\n" ::"r"(
+          smem_addr(bar)),
+      "r"(bytes)
+      : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Waits for the phase of `bar` with the given parity to complete; false on timeout.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (uint32_t it = 0; it < kMaxWaitSpins; ++it)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+// --- TMA loads into shared memory, completing on an mbarrier.
+__device__ __forceinline__ void tma_box(uint32_t dst, const CUtensorMap* map, int col, int row,
+                                        uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
+      "l"(map), "r"(col), "r"(row), "r"(smem_addr(bar))
+      : "memory");
+}
+__device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+// Named barrier over the consumer warps only (the producer warp never joins).
+__device__ __forceinline__ void consumer_sync() {
+  asm volatile("bar.sync 1, %0;\n" ::"n"(kWarps * 32) : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Shared-memory layout of one pipeline stage (1024-byte aligned)
+// ---------------------------------------------------------------------------
+
+template <int D, int G>
+struct Stage {
+  static constexpr int kHalves = D / 64;               // 128-byte column boxes per row
+  static constexpr int kK = 0;                         // K boxes [half][64 rows][128 B]
+  static constexpr int kV = kHalves * kHalfBytes;      // V boxes
+  static constexpr int kBytes = 2 * kHalves * kHalfBytes;  // a multiple of 1024
+  // Small per-stage areas, kept apart so that stages stay 1024-byte aligned:
+  static constexpr int kQ = 0;                         // query rows [G][D] bf16
+  static constexpr int kNew = G * D * 2;               // new token K row, V row (fused step)
+  static constexpr int kHdr = kNew + 2 * D * 2;        // header words (H_*)
+  static constexpr int kAuxBytes = kHdr + 128;
+};
+
+// Per-stage header words: rows of the tile that may hold a key, the new
+// token's ring slot and tile row (fused step; -1 if not in this tile),
+// whether any of the 64 rows holds no key (its V row must be zeroed), and the
+// bit masks of rows 0-31 / 32-63 whose Tier-1 index is out of range.
+enum { H_NROWS = 0, H_NEWSLOT = 1, H_NEWROW = 2, H_MASKED = 3, H_BADLO = 4, H_BADHI = 5 };
+
+template <int D, int G, int NST>
+constexpr size_t attn_smem_bytes() {
+  return 1024 /* alignment slack */ + static_cast<size_t>(NST) * (Stage<D, G>::kBytes + Stage<D, G>::kAuxBytes) +
+         kMetaSlots * (kTileKeys * 4 + 16) +
+         static_cast<size_t>(kWarps) * (2 * 8 + G * D) * sizeof(float);
+}
+
+// Byte offset of 16-byte chunk c (0 .. D/8-1) of tile row r within a K or V
+// region: 128-byte column box c / 8, swizzled position (c % 8) ^ (r % 8).
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+  return static_cast<uint32_t>((c >> 3) * kHalfBytes + r * 128 + (((c & 7) ^ (r & 7)) << 4));
+}
+
+__device__ __forceinline__ long long cta_first_tile(long long c, long long base, long long rem) {
+  return c * base + (c < rem ? c : rem);
+}
+__device__ __forceinline__ long long cta_of_tile(long long t, long long base, long long rem) {
+  const long long big = rem * (base + 1);
+  return t < big ? t / (base + 1) : rem + (t - big) / base;
+}
+
+// Unit coordinates of the tile at a position of the flattened (unit, j)
+// order, advanced one tile at a time so that the main loop does no integer
+// division.  Within a unit, position j holds key tile lt = (j + rot) % tpu:
+// the ring tiles come first, so a CTA's first loads need no idx entries.
+struct TileCursor {
+  int u, j, lt, b, l, g;  // unit, position and key tile within it, the unit's (b, l, g)
+  __device__ __forceinline__ void init(long long t, const AttnParams& p) {
+    const int LH = p.L * p.Hkv;
+    u = static_cast<int>(t / p.tpu);
+    j = static_cast<int>(t - static_cast<long long>(u) * p.tpu);
+    lt = j + p.rot;
+    if (lt >= p.tpu) lt -= p.tpu;
+    b = u / LH;
+    const int lg = u - b * LH;
+    l = lg / p.Hkv;
+    g = lg - l * p.Hkv;
+  }
+  __device__ __forceinline__ void next(const AttnParams& p) {
+    if (++j == p.tpu) {
+      j = 0;
+      ++u;
+      if (++g == p.Hkv) {
+        g = 0;
+        if (++l == p.L) {
+          l = 0;
+          ++b;
+        }
+      }
+    }
+    lt = j + p.rot;
+    if (lt >= p.tpu) lt -= p.tpu;
+  }
+};
+
+// What the producer needs to issue one tile -- the idx entries of its 64 rows
+// (gathered Tier-1 tiles only) and pos of its sequence -- staged in shared
+// memory by asynchronous 4- and 8-byte copies kMetaSlots tiles ahead of their
+// use, so the producer never waits on a global load.
+struct MetaSlot {
+  int32_t idx[kTileKeys];
+  long long pos;
+  long long pad;
+};
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes));
+}
+// Adds one pending arrival to `bar` now and completes it once every cp.async
+// this thread issued so far has landed.
+__device__ __forceinline__ void mbar_arrive_cp_async(uint64_t* bar) {
+  asm volatile("cp.async.mbarrier.arrive.shared::cta.b64 [%0];\n" ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes));
+}
+__device__ __forceinline__ void cp_async_8(uint32_t dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(dst), "l"(src));
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ bool gathered_tile(const AttnParams& p, const TileCursor& c) {
+  return p.idx != nullptr && c.lt < p.t1_tiles;
+}
+
+// Every producer lane commits exactly one copy group per call.
+__device__ __forceinline__ void prefetch_meta(const AttnParams& p, const TileCursor& c, bool live,
+                                              int lane, MetaSlot* slot) {
+  if (live) {
+    if (gathered_tile(p, c)) {
+      const int key0 = c.lt * kTileKeys;
+      const int32_t* irow = p.idx + static_cast<long long>(c.b) * p.k;
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int i = key0 + lane + 32 * e;
+        cp_async_4(smem_addr(&slot->idx[lane + 32 * e]), i < p.k ? irow + i : irow, i < p.k ? 4u : 0u);
+      }
+    }
+    if (lane == 0) cp_async_8(smem_addr(&slot->pos), p.pos + c.b);
+  }
+  cp_async_commit();
+}
+
+struct TileMeta {
+  long long pos;
+  int idx_lo, idx_hi;  // idx entries of rows lane and lane + 32 (gathered tiles)
+};
+
+// What a sequence's pos gives every tile of that sequence: the ring slots
+// that hold keys and the new token's slot (fused step).  Computed once per
+// run of tiles of one sequence.
+struct SeqState {
+  long long pos;
+  int count;     // occupied ring slots (after the append in the fused step)
+  int new_slot;  // ring slot of the new token, -1 if none
+  bool bad;      // pos < 0: the sequence is skipped
+};
+
+template <bool FUSED>
+__device__ __forceinline__ SeqState seq_state(const AttnParams& p, long long pos) {
+  SeqState q;
+  q.pos = pos;
+  q.bad = pos < 0;
+  q.count = 0;
+  q.new_slot = -1;
+  if (!q.bad) {
+    if (FUSED) {
+      q.count = static_cast<int>(pos + 1 < p.W ? pos + 1 : p.W);
+      q.new_slot = static_cast<int>(pos % p.W);
+    } else {
+      q.count = static_cast<int>(pos < p.W ? pos : p.W);
+    }
+  }
+  return q;
+}
+
+// Producer warp: everything for one tile -- its K/V loads, the header the
+// consumers read (rows that may hold keys, rows with a bad index, the new
+// token's row), the unit's query rows and, in the fused step, the new token's
+// K/V rows -- and the arrive that, once the bytes have landed, releases the
+// stage to the consumers.
 template <int D, int G, bool FUSED>
-__global__ void __launch_bounds__(kAttnThreads)
-two_tier_attn_kernel(const AttnParams p) {
-  constexpr int LPK = D / 8;                 // lanes per key
-  constexpr int KPW = 32 / LPK;              // keys per warp step
-  constexpr int GROUPS = kAttnWarps * KPW;   // key groups per CTA
-  constexpr int STEP = GROUPS * kAttnUnroll; // keys per CTA iteration
+__device__ __forceinline__ void produce_tile(const AttnParams& p, const AttnMaps& maps,
+                                             uint8_t* stage, uint8_t* aux, const TileCursor& c,
+                                             const TileMeta& meta, const SeqState& sq, int lane,
+                                             uint64_t* full) {
+  using S = Stage<D, G>;
+  constexpr int H = S::kHalves;
+  const bool t1 = c.lt < p.t1_tiles;
+  int n_rows, new_row = -1;
+  if (t1) {
+    n_rows = sq.bad ? 0 : min(p.k - c.lt * kTileKeys, kTileKeys);
+  } else {
+    const int slot0 = (c.lt - p.t1_tiles) * kTileKeys;  // ring slot of row 0
+    n_rows = min(max(sq.count - slot0, 0), kTileKeys);
+    if (FUSED && sq.new_slot >= slot0 && sq.new_slot - slot0 < n_rows) new_row = sq.new_slot - slot0;
+  }
+  const uint32_t sK = smem_addr(stage + S::kK);
+  const uint32_t sV = smem_addr(stage + S::kV);
+  uint32_t bad_lo = 0, bad_hi = 0;  // rows with an out-of-range index (gathered tiles)
+  const bool gath = t1 && p.idx != nullptr;
+  if (gath) {
+    // Tier-1 rows gathered by idx: 16-byte cp.async copies by the producer
+    // lanes (d/8 lanes sweep a row) to the swizzled positions; rows past k and
+    // rows with an out-of-range index are zero-filled.  Each lane's copies
+    // reach the full barrier through cp.async.mbarrier.arrive.
+    constexpr int LPR = D / 8;     // lanes per row
+    constexpr int RPP = 32 / LPR;  // rows per pass
+    const int chunk = lane % LPR;
+    const int rsub = lane / LPR;
+    const long long ubase = static_cast<long long>(c.u) * p.N * D + chunk * 8;
+#pragma unroll 8
+    for (int jj = 0; jj < kTileKeys / RPP; ++jj) {
+      const int r = jj * RPP + rsub;
+      const int row = __shfl_sync(0xffffffffu, (jj * RPP < 32) ? meta.idx_lo : meta.idx_hi, r & 31);
+      const bool ok = r < n_rows && static_cast<unsigned>(row) < static_cast<unsigned>(p.N);
+      const long long e = ubase + static_cast<long long>(ok ? row : 0) * D;
+      const uint32_t off = swz(r, chunk);
+      cp_async16(sK + off, p.t1k + e, ok ? 16u : 0u);
+      cp_async16(sV + off, p.t1v + e, ok ? 16u : 0u);
+    }
+    mbar_arrive_cp_async(full);
+    bad_lo = __ballot_sync(0xffffffffu, lane < n_rows && static_cast<unsigned>(meta.idx_lo) >= static_cast<unsigned>(p.N));
+    bad_hi = __ballot_sync(0xffffffffu, lane + 32 < n_rows && static_cast<unsigned>(meta.idx_hi) >= static_cast<unsigned>(p.N));
+    __syncwarp();
+  }
+  if (lane == 0) {
+    if (bad_lo | bad_hi) atomicOr(p.status, CMC_DEVFLAG_BAD_INDEX);
+    if (sq.bad && c.lt == 0) atomicOr(p.status, CMC_DEVFLAG_BAD_POS);
+    int* hw = reinterpret_cast<int*>(aux + S::kHdr);
+    hw[H_NROWS] = n_rows;
+    hw[H_NEWSLOT] = sq.new_slot;
+    hw[H_NEWROW] = new_row;
+    hw[H_MASKED] = (n_rows < kTileKeys || (bad_lo | bad_hi)) ? 1 : 0;
+    hw[H_BADLO] = static_cast<int>(bad_lo);
+    hw[H_BADHI] = static_cast<int>(bad_hi);
+    uint32_t tx = G * D * 2;  // query rows
+    if (new_row >= 0) tx += 2 * D * 2;
+    if (!gath) tx += 2 * H * kHalfBytes;
+    mbar_arrive_expect_tx(full, tx);  // releases the header; completes when the bytes land
+    if (!gath) {
+      // Two-dimensional boxes of 64 consecutive rows of the ring, or of the
+      // Tier-1 tensor under identity selection.  Rows past the unit's keys
+      // are masked; rows past the tensor are zero-filled by the TMA unit.
+      const int row = t1 ? c.u * p.N + c.lt * kTileKeys : c.u * p.W + (c.lt - p.t1_tiles) * kTileKeys;
+      const CUtensorMap* mk = t1 ? &maps.t1k_box : &maps.rk_box;
+      const CUtensorMap* mv = t1 ? &maps.t1v_box : &maps.rv_box;
+#pragma unroll
+      for (int h = 0; h < H; ++h) {
+        tma_box(sK + h * kHalfBytes, mk, h * 64, row, full);
+        tma_box(sV + h * kHalfBytes, mv, h * 64, row, full);
+      }
+    }
+    const uint16_t* qsrc =
+        p.q + ((static_cast<long long>(c.b) * p.L + c.l) * p.Hq + static_cast<long long>(c.g) * G) * D;
+    bulk_copy(smem_addr(aux + S::kQ), qsrc, G * D * 2, full);
+    if (new_row >= 0) {
+      bulk_copy(smem_addr(aux + S::kNew), p.k_new + static_cast<long long>(c.u) * D, D * 2, full);
+      bulk_copy(smem_addr(aux + S::kNew + D * 2), p.v_new + static_cast<long long>(c.u) * D, D * 2, full);
+    }
+  }
+}
 
-  __shared__ int s_idx[kMaxChunk];
-  __shared__ float s_m[GROUPS][G];
-  __shared__ float s_l[GROUPS][G];
-  __shared__ float s_o[GROUPS][G][D];
-  __shared__ int s_last;
+// Fused step: a CTA has read pos[b] for its run of `tiles` tiles of sequence
+// b.  The run that brings the sequence's count to all of its tiles is the last
+// reader of pos[b]; it advances pos[b] and clears the count for the next call.
+__device__ __forceinline__ void seq_run_done(const AttnParams& p, int b, long long tiles,
+                                             const SeqState& sq) {
+  const unsigned long long total = static_cast<unsigned long long>(p.L) * p.Hkv * p.tpu;
+  const unsigned long long old = atomicAdd(p.tickets + b, static_cast<unsigned long long>(tiles));
+  if (old + static_cast<unsigned long long>(tiles) == total) {
+    if (!sq.bad) p.pos[b] = sq.pos + 1;
+    p.tickets[b] = 0ull;
+  }
+}
 
-  const int split = blockIdx.x;
-  const int unit = blockIdx.y;
+// One CTA = kWarps consumer warps + 1 producer warp.  The producer streams
+// the CTA's tiles through NST shared-memory stages; stage s is handed over by
+// full[s] (its bytes have landed and its header is written) and handed back
+// by empty[s] (every consumer warp is done with it).
+template <int D, int G, bool FUSED, int NST>
+__global__ void __launch_bounds__(kThreads + 32)
+two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) {
+  using S = Stage<D, G>;
+  constexpr int KS = D / 16;  // k-steps of the Q K^T product
+  constexpr int NT = D / 8;   // n8 tiles of the output
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* aux0 = smem + NST * S::kBytes;                              // NST aux areas
+  uint8_t* meta0 = aux0 + NST * S::kAuxBytes;                          // kMetaSlots slots
+  float* merge_m = reinterpret_cast<float*>(meta0 + kMetaSlots * sizeof(MetaSlot));  // [kWarps][8]
+  float* merge_l = merge_m + kWarps * 8;                               // [kWarps][8]
+  float* merge_o = merge_l + kWarps * 8;                               // [kWarps][G][D]
+  __shared__ __align__(8) uint64_t full_bar[NST];
+  __shared__ __align__(8) uint64_t empty_bar[NST];
+
   const int tid = threadIdx.x;
   const int lane = tid & 31;
   const int warp = tid >> 5;
-  const int sub = lane / LPK;
-  const int kl = lane % LPK;
-  const int grp = warp * KPW + sub;
 
-  const int LH = p.L * p.Hkv;
-  const int b = unit / LH;
-  const int lg = unit - b * LH;
-  const int l = lg / p.Hkv;
-  const int g = lg - l * p.Hkv;
+  const long long cta = blockIdx.x;
+  const long long t_begin = cta_first_tile(cta, p.base, p.rem);
+  const long long t_end = t_begin + p.base + (cta < p.rem ? 1 : 0);
+  const int n_tiles = static_cast<int>(t_end - t_begin);
 
-  const long long pos_b = p.pos[b];
-  const bool bad_pos = pos_b < 0;
-  int count = 0, new_slot = -1;
-  if (!bad_pos) {
-    if (FUSED) {
-      count = static_cast<int>(pos_b + 1 < p.W ? pos_b + 1 : p.W);
-      new_slot = static_cast<int>(pos_b % p.W);
-    } else {
-      count = static_cast<int>(pos_b < p.W ? pos_b : p.W);
+  if (tid == 0) {
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&full_bar[s], 1);        // the producer's arrive (plus tracked cp.async arrivals)
+      mbar_init(&empty_bar[s], kWarps);  // one arrive per consumer warp
     }
-  }
-  const int k_eff = bad_pos ? 0 : p.k;
-  const int n_keys = k_eff + count;
-  const int kbeg = split * p.chunk;
-  const int kend = min(kbeg + p.chunk, n_keys);
-  if (bad_pos && split == 0 && tid == 0) atomicOr(p.status, CMC_DEVFLAG_BAD_POS);
-
-  // Tier-1 rows of this chunk
-  const int t1_end = min(kend, k_eff);
-  for (int i = kbeg + tid; i < t1_end; i += kAttnThreads) {
-    int r = p.idx[static_cast<long long>(b) * p.k + i];
-    if (r < 0 || r >= p.N) {
-      atomicOr(p.status, CMC_DEVFLAG_BAD_INDEX);
-      r = -1;
-    }
-    s_idx[i - kbeg] = r;
-  }
-
-  const long long unit_l = unit;
-  // Fused step: store the new token into its slot if this chunk owns the slot.
-  if (FUSED && !bad_pos) {
-    const int key_new = k_eff + new_slot;
-    if (key_new >= kbeg && key_new < kend) {
-      const uint4* sk = reinterpret_cast<const uint4*>(p.k_new + unit_l * D);
-      const uint4* sv = reinterpret_cast<const uint4*>(p.v_new + unit_l * D);
-      uint4* dk = reinterpret_cast<uint4*>(p.ring_k + (unit_l * p.W + new_slot) * D);
-      uint4* dv = reinterpret_cast<uint4*>(p.ring_v + (unit_l * p.W + new_slot) * D);
-      for (int v = tid; v < D / 8; v += kAttnThreads) {
-        dk[v] = sk[v];
-        dv[v] = sv[v];
-      }
-    }
-  }
-
-  // This lane's slice of the G query heads, pre-multiplied by scale*log2(e).
-  float qf[G][8];
-  {
-    const long long qbase = (static_cast<long long>(b) * p.L + l) * p.Hq + static_cast<long long>(g) * G;
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      const uint4 v = *reinterpret_cast<const uint4*>(p.q + (qbase + h) * D + kl * 8);
-      float f[8];
-      unpack8(v, f);
-#pragma unroll
-      for (int e = 0; e < 8; ++e) qf[h][e] = f[e] * p.scale_log2;
-    }
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
   __syncthreads();
+  // Programmatic dependent launch: everything above overlapped the previous
+  // kernel; inputs may be that kernel's outputs, so wait for it here.  Then let
+  // the combine kernel that follows launch early.
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 
-  float m[G], lsum[G], o[G][8];
+  if (warp == kWarps) {
+    // ======================= producer warp =======================
+    if (lane == 0) {
+      asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.rk_box) : "memory");
+      asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.rv_box) : "memory");
+      if (p.idx == nullptr && p.k > 0) {
+        asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.t1k_box) : "memory");
+        asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.t1v_box) : "memory");
+      }
+    }
+    TileCursor cm, ci;  // tile whose metadata is prefetched, tile issued
+    cm.init(t_begin, p);
+    ci = cm;
+    MetaSlot* slots = reinterpret_cast<MetaSlot*>(meta0);
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-    m[h] = -INFINITY;
-    lsum[h] = 0.f;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) o[h][e] = 0.f;
+    for (int m = 0; m < kMetaSlots; ++m) {
+      prefetch_meta(p, cm, m < n_tiles, lane, &slots[m]);
+      cm.next(p);
+    }
+    int issued = 0;
+    int run_b = -1;           // sequence of the current run of tiles
+    long long run_tiles = 0;  // tiles in that run so far
+    SeqState sq;
+    sq.pos = 0; sq.count = 0; sq.new_slot = -1; sq.bad = true;
+    for (int i = 0; i < n_tiles; ++i) {
+      const int s = i % NST;
+      if (i >= NST && !mbar_wait(&empty_bar[s], static_cast<uint32_t>((i / NST - 1) & 1))) {
+        if (lane == 0) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
+        break;
+      }
+      MetaSlot* ms = &slots[i % kMetaSlots];
+      cp_async_wait<kMetaSlots - 1>();  // this tile's metadata has landed
+      __syncwarp();
+      TileMeta meta;
+      meta.pos = ms->pos;
+      meta.idx_lo = meta.idx_hi = -1;
+      if (gathered_tile(p, ci)) {
+        meta.idx_lo = ms->idx[lane];
+        meta.idx_hi = ms->idx[lane + 32];
+      }
+      if (ci.b != run_b) {  // a new sequence: pos-derived state, once per run
+        if (FUSED && run_b >= 0 && lane == 0) seq_run_done(p, run_b, run_tiles, sq);
+        run_b = ci.b;
+        run_tiles = 0;
+        sq = seq_state<FUSED>(p, meta.pos);
+      }
+      ++run_tiles;
+      produce_tile<D, G, FUSED>(p, maps, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, meta, sq,
+                                lane, &full_bar[s]);
+      ci.next(p);
+      issued = i + 1;
+      __syncwarp();
+      prefetch_meta(p, cm, i + kMetaSlots < n_tiles, lane, ms);  // the slot just read
+      cm.next(p);
+    }
+    if (FUSED && run_b >= 0 && issued == n_tiles && lane == 0) seq_run_done(p, run_b, run_tiles, sq);
+    cp_async_wait<0>();
+    // Let this CTA's loads land before the warp exits (bounded).
+    if (issued > 0) mbar_wait(&full_bar[(issued - 1) % NST], static_cast<uint32_t>(((issued - 1) / NST) & 1));
+    return;
   }
 
-  const long long bank_row0 = unit_l * p.N;
-  const long long ring_row0 = unit_l * p.W;
-  for (int base = kbeg; base < kend; base += STEP) {
-    uint4 kr[kAttnUnroll], vr[kAttnUnroll];
-    bool valid[kAttnUnroll];
+  // ======================= consumer warps =======================
+  const int gq = lane >> 2;  // mma row (query head within the group)
+  const int tq = lane & 3;   // mma column pair
+  TileCursor cc;
+  cc.init(t_begin, p);
+  int cur_u = -1;
+  bool dead = false;
+  uint32_t qa[KS][2];
+  float m_run = -INFINITY, l_run = 0.f;
+  float o[NT][4];
 #pragma unroll
-    for (int u = 0; u < kAttnUnroll; ++u) {
-      const int i = base + u * GROUPS + grp;
-      const uint16_t* kp = nullptr;
-      const uint16_t* vp = nullptr;
-      if (i < kend) {
-        if (i < k_eff) {
-          const int r = s_idx[i - kbeg];
-          if (r >= 0) {
-            kp = p.t1k + (bank_row0 + r) * D;
-            vp = p.t1v + (bank_row0 + r) * D;
-          }
-        } else {
-          const int slot = i - k_eff;
-          if (FUSED && slot == new_slot) {
-            kp = p.k_new + unit_l * D;
-            vp = p.v_new + unit_l * D;
-          } else {
-            kp = p.ring_k + (ring_row0 + slot) * D;
-            vp = p.ring_v + (ring_row0 + slot) * D;
-          }
+  for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+#pragma unroll
+  for (int ks = 0; ks < KS; ++ks) qa[ks][0] = qa[ks][1] = 0u;
+
+  for (int i = 0; i < n_tiles; ++i) {
+    const int s = i % NST;
+    uint8_t* stage = smem + s * S::kBytes;
+    const uint8_t* aux = aux0 + s * S::kAuxBytes;
+    if (!dead && !mbar_wait(&full_bar[s], static_cast<uint32_t>((i / NST) & 1))) {
+      dead = true;
+      if (lane == 0) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
+    }
+    const int* hw = reinterpret_cast<const int*>(aux + S::kHdr);
+    const int u = cc.u;
+    const int n_rows = dead ? 0 : hw[H_NROWS];
+    const int new_row = dead ? -1 : hw[H_NEWROW];
+    // bit r: row r holds a key (the new token's row included)
+    const unsigned long long keys =
+        (n_rows >= kTileKeys ? ~0ull : ((1ull << n_rows) - 1ull)) &
+        ~((static_cast<unsigned long long>(static_cast<uint32_t>(hw[H_BADHI])) << 32) |
+          static_cast<uint32_t>(hw[H_BADLO]));
+    bool wrote_stage = false;  // generic-proxy writes into the stage by this warp
+
+    if (FUSED && new_row >= 0) {
+      // Patch the new token over its stale ring row (swizzled) and append it
+      // to the ring in global memory.  Warp 0 writes, all consumers wait.
+      if (warp == 0 && lane < 2 * (D / 8)) {
+        const int which = lane / (D / 8);  // 0: K, 1: V
+        const int c = lane - which * (D / 8);
+        const uint4 v = *reinterpret_cast<const uint4*>(aux + S::kNew + which * D * 2 + c * 16);
+        *reinterpret_cast<uint4*>(stage + (which ? S::kV : S::kK) + swz(new_row, c)) = v;
+        uint16_t* ring = which ? p.ring_v : p.ring_k;
+        *reinterpret_cast<uint4*>(ring + (static_cast<long long>(u) * p.W + hw[H_NEWSLOT]) * D + c * 8) = v;
+      }
+      consumer_sync();
+      wrote_stage = (warp == 0);
+    }
+
+    if (u != cur_u) {  // first tile of a unit in this CTA
+      cur_u = u;
+      const uint8_t* qs = aux + S::kQ;
+#pragma unroll
+      for (int ks = 0; ks < KS; ++ks) {
+        if (gq < G && !dead) {
+          qa[ks][0] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq) * 2);
+          qa[ks][1] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq + 8) * 2);
         }
       }
-      valid[u] = kp != nullptr;
-      if (valid[u]) {
-        kr[u] = ld_stream_u4(kp + kl * 8);
-        vr[u] = ld_stream_u4(vp + kl * 8);
-      } else {
-        kr[u] = make_uint4(0u, 0u, 0u, 0u);
-        vr[u] = make_uint4(0u, 0u, 0u, 0u);
-      }
+      m_run = -INFINITY;
+      l_run = 0.f;
+#pragma unroll
+      for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
     }
-#pragma unroll
-    for (int u = 0; u < kAttnUnroll; ++u) {
-      float kf[8];
-      unpack8(kr[u], kf);
-      float z[G];
-#pragma unroll
-      for (int h = 0; h < G; ++h) {
-        float acc = 0.f;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc = fmaf(qf[h][e], kf[e], acc);
-        z[h] = acc;
+
+    if (n_rows > 0) {
+      if (hw[H_MASKED]) {
+        // Zero the V rows of this warp's 16 keys that hold no key: their
+        // probabilities are 0, but the rows may hold stale or unwritten
+        // memory, and 0 times a non-finite value is not 0.
+        constexpr int CPR = D / 8;  // 16-byte chunks per row
+        for (int x = lane; x < 16 * CPR; x += 32) {
+          const int r = 16 * warp + x / CPR;
+          if (!((keys >> r) & 1ull))
+            *reinterpret_cast<uint4*>(stage + S::kV + swz(r, x % CPR)) = make_uint4(0u, 0u, 0u, 0u);
+        }
+        __syncwarp();
+        wrote_stage = true;
       }
+      const uint32_t sK = smem_addr(stage + S::kK);
+      const uint32_t sV = smem_addr(stage + S::kV);
+      // ---- S = Q K^T over this warp's 16 keys: two n8 blocks, two chains each ----
+      float sa[2][4], sb[2][4];
 #pragma unroll
-      for (int off = LPK / 2; off >= 1; off >>= 1) {
+      for (int nb = 0; nb < 2; ++nb)
 #pragma unroll
-        for (int h = 0; h < G; ++h) z[h] += __shfl_xor_sync(0xffffffffu, z[h], off);
+        for (int e = 0; e < 4; ++e) sa[nb][e] = sb[nb][e] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < KS; ks += 2) {
+#pragma unroll
+        for (int nb = 0; nb < 2; ++nb) {
+          const int key = 16 * warp + 8 * nb + (lane & 7);
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(sK + swz(key, 2 * ks + (lane >> 3)), b0, b1, b2, b3);
+          mma_rows0to7(sa[nb], qa[ks][0], qa[ks][1], b0, b1);
+          mma_rows0to7(sb[nb], qa[ks + 1][0], qa[ks + 1][1], b2, b3);
+        }
       }
-      if (valid[u]) {
-        float vf[8];
-        unpack8(vr[u], vf);
+      // ---- online softmax (log2 domain) ----
+      float v[2][2];
+      float mx = -INFINITY;
 #pragma unroll
-        for (int h = 0; h < G; ++h) {
-          if (z[h] > m[h]) {
-            const float a = exp2f(m[h] - z[h]);
-            lsum[h] *= a;
+      for (int nb = 0; nb < 2; ++nb) {
 #pragma unroll
-            for (int e = 0; e < 8; ++e) o[h][e] *= a;
-            m[h] = z[h];
-          }
-          const float pr = exp2f(z[h] - m[h]);
-          lsum[h] += pr;
+        for (int e = 0; e < 2; ++e) {
+          const int kk = 16 * warp + 8 * nb + 2 * tq + e;
+          const bool ok = (keys >> kk) & 1ull;
+          v[nb][e] = ok ? (sa[nb][e] + sb[nb][e]) * p.scale_log2 : -INFINITY;
+          mx = fmaxf(mx, v[nb][e]);
+        }
+      }
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float m_new = fmaxf(m_run, mx);
+      float alpha = 1.f;
+      float pr[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+      if (m_new != -INFINITY) {
+        alpha = ex2(m_run - m_new);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) o[h][e] = fmaf(pr, vf[e], o[h][e]);
+        for (int nb = 0; nb < 2; ++nb)
+#pragma unroll
+          for (int e = 0; e < 2; ++e) pr[nb][e] = ex2(v[nb][e] - m_new);
+      }
+      m_run = m_new;
+      l_run = l_run * alpha + (pr[0][0] + pr[0][1]) + (pr[1][0] + pr[1][1]);
+      if (!__all_sync(0xffffffffu, alpha == 1.f)) {
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+          o[j][0] *= alpha;
+          o[j][1] *= alpha;
+        }
+      }
+      // ---- O += P V ----
+      const uint32_t pa0 = pack_bf16_rn(pr[0][0], pr[0][1]);
+      const uint32_t pa2 = pack_bf16_rn(pr[1][0], pr[1][1]);
+      {
+        const int key = 16 * warp + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+        for (int j = 0; j < NT; j += 2) {
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(sV + swz(key, j + (lane >> 4)), b0, b1, b2, b3);
+          mma_rows0to7(o[j], pa0, pa2, b0, b1);
+          mma_rows0to7(o[j + 1], pa0, pa2, b2, b3);
         }
       }
     }
-  }
-
-  // Merge the key groups of this CTA.
-  if (kl == 0) {
-#pragma unroll
-    for (int h = 0; h < G; ++h) {
-      s_m[grp][h] = m[h];
-      s_l[grp][h] = lsum[h];
+    if (wrote_stage) {
+      // generic-proxy writes to this stage must be ordered before the
+      // producer's next TMA writes into it
+      asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
     }
-  }
-#pragma unroll
-  for (int h = 0; h < G; ++h) {
-#pragma unroll
-    for (int e = 0; e < 8; ++e) s_o[grp][h][kl * 8 + e] = o[h][e];
-  }
-  __syncthreads();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&empty_bar[s]);  // this warp is done with stage s
 
-  constexpr int PAIRS = G * D / 2;  // output element pairs of the unit
-  const long long out_base = ((static_cast<long long>(b) * p.L + l) * p.Hq + static_cast<long long>(g) * G) * D;
-  const int PW = G * (D + 2);       // floats per partial
-  float* my_part = p.partials + (unit_l * p.splits + split) * PW;
-
-  for (int t = tid; t < PAIRS; t += kAttnThreads) {
-    const int h = (2 * t) / D;
-    const int c = (2 * t) % D;
-    float M = -INFINITY;
+    // ---- end of a unit within this CTA: merge warps, write out or a partial ----
+    const bool unit_end = (i + 1 == n_tiles) || (cc.j == p.tpu - 1);
+    if (unit_end) {
+      l_run += __shfl_xor_sync(0xffffffffu, l_run, 1);
+      l_run += __shfl_xor_sync(0xffffffffu, l_run, 2);
+      if (gq < G) {
+        if (tq == 0) {
+          merge_m[warp * 8 + gq] = m_run;
+          merge_l[warp * 8 + gq] = l_run;
+        }
+        float* ow = merge_o + (warp * G + gq) * D;
 #pragma unroll
-    for (int q = 0; q < GROUPS; ++q) M = fmaxf(M, s_m[q][h]);
-    float Ls = 0.f, O0 = 0.f, O1 = 0.f;
-    if (M != -INFINITY) {
-#pragma unroll
-      for (int q = 0; q < GROUPS; ++q) {
-        const float f = exp2f(s_m[q][h] - M);
-        Ls = fmaf(f, s_l[q][h], Ls);
-        O0 = fmaf(f, s_o[q][h][c], O0);
-        O1 = fmaf(f, s_o[q][h][c + 1], O1);
+        for (int j = 0; j < NT; ++j) {
+          *reinterpret_cast<float2*>(ow + 8 * j + 2 * tq) = make_float2(o[j][0], o[j][1]);
+        }
       }
-    }
-    if (p.splits == 1) {
-      const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-      reinterpret_cast<uint32_t*>(p.out + out_base + h * D + c)[0] = pack_bf16x2(O0 * inv, O1 * inv);
-    } else {
-      if (c == 0) {
-        my_part[h] = M;
-        my_part[G + h] = Ls;
-      }
-      my_part[2 * G + h * D + c] = O0;
-      my_part[2 * G + h * D + c + 1] = O1;
-    }
-  }
+      consumer_sync();
 
-  bool unit_done = true;  // this CTA finishes the unit
-  if (p.splits > 1) {
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) {
-      const uint32_t ticket = atomicAdd(&p.unit_ticket[unit], 1u);
-      s_last = (ticket == static_cast<uint32_t>(p.splits - 1)) ? 1 : 0;
-    }
-    __syncthreads();
-    unit_done = s_last != 0;
-    if (unit_done) {
-      __threadfence();
-      const float* parts = p.partials + unit_l * p.splits * PW;
-      for (int t = tid; t < PAIRS; t += kAttnThreads) {
-        const int h = (2 * t) / D;
-        const int c = (2 * t) % D;
+      const long long c0 = cta_of_tile(static_cast<long long>(u) * p.tpu, p.base, p.rem);
+      const long long c1 = cta_of_tile(static_cast<long long>(u) * p.tpu + p.tpu - 1, p.base, p.rem);
+      const bool whole = (c0 == c1);
+      const int PW = G * (D + 2);
+      float* rec = p.partials + (static_cast<long long>(u) * p.tpu + (cta - c0)) * PW;
+      const long long out_base =
+          ((static_cast<long long>(cc.b) * p.L + cc.l) * p.Hq + static_cast<long long>(cc.g) * G) * D;
+      constexpr int PAIRS = G * D / 2;
+      for (int x = tid; x < PAIRS; x += kThreads) {
+        const int hh = (2 * x) / D;
+        const int c = (2 * x) % D;
         float M = -INFINITY;
-        for (int s = 0; s < p.splits; ++s) M = fmaxf(M, __ldcg(parts + s * PW + h));
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + hh]);
         float Ls = 0.f, O0 = 0.f, O1 = 0.f;
         if (M != -INFINITY) {
-          for (int s = 0; s < p.splits; ++s) {
-            const float* ps = parts + s * PW;
-            const float f = exp2f(__ldcg(ps + h) - M);
-            Ls = fmaf(f, __ldcg(ps + G + h), Ls);
-            O0 = fmaf(f, __ldcg(ps + 2 * G + h * D + c), O0);
-            O1 = fmaf(f, __ldcg(ps + 2 * G + h * D + c + 1), O1);
+#pragma unroll
+          for (int w = 0; w < kWarps; ++w) {
+            const float f = ex2(merge_m[w * 8 + hh] - M);
+            const float2 ow = *reinterpret_cast<const float2*>(merge_o + (w * G + hh) * D + c);
+            Ls = fmaf(f, merge_l[w * 8 + hh], Ls);
+            O0 = fmaf(f, ow.x, O0);
+            O1 = fmaf(f, ow.y, O1);
           }
         }
-        const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-        reinterpret_cast<uint32_t*>(p.out + out_base + h * D + c)[0] = pack_bf16x2(O0 * inv, O1 * inv);
+        if (whole) {
+          const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+          *reinterpret_cast<uint32_t*>(p.out + out_base + hh * D + c) = pack_bf16x2(O0 * inv, O1 * inv);
+        } else {  // merged by two_tier_combine_kernel
+          if (c == 0) {
+            rec[hh] = M;
+            rec[G + hh] = Ls;
+          }
+          *reinterpret_cast<float2*>(rec + 2 * G + hh * D + c) = make_float2(O0, O1);
+        }
       }
-      if (tid == 0) p.unit_ticket[unit] = 0u;
+      consumer_sync();  // merge buffers are reused by the next unit
     }
+    cc.next(p);
   }
+}
 
-  if (FUSED && unit_done && tid == 0) {
-    // Every CTA of this unit has read pos[b]; count the unit towards its sequence.
-    __threadfence();
-    const uint32_t t = atomicAdd(&p.seq_ticket[b], 1u);
-    if (t == static_cast<uint32_t>(LH - 1)) {
-      p.seq_ticket[b] = 0u;
-      if (!bad_pos) p.pos[b] = pos_b + 1;
+// Finishes the units that two_tier_attn_kernel split between CTAs: merges
+// their fp32 partial records (max, sum, output per head) with a log-sum-exp
+// rescale and writes the bf16 output.  Runs after two_tier_attn_kernel on the
+// same stream, only when some unit was split; one CTA per unit.
+template <int D, int G>
+__global__ void __launch_bounds__(kThreads)
+two_tier_combine_kernel(const AttnParams p) {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");  // the attention kernel's records
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+  const int u = blockIdx.x;
+  const int LH = p.L * p.Hkv;
+  const int b = u / LH;
+  const int lg = u - b * LH;
+  const int l = lg / p.Hkv;
+  const int g = lg - l * p.Hkv;
+  const long long c0 = cta_of_tile(static_cast<long long>(u) * p.tpu, p.base, p.rem);
+  const long long c1 = cta_of_tile(static_cast<long long>(u) * p.tpu + p.tpu - 1, p.base, p.rem);
+  if (c0 == c1) return;  // written by the attention kernel
+  const int nrec = static_cast<int>(c1 - c0 + 1);
+  const int PW = G * (D + 2);
+  const float* recs = p.partials + static_cast<long long>(u) * p.tpu * PW;
+  const long long out_base =
+      ((static_cast<long long>(b) * p.L + l) * p.Hq + static_cast<long long>(g) * G) * D;
+  for (int x = threadIdx.x; x < G * D / 2; x += blockDim.x) {
+    const int hh = (2 * x) / D;
+    const int c = (2 * x) % D;
+    float M = -INFINITY;
+    for (int r = 0; r < nrec; ++r) M = fmaxf(M, recs[r * PW + hh]);
+    float Ls = 0.f, O0 = 0.f, O1 = 0.f;
+    if (M != -INFINITY) {
+      for (int r = 0; r < nrec; ++r) {
+        const float* pr = recs + r * PW;
+        const float f = ex2(pr[hh] - M);
+        const float2 o2 = *reinterpret_cast<const float2*>(pr + 2 * G + hh * D + c);
+        Ls = fmaf(f, pr[G + hh], Ls);
+        O0 = fmaf(f, o2.x, O0);
+        O1 = fmaf(f, o2.y, O1);
+      }
     }
+    const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+    *reinterpret_cast<uint32_t*>(p.out + out_base + hh * D + c) = pack_bf16x2(O0 * inv, O1 * inv);
   }
 }
 
@@ -369,48 +845,187 @@ __global__ void window_append_kernel(uint16_t* __restrict__ ring_k, uint16_t* __
   if (threadIdx.x == 0 && pb >= 0) pos[b] = pb + 1;
 }
 
+// Tier-1 compaction (the "M*" of Section 2.5, formed once per question):
+//   tier1[b, l, g, i] = bank[b, l, g, idx[b, i]]   for i < k.
+// A CTA copies a block of kGatherRows output rows of one unit; each row's d/8
+// 16-byte chunks are read by consecutive threads.  Out-of-range indices give a
+// zero row and CMC_DEVFLAG_BAD_INDEX.
+constexpr int kGatherRows = 64;
+
+__device__ __forceinline__ uint4 ld_stream(const uint4* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+__global__ void __launch_bounds__(256)
+tier1_gather_kernel(const uint4* __restrict__ bank_k, const uint4* __restrict__ bank_v,
+                    const int32_t* __restrict__ idx, uint4* __restrict__ out_k,
+                    uint4* __restrict__ out_v, uint32_t* status, long long blocks, int row_blocks,
+                    int LH, int N, int k, int cpr) {
+  bool bad = false;
+  for (long long blk = blockIdx.x; blk < blocks; blk += gridDim.x) {
+    const long long u = blk / row_blocks;
+    const int i0 = static_cast<int>(blk - u * row_blocks) * kGatherRows;
+    const int nrow = min(kGatherRows, k - i0);
+    const int32_t* irow = idx + (u / LH) * k;
+    for (int x = threadIdx.x; x < nrow * cpr; x += blockDim.x) {
+      const int i = i0 + x / cpr;
+      const int c = x % cpr;
+      const int j = __ldg(irow + i);
+      uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
+      if (static_cast<unsigned>(j) < static_cast<unsigned>(N)) {
+        const long long src = (u * N + j) * cpr + c;
+        kv = ld_stream(bank_k + src);
+        vv = ld_stream(bank_v + src);
+      } else {
+        bad = true;
+      }
+      const long long dst = (u * k + i) * cpr + c;
+      out_k[dst] = kv;
+      out_v[dst] = vv;
+    }
+  }
+  if (bad && status) atomicOr(status, CMC_DEVFLAG_BAD_INDEX);
+}
+
 // ---------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------
 
 struct WsLayout {
   size_t tickets_off, partials_off, total;
-  int smax;
 };
 
+static int tier1_tiles(const cmc_dims& m) { return (m.k + kTileKeys - 1) / kTileKeys; }
+static int tiles_per_unit(const cmc_dims& m) { return tier1_tiles(m) + (m.W + kTileKeys - 1) / kTileKeys; }
+
+// [0, 256): status word; then one 8-byte pos-read count per sequence (padded
+// to 256 bytes); then one partial record per (unit, tile) slot.
 static WsLayout ws_layout(const cmc_dims& m) {
   WsLayout w;
   const long long units = static_cast<long long>(m.B) * m.L * m.Hkv;
-  const int n_max = m.k + m.W;
-  w.smax = max_splits(n_max);
   const int G = m.Hq / m.Hkv;
   w.tickets_off = kWsHeader;
-  w.partials_off = w.tickets_off + align_up(sizeof(uint32_t) * static_cast<size_t>(units + m.B), 256);
-  w.total = w.partials_off + static_cast<size_t>(units) * w.smax * G * (m.d + 2) * sizeof(float);
+  w.partials_off = w.tickets_off + ((static_cast<size_t>(m.B) * 8 + 255) / 256) * 256;
+  w.total = w.partials_off + static_cast<size_t>(units) * tiles_per_unit(m) * G * (m.d + 2) * sizeof(float);
   return w;
 }
 
+// cuTensorMapEncodeTiled, reached through the runtime's driver entry point.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(f);
+  });
+  return fn;
+}
+
+// A [rows, d] bf16 tensor viewed by boxes of 64 columns x box_rows rows,
+// 128-byte swizzle, zero fill outside the tensor.
+static bool encode_rows(CUtensorMap* map, const void* base, long long rows, int d, int box_rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * 2};
+  cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t es[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Pipeline depth: stages of 64 keys per CTA.  Three stages keep a CTA at
+// ~110 KB of shared memory at d = 128, G <= 4, so two CTAs share an SM.
+constexpr int kStages = 3;
+
 template <int D, int G, bool FUSED>
-static void launch_attn(const AttnParams& p, dim3 grid, cudaStream_t s) {
-  two_tier_attn_kernel<D, G, FUSED><<<grid, kAttnThreads, 0, s>>>(p);
+static int launch_attn(const AttnMaps& maps, const AttnParams& p0, long long total_tiles,
+                       cudaStream_t s) {
+  constexpr size_t smem = attn_smem_bytes<D, G, kStages>();
+  auto kern = two_tier_attn_kernel<D, G, FUSED, kStages>;
+  static int configured[64] = {0};  // per device: attribute set and occupancy known
+  int dev = 0;
+  int st = record_cuda_error(cudaGetDevice(&dev));
+  if (st != CMC_OK) return st;
+  int per_sm = (dev >= 0 && dev < 64) ? configured[dev] : 0;
+  if (per_sm <= 0) {
+    st = record_cuda_error(
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
+    if (st != CMC_OK) return st;
+    st = record_cuda_error(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads + 32, smem));
+    if (st != CMC_OK) return st;
+    if (per_sm < 1) per_sm = 1;
+    if (dev >= 0 && dev < 64) configured[dev] = per_sm;
+  }
+  AttnParams p = p0;
+  // Grid: with no more units than resident CTAs, a whole number of CTAs per
+  // unit (one per unit when they fit: no unit is split and no combine kernel
+  // runs); otherwise one wave of resident CTAs, each taking an equal share of
+  // the flattened tiles.
+  const long long slots = static_cast<long long>(per_sm) * sm_count();
+  const long long units = total_tiles / p.tpu;
+  long long ctas = units <= slots ? units * (slots / units) : slots;
+  if (ctas > total_tiles) ctas = total_tiles;
+  if (ctas < 1) ctas = 1;
+  p.base = total_tiles / ctas;
+  p.rem = total_tiles % ctas;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+  cfg.blockDim = dim3(kThreads + 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  st = record_cuda_error(cudaLaunchKernelEx(&cfg, kern, maps, p));
+  if (st != CMC_OK) return st;
+  // Is any unit split between CTAs (a CTA boundary inside a unit)?
+  bool split = false;
+  for (long long c = 1; c < ctas && !split; ++c) {
+    const long long t = c * p.base + (c < p.rem ? c : p.rem);
+    split = (t % p.tpu) != 0;
+  }
+  if (split) {
+    cfg.gridDim = dim3(static_cast<unsigned>(units));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = 0;
+    st = record_cuda_error(cudaLaunchKernelEx(&cfg, two_tier_combine_kernel<D, G>, p));
+  }
+  return st;
 }
 
 template <bool FUSED>
-static void dispatch_attn(const AttnParams& p, int d, int G, dim3 grid, cudaStream_t s) {
+static int dispatch_attn(const AttnMaps& maps, const AttnParams& p, int d, int G, long long tiles,
+                         cudaStream_t s) {
   if (d == 128) {
     switch (G) {
-      case 1: launch_attn<128, 1, FUSED>(p, grid, s); break;
-      case 2: launch_attn<128, 2, FUSED>(p, grid, s); break;
-      case 4: launch_attn<128, 4, FUSED>(p, grid, s); break;
-      default: launch_attn<128, 8, FUSED>(p, grid, s); break;
+      case 1: return launch_attn<128, 1, FUSED>(maps, p, tiles, s);
+      case 2: return launch_attn<128, 2, FUSED>(maps, p, tiles, s);
+      case 4: return launch_attn<128, 4, FUSED>(maps, p, tiles, s);
+      default: return launch_attn<128, 8, FUSED>(maps, p, tiles, s);
     }
-  } else {
-    switch (G) {
-      case 1: launch_attn<64, 1, FUSED>(p, grid, s); break;
-      case 2: launch_attn<64, 2, FUSED>(p, grid, s); break;
-      case 4: launch_attn<64, 4, FUSED>(p, grid, s); break;
-      default: launch_attn<64, 8, FUSED>(p, grid, s); break;
-    }
+  }
+  switch (G) {
+    case 1: return launch_attn<64, 1, FUSED>(maps, p, tiles, s);
+    case 2: return launch_attn<64, 2, FUSED>(maps, p, tiles, s);
+    case 4: return launch_attn<64, 4, FUSED>(maps, p, tiles, s);
+    default: return launch_attn<64, 8, FUSED>(maps, p, tiles, s);
   }
 }
 
@@ -423,7 +1038,6 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   if (st != CMC_OK) return st;
   const cmc_dims& m = *dims;
   if (!q || !tier1_k || !tier1_v || !ring_k || !ring_v || !pos || !out) return CMC_ERR_NULL;
-  if (m.k > 0 && !idx) return CMC_ERR_NULL;
   if (fused && (!k_new || !v_new)) return CMC_ERR_NULL;
   if (!aligned16(q) || !aligned16(tier1_k) || !aligned16(tier1_v) || !aligned16(ring_k) ||
       !aligned16(ring_v) || !aligned16(out))
@@ -436,14 +1050,27 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   if (!aligned16(workspace)) return CMC_ERR_ALIGN;
 
   const long long units = static_cast<long long>(m.B) * m.L * m.Hkv;
-  if (units > 65535) return CMC_ERR_SHAPE;  // grid.y limit
-  const SplitPlan plan = plan_splits(units, m.k + m.W);
+  const int tpu = tiles_per_unit(m);
+  const long long tiles = units * tpu;
+  // tile indices, unit ids and tensor-map row coordinates are 32-bit
+  if (tiles >= (1LL << 31) || units * m.N >= (1LL << 31) || units * m.W >= (1LL << 31))
+    return CMC_ERR_SHAPE;
+
+  AttnMaps maps;
+  memset(&maps, 0, sizeof(maps));
+  if (!encode_rows(&maps.rk_box, ring_k, units * m.W, m.d, kTileKeys) ||
+      !encode_rows(&maps.rv_box, ring_v, units * m.W, m.d, kTileKeys))
+    return CMC_ERR_CUDA;
+  if (!idx && m.k > 0 &&
+      (!encode_rows(&maps.t1k_box, tier1_k, units * m.N, m.d, kTileKeys) ||
+       !encode_rows(&maps.t1v_box, tier1_v, units * m.N, m.d, kTileKeys)))
+    return CMC_ERR_CUDA;
 
   AttnParams p;
   p.q = static_cast<const uint16_t*>(q);
   p.t1k = static_cast<const uint16_t*>(tier1_k);
   p.t1v = static_cast<const uint16_t*>(tier1_v);
-  p.idx = idx;
+  p.idx = m.k > 0 ? idx : nullptr;
   p.ring_k = static_cast<uint16_t*>(ring_k);
   p.ring_v = static_cast<uint16_t*>(ring_v);
   p.pos = pos;
@@ -452,21 +1079,20 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   p.out = static_cast<uint16_t*>(out);
   char* ws = static_cast<char*>(workspace);
   p.status = reinterpret_cast<uint32_t*>(ws);
-  p.unit_ticket = reinterpret_cast<uint32_t*>(ws + w.tickets_off);
-  p.seq_ticket = p.unit_ticket + units;
+  p.tickets = reinterpret_cast<unsigned long long*>(ws + w.tickets_off);
   p.partials = reinterpret_cast<float*>(ws + w.partials_off);
   p.B = m.B; p.L = m.L; p.Hq = m.Hq; p.Hkv = m.Hkv; p.N = m.N; p.k = m.k; p.W = m.W;
-  p.splits = plan.splits;
-  p.chunk = plan.chunk;
+  p.tpu = tpu;
+  p.t1_tiles = tier1_tiles(m);
+  p.rot = p.t1_tiles % tpu;  // the first ring tile
+  p.base = 0;
+  p.rem = 0;
   const float sc = scale > 0.f ? scale : 1.0f / sqrtf(static_cast<float>(m.d));
   p.scale_log2 = sc * 1.4426950408889634f;
-
-  const dim3 grid(static_cast<unsigned>(plan.splits), static_cast<unsigned>(units));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int G = m.Hq / m.Hkv;
-  if (fused) dispatch_attn<true>(p, m.d, G, grid, s);
-  else dispatch_attn<false>(p, m.d, G, grid, s);
-  return check_launch();
+  return fused ? dispatch_attn<true>(maps, p, m.d, G, tiles, s)
+               : dispatch_attn<false>(maps, p, m.d, G, tiles, s);
 }
 
 }  // namespace cmc
@@ -493,6 +1119,31 @@ int cmc_decode_step(const void* q, const void* tier1_k, const void* tier1_v, con
                     size_t workspace_bytes, void* stream) {
   return cmc::run_attention(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, dims,
                             scale, out, workspace, workspace_bytes, stream, true);
+}
+
+int cmc_tier1_gather(const void* bank_k, const void* bank_v, const int32_t* idx,
+                     const cmc_dims* dims, void* tier1_k, void* tier1_v, uint32_t* status,
+                     void* stream) {
+  using namespace cmc;
+  if (!dims) return CMC_ERR_NULL;
+  cmc_dims m = *dims;
+  m.Hq = m.Hkv;  // query heads play no part here
+  int st = validate_dims(&m, true);
+  if (st != CMC_OK) return st;
+  if (m.k == 0) return CMC_OK;
+  if (!bank_k || !bank_v || !idx || !tier1_k || !tier1_v) return CMC_ERR_NULL;
+  if (!aligned16(bank_k) || !aligned16(bank_v) || !aligned16(tier1_k) || !aligned16(tier1_v) ||
+      (reinterpret_cast<uintptr_t>(idx) & 3) || (reinterpret_cast<uintptr_t>(status) & 3))
+    return CMC_ERR_ALIGN;
+  const long long units = static_cast<long long>(m.B) * m.L * m.Hkv;
+  const int row_blocks = (m.k + kGatherRows - 1) / kGatherRows;
+  const long long blocks = units * row_blocks;
+  const long long grid = blocks < (1LL << 30) ? blocks : (1LL << 30);
+  tier1_gather_kernel<<<static_cast<unsigned>(grid), 256, 0, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<const uint4*>(bank_k), static_cast<const uint4*>(bank_v), idx,
+      static_cast<uint4*>(tier1_k), static_cast<uint4*>(tier1_v), status, blocks, row_blocks,
+      m.L * m.Hkv, m.N, m.k, m.d / 8);
+  return check_launch();
 }
 
 int cmc_window_append(void* ring_k, void* ring_v, int64_t* pos, const void* k_new,

@@ -109,7 +109,8 @@ def test_attention_argument_checks(L):
     assert _attn(L, _dims(k=101)) == RANGE
     assert _attn(L, _dims(k=-1)) == RANGE
     assert _attn(L, _dims(), q=0) == NULL
-    assert _attn(L, _dims(), idx=0) == NULL
+    # idx NULL is identity selection (Tier-1 = rows 0 .. k-1): not an error
+    assert _attn(L, _dims(), idx=0) not in (NULL, SHAPE, RANGE, ALIGN, WORKSPACE)
     assert _attn(L, _dims(), out=0) == NULL
     assert _attn(L, _dims(), q=FAKE + 2) == ALIGN
     assert _attn(L, _dims(), pos=FAKE + 4) == ALIGN
@@ -132,13 +133,23 @@ def test_window_append_argument_checks(L):
 
 
 def test_attention_workspace_size(L):
+    # a 256-byte status header, 8 bytes per sequence padded to 256, then one
+    # fp32 partial record of G * (d + 2) floats per (unit, 64-key tile) slot;
+    # a unit has ceil(k / 64) Tier-1 tiles and ceil(W / 64) ring tiles
     d = _dims()
-    n = L.cmc_decode_attn_workspace_size(ctypes.byref(d))
     units = 2 * 3 * 2
-    smax = -(-(10 + 16) // 32)
     G = 4
-    tickets = -(-(4 * (units + 2)) // 256) * 256
-    assert n == 256 + tickets + units * smax * G * (128 + 2) * 4
+    n = L.cmc_decode_attn_workspace_size(ctypes.byref(d))
+    assert n == 256 + 256 + units * (1 + 1) * G * (128 + 2) * 4
+    big = _dims(k=100, W=1000)
+    assert L.cmc_decode_attn_workspace_size(ctypes.byref(big)) == (
+        256 + 256 + units * (2 + 16) * G * (128 + 2) * 4)
+    none = _dims(k=0, W=64)
+    assert L.cmc_decode_attn_workspace_size(ctypes.byref(none)) == (
+        256 + 256 + units * (0 + 1) * G * (128 + 2) * 4)
+    many = _dims(B=40, Hkv=1, Hq=1, L=1, k=0, W=64)
+    assert L.cmc_decode_attn_workspace_size(ctypes.byref(many)) == (
+        256 + 512 + 40 * 1 * 1 * (128 + 2) * 4)
     assert L.cmc_decode_attn_workspace_size(ctypes.byref(_dims(d=80))) == 0
 
 
@@ -152,3 +163,21 @@ def test_binding_rejects_cpu_tensors():
     import torch
     with pytest.raises(ValueError, match="CUDA"):
         cmc.score_select(torch.zeros(1, 8), torch.zeros(1, 4, 8), 2)
+
+
+@host_only
+def test_tier1_gather_argument_checks(L):
+    d = _dims()
+    def g(bank=FAKE, idx=FAKE, out=FAKE, status=0, dims=d):
+        return L.cmc_tier1_gather(bank, FAKE, idx, ctypes.byref(dims), out, FAKE, status, None)
+    assert g(bank=0) == NULL
+    assert g(idx=0) == NULL
+    assert g(out=0) == NULL
+    assert g(bank=FAKE + 8) == ALIGN
+    assert g(idx=FAKE + 2) == ALIGN
+    assert g(status=FAKE + 2) == ALIGN
+    assert g(dims=_dims(k=101)) == RANGE
+    assert g(dims=_dims(d=32)) == SHAPE
+    assert g(dims=_dims(Hq=3)) not in (SHAPE,)  # query heads are ignored
+    assert g(bank=0, idx=0, out=0, dims=_dims(k=0)) == 0  # k = 0: nothing to do
+    assert L.cmc_tier1_gather(FAKE, FAKE, FAKE, None, FAKE, FAKE, 0, None) == NULL

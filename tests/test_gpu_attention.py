@@ -3,7 +3,11 @@ oracle, on the seeded workloads and on edge cases.
 
 Full-size workloads run every decode step on the GPU and compare every head
 of every layer at sampled steps (first steps, around the ring's wrap, middle,
-last), with the oracle replaying the same appends."""
+last), with the oracle replaying the same appends.
+
+Both Tier-1 forms are covered: "gather" passes the per-CME bank and idx to
+every step; "dense" compacts the selected rows once with tier1_gather and
+passes idx=None.  The oracle always gathers from the bank itself."""
 
 import numpy as np
 import pytest
@@ -19,10 +23,17 @@ from _gpu_helpers import assert_attn_close, dev_bf16, host_bits, to_f64
 pytestmark = pytest.mark.gpu
 
 
-class Problem:
-    """Device and host (oracle) copies of one decode problem."""
+MODES = ["gather", "dense"]
 
-    def __init__(self, w, dev, idx=None):
+
+class Problem:
+    """Device and host (oracle) copies of one decode problem.
+
+    mode "gather": the attention calls get the bank and idx; "dense": the
+    selected rows are compacted once by tier1_gather (checked bit-exact
+    against indexing the host bank) and the calls get idx=None."""
+
+    def __init__(self, w, dev, idx=None, mode="gather"):
         self.w = w
         self.dev = dev
         kv = kv_inputs(w)
@@ -30,9 +41,16 @@ class Problem:
         if idx is None and w.k > 0:
             idx = random_tier1_indices(w)
         self.idx_host = None if w.k == 0 else np.asarray(idx, dtype=np.int64)
-        self.idx = None if w.k == 0 else torch.from_numpy(
-            np.asarray(idx, dtype=np.int32)).to(dev)
+        self.idx = (torch.empty((w.B, 0), dtype=torch.int32, device=dev) if w.k == 0 else
+                    torch.from_numpy(np.asarray(idx, dtype=np.int32)).to(dev))
         self.t1k, self.t1v = dev_bf16(kv.tier1_k, dev), dev_bf16(kv.tier1_v, dev)
+        self.mode = mode if w.k > 0 else "gather"
+        if self.mode == "dense":
+            self.t1k, self.t1v = cmc.tier1_gather(self.t1k, self.t1v, self.idx)
+            for dev_t, host in ((self.t1k, kv.tier1_k), (self.t1v, kv.tier1_v)):
+                want = np.stack([host[b][:, :, self.idx_host[b]] for b in range(w.B)])
+                np.testing.assert_array_equal(host_bits(dev_t), want)
+            self.idx = None
         self.ring_k, self.ring_v = dev_bf16(kv.ring_k, dev), dev_bf16(kv.ring_v, dev)
         self.pos = torch.from_numpy(kv.pos0.copy()).to(dev)
         self.o_ring_k, self.o_ring_v = kv.ring_k.copy(), kv.ring_v.copy()
@@ -64,11 +82,12 @@ class Problem:
         assert self.ws.status() == 0
 
 
-def test_tiny_every_step(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_tiny_every_step(cuda_device, mode):
     w = WORKLOADS["tiny"]
     si = selection_inputs(w)
     idx_ref, _ = oracle.score_select(si.question_emb, si.cme_bank, w.k)
-    P = Problem(w, cuda_device, idx=idx_ref)
+    P = Problem(w, cuda_device, idx=idx_ref, mode=mode)
     for t in range(w.T):
         out, ref = P.step(step_inputs(w, t))
         assert_attn_close(to_f64(out), ref, f"tiny step {t}")
@@ -85,8 +104,8 @@ def test_tiny_peaked(cuda_device, q_scale):
         assert_attn_close(to_f64(out), ref, f"tiny peaked step {t}")
 
 
-def _sampled_run(w, dev, sample_steps, idx=None, q_std=None):
-    P = Problem(w, dev, idx=idx)
+def _sampled_run(w, dev, sample_steps, idx=None, q_std=None, mode="gather"):
+    P = Problem(w, dev, idx=idx, mode=mode)
     q_fill = dev_bf16(step_inputs(w, 0, parts="q", q_std=q_std).q, dev)
     sample_steps = set(sample_steps)
     for t in range(w.T):
@@ -104,7 +123,8 @@ def _samples(w):
     return sorted({0, 1, 2, w.W - 1, w.W, w.W + 1, w.T // 2, w.T - 1} & set(range(w.T)))
 
 
-def test_llama3_8b_full(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_llama3_8b_full(cuda_device, mode):
     """The 32-layer Llama-3-8B-shaped workload, all 3,000 steps, with the
     selection taken from the Tier-1 scoring of its own CME bank."""
     w = WORKLOADS["llama3_8b"]
@@ -114,34 +134,39 @@ def test_llama3_8b_full(cuda_device):
     idx_host = idx.cpu().numpy()
     np.testing.assert_array_equal(idx_host, oracle.score_select(si.question_emb, si.cme_bank,
                                                                 w.k)[0])
-    _sampled_run(w, cuda_device, _samples(w), idx=idx_host)
+    _sampled_run(w, cuda_device, _samples(w), idx=idx_host, mode=mode)
 
 
-def test_llama3_8b_peaked(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_llama3_8b_peaked(cuda_device, mode):
     w = WORKLOADS["llama3_8b"].with_(T=3, L=4)
-    _sampled_run(w, cuda_device, range(3), q_std=3.0 / w.kv_std)
+    _sampled_run(w, cuda_device, range(3), q_std=3.0 / w.kv_std, mode=mode)
 
 
-def test_mistral_batched_full(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_mistral_batched_full(cuda_device, mode):
     w = WORKLOADS["mistral_batched"]
-    _sampled_run(w, cuda_device, _samples(w))
+    _sampled_run(w, cuda_device, _samples(w), mode=mode)
 
 
-def test_long_context_full(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_long_context_full(cuda_device, mode):
     w = WORKLOADS["long_context"]
-    _sampled_run(w, cuda_device, _samples(w))
+    _sampled_run(w, cuda_device, _samples(w), mode=mode)
 
 
+@pytest.mark.parametrize("mode", MODES)
 @pytest.mark.parametrize("w", ablation_workloads(L=1, T=3), ids=lambda w: w.name)
-def test_ablation_grid(cuda_device, w):
-    _sampled_run(w, cuda_device, [0, w.T - 1])
+def test_ablation_grid(cuda_device, w, mode):
+    _sampled_run(w, cuda_device, [0, w.T - 1], mode=mode)
 
 
-def test_all_cmes_unbounded_window_is_plain_attention(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_all_cmes_unbounded_window_is_plain_attention(cuda_device, mode):
     """k = N and a window that never evicts: GPU output equals the oracle and
     plain softmax attention over [whole bank | every token so far]."""
     w = full_window_workload(B=2, T=6)
-    P = Problem(w, cuda_device, idx=np.tile(np.arange(w.N), (w.B, 1)))
+    P = Problem(w, cuda_device, idx=np.tile(np.arange(w.N), (w.B, 1)), mode=mode)
     hist_k = [list(P.kv.ring_k[b, :, :, :P.kv.pos0[b]].transpose(2, 0, 1, 3))
               for b in range(w.B)]
     hist_v = [list(P.kv.ring_v[b, :, :, :P.kv.pos0[b]].transpose(2, 0, 1, 3))
@@ -169,11 +194,12 @@ def test_all_cmes_unbounded_window_is_plain_attention(cuda_device):
             assert_attn_close(got[b, l, h], plain, "plain attention")
 
 
-def test_fused_step_equals_append_then_attend(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_fused_step_equals_append_then_attend(cuda_device, mode):
     """The fused step and the two separate calls give bit-identical results."""
     for w in (WORKLOADS["tiny"], WORKLOADS["llama3_8b"].with_(L=2, T=3)):
-        A = Problem(w, cuda_device)
-        Bp = Problem(w, cuda_device)
+        A = Problem(w, cuda_device, mode=mode)
+        Bp = Problem(w, cuda_device, mode=mode)
         for t in range(3):
             st = step_inputs(w, t)
             q = dev_bf16(st.q, cuda_device)
@@ -189,42 +215,46 @@ def test_fused_step_equals_append_then_attend(cuda_device):
             assert torch.equal(A.ring_k, Bp.ring_k) and torch.equal(A.pos, Bp.pos)
 
 
-def test_deterministic(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_deterministic(cuda_device, mode):
     w = WORKLOADS["llama3_8b"].with_(L=2)
     outs = []
     for _ in range(2):
-        P = Problem(w, cuda_device)
+        P = Problem(w, cuda_device, mode=mode)
         st = step_inputs(w, 0)
         out, _ = P.step(st, compare=False)
         outs.append(out.view(torch.int16).clone())
     assert torch.equal(outs[0], outs[1])
 
 
+@pytest.mark.parametrize("mode", MODES)
 @pytest.mark.parametrize("G,d", [(1, 64), (2, 128), (8, 64), (8, 128), (4, 64)])
-def test_head_shapes(cuda_device, G, d):
+def test_head_shapes(cuda_device, G, d, mode):
     Hkv = 2
     w = WORKLOADS["tiny"].with_(B=2, L=3, Hq=G * Hkv, Hkv=Hkv, d=d, N=70, k=9, W=33, T=4,
                                 kv_std=1.0, q_std=1.0 / np.sqrt(d), W0=(33, 5))
-    P = Problem(w, cuda_device)
+    P = Problem(w, cuda_device, mode=mode)
     for t in range(w.T):
         out, ref = P.step(step_inputs(w, t))
         assert_attn_close(to_f64(out), ref, f"G={G} d={d} step {t}")
     P.check_state()
 
 
-def test_ragged_fill_and_wrap(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_ragged_fill_and_wrap(cuda_device, mode):
     """Sequences at different ring fills, including empty, crossing the wrap."""
     w = WORKLOADS["tiny"].with_(B=5, W=16, k=7, T=20, W0=(0, 1, 9, 15, 16))
-    P = Problem(w, cuda_device)
+    P = Problem(w, cuda_device, mode=mode)
     for t in range(w.T):
         out, ref = P.step(step_inputs(w, t))
         assert_attn_close(to_f64(out), ref, f"ragged step {t}")
     P.check_state()
 
 
-def test_window_of_one(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_window_of_one(cuda_device, mode):
     w = WORKLOADS["tiny"].with_(W=1, k=3, T=5)
-    P = Problem(w, cuda_device)
+    P = Problem(w, cuda_device, mode=mode)
     for t in range(w.T):
         out, ref = P.step(step_inputs(w, t))
         assert_attn_close(to_f64(out), ref, f"W=1 step {t}")
@@ -236,7 +266,7 @@ def test_k_zero_and_empty_cache(cuda_device):
     P = Problem(w, cuda_device)
     # attention without append on an empty ring: zero output for sequence 0
     st = step_inputs(w, 0)
-    out = cmc.two_tier_decode_attn(dev_bf16(st.q, cuda_device), P.t1k, P.t1v, None, P.ring_k,
+    out = cmc.two_tier_decode_attn(dev_bf16(st.q, cuda_device), P.t1k, P.t1v, P.idx, P.ring_k,
                                    P.ring_v, P.pos, workspace=P.ws)
     ref = oracle.two_tier_attention(st.q, P.kv.tier1_k, P.kv.tier1_v, None, P.o_ring_k,
                                     P.o_ring_v, P.o_pos)
@@ -249,11 +279,12 @@ def test_k_zero_and_empty_cache(cuda_device):
     P.check_state()
 
 
-def test_unsorted_idx_and_explicit_scale(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_unsorted_idx_and_explicit_scale(cuda_device, mode):
     w = WORKLOADS["tiny"].with_(T=2)
     idx = random_tier1_indices(w)
     perm = np.random.default_rng(0).permutation(w.k)
-    P = Problem(w, cuda_device, idx=idx[:, perm])
+    P = Problem(w, cuda_device, idx=idx[:, perm], mode=mode)
     for t in range(w.T):
         out, ref = P.step(step_inputs(w, t), scale=0.05)
         assert_attn_close(to_f64(out), ref, f"unsorted idx step {t}")
@@ -289,10 +320,11 @@ def test_bad_index_and_bad_pos_are_flagged_and_skipped(cuda_device):
             assert_attn_close(got[b, 0, h], ref, f"bad idx b={b} h={h}")
 
 
-def test_large_unit_count(cuda_device):
+@pytest.mark.parametrize("mode", MODES)
+def test_large_unit_count(cuda_device, mode):
     """B * L * Hkv = 16,384 units in one launch (batch 64, 32 layers)."""
     w = WORKLOADS["llama3_8b"].with_(B=64, L=32, N=40, k=8, W=24, T=1, W0=None)
-    P = Problem(w, cuda_device)
+    P = Problem(w, cuda_device, mode=mode)
     st = step_inputs(w, 0)
     out, _ = P.step(st, compare=False)
     got = to_f64(out)
@@ -304,3 +336,41 @@ def test_large_unit_count(cuda_device):
                                              ring_k, ring_v, pos, b, l, h)
         assert_attn_close(got[b, l, h], ref, f"unit sample {(b, l, h)}")
     P.check_state()
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_unoccupied_slots_holding_nan_do_not_leak(cuda_device, mode):
+    """Ring slots past the fill (and so outside the cache) hold NaN on the
+    device: masked keys must not reach the output, whatever memory holds."""
+    w = WORKLOADS["tiny"].with_(B=3, W=100, k=40, T=3, W0=(0, 37, 64))
+    P = Problem(w, cuda_device, mode=mode)
+    nan = torch.tensor(0x7FC0, dtype=torch.int16).view(torch.bfloat16).to(cuda_device)
+    for b, f in enumerate(w.fill()):
+        P.ring_k[b, :, :, f:] = nan
+        P.ring_v[b, :, :, f:] = nan
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t))
+        got = to_f64(out)
+        assert np.isfinite(got).all()
+        assert_attn_close(got, ref, f"NaN-filled free slots step {t}")
+
+
+def test_tier1_gather_bad_index_zero_row_and_flag(cuda_device):
+    w = WORKLOADS["tiny"].with_(B=2, L=2)
+    kv = kv_inputs(w)
+    idx = random_tier1_indices(w).astype(np.int32)
+    idx[1, 5] = w.N
+    idx[0, 0] = -3
+    dims = cmc.dims_of(torch.empty(w.B, w.L, w.Hq, w.d, dtype=torch.bfloat16),
+                       torch.empty(w.B, w.L, w.Hkv, w.N, w.d, dtype=torch.bfloat16),
+                       None, torch.empty(w.B, w.L, w.Hkv, w.W, w.d, dtype=torch.bfloat16))
+    ws = cmc.DecodeWorkspace(dims, cuda_device)
+    tk, tv = cmc.tier1_gather(dev_bf16(kv.tier1_k, cuda_device), dev_bf16(kv.tier1_v, cuda_device),
+                              torch.from_numpy(idx).to(cuda_device), workspace=ws)
+    assert ws.status() == cmc.DEVFLAG_BAD_INDEX
+    for dev_t, host in ((tk, kv.tier1_k), (tv, kv.tier1_v)):
+        got = host_bits(dev_t)
+        for b in range(w.B):
+            for i, j in enumerate(idx[b]):
+                want = host[b][:, :, j] if 0 <= j < w.N else 0
+                np.testing.assert_array_equal(got[b][:, :, i], want)
