@@ -496,8 +496,8 @@ def run_gpu(args, w, world, rank, local):
         "variant": variant,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
-                     "kernel": ("fused decode step: two_tier_attn_kernel<128,4,fused> + "
-                                "two_tier_combine_kernel"),
+                     "kernel": ("fused decode step: two_tier_attn_kernel<128,4,fused,3> "
+                                "(one CTA per unit; no combine launch at this shape)"),
                      "bytes_per_launch": nbytes, "traffic": profiled_traffic(),
                      "flops_per_launch": decode_step_flops(w.B, w.L, w.Hq, w.d, w.k, w.W)},
         "select_roofline": {"bound": "hbm", "bytes": select_bytes(w.B, w.N, w.D, w.k),

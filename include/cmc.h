@@ -139,9 +139,11 @@ CMC_API int cmc_window_append(void* ring_k, void* ring_v, int64_t* pos, const vo
  * ------------------------------------------------------------------------ */
 
 /* Bytes of workspace the two attention entry points need for `dims`.  The
- * workspace starts with the device status word (read by cmc_read_status),
- * which must be zero before the first call: zero-fill the workspace once.
- * The rest holds fp32 partial results that each call writes before reading. */
+ * workspace holds the device status word (read by cmc_read_status), one
+ * 8-byte counter per sequence that the fused step uses to advance pos, and
+ * fp32 partial results.  Zero-fill it once before its first use; every call
+ * leaves the counters at zero again.  After a call that raised
+ * CMC_DEVFLAG_TIMEOUT, zero-fill it again. */
 CMC_API size_t cmc_decode_attn_workspace_size(const cmc_dims* dims);
 
 /*

@@ -2,17 +2,18 @@
 // cache (Section 2.5, "Tier-1", "Tier-2: local context window" and "KV cache
 // assembly"; cost model in the appendix "Attention MACs Analysis").
 //
-// Work decomposition (stream-K over keys).  A unit is one (sequence b,
-// layer l, KV head g).  Its keys are cut into tiles of 64: ceil(k / 64)
-// Tier-1 tiles, then ceil(W / 64) tiles of ring slots; no tile mixes the two
-// tiers.  The flattened list of (unit, tile) pairs is split into equal
-// contiguous ranges, one per CTA, with the grid sized to the SMs that fit, so
-// every CTA streams the same number of bytes.  A CTA accumulates across the
-// tiles of a unit and writes the bf16 output of every unit it covers whole;
-// for a unit cut between CTAs each CTA writes an fp32 (max, sum, output)
-// partial record, and a small combine kernel that follows on the stream
-// merges the records with a log-sum-exp rescale.  The attention kernel has no
-// atomics, fences or inter-CTA waits.
+// Work decomposition.  A unit is one (sequence b, layer l, KV head g).  Its
+// keys are cut into tiles of 64: ceil(k / 64) Tier-1 tiles, then ceil(W / 64)
+// tiles of ring slots; no tile mixes the two tiers.  The flattened list of
+// (unit, tile) pairs is split into equal contiguous ranges, one per CTA.  When
+// the units fit in one wave of resident CTAs the grid is a whole number of
+// CTAs per unit -- one per unit at the model shapes, so no unit is split and
+// every CTA streams the same bytes; otherwise it is one wave of resident CTAs
+// (stream-K).  A CTA accumulates across the tiles of a unit and writes the
+// bf16 output of every unit it covers whole; for a unit cut between CTAs each
+// CTA writes an fp32 (max, sum, output) partial record, and a small combine
+// kernel that follows on the stream merges the records with a log-sum-exp
+// rescale.  No CTA ever waits on another.
 //
 // Inside a CTA one producer warp streams the tiles through a ring of shared-
 // memory stages.  Ring tiles, and Tier-1 tiles when the Tier-1 rows are the
@@ -40,8 +41,10 @@
 // The fused decode step also appends the new token: the producer copies the
 // new token's K/V rows next to the tile that holds its ring slot, a consumer
 // warp patches them over the stale ring row in shared memory and stores them
-// into the ring, and the combine kernel advances pos[b] after the attention
-// kernel has finished.
+// into the ring.  pos[b] is advanced by the last CTA to read it: each CTA adds
+// the number of tiles of sequence b it has read pos[b] for to a per-sequence
+// count in the workspace, and the CTA whose addition completes the count
+// (L * Hkv * tiles per unit) writes pos[b] + 1 and clears the count.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <math.h>
