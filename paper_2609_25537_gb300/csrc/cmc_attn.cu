@@ -64,6 +64,11 @@ constexpr size_t kWsHeader = 256;
 constexpr int kHalfBytes = kTileKeys * 128;  // one 64-row x 128-byte swizzled box
 constexpr int kMetaSlots = 4;                // producer metadata prefetch distance (tiles)
 
+// fp32 partial record of one CTA's share of a unit: max[G], sum[G], then, from
+// a 16-byte aligned offset, the unnormalised output [G][d].
+__host__ __device__ constexpr int rec_out_offset(int G) { return (2 * G + 3) & ~3; }
+__host__ __device__ constexpr int rec_floats(int G, int D) { return rec_out_offset(G) + G * D; }
+
 // Tensor maps of one launch (passed by value, in the kernel's parameter space).
 struct AttnMaps {
   CUtensorMap rk_box, rv_box;      // ring [units * W, d], box 64 cols x 64 rows
@@ -242,6 +247,12 @@ __device__ __forceinline__ long long cta_of_tile(long long t, long long base, lo
   const long long big = rem * (base + 1);
   return t < big ? t / (base + 1) : rem + (t - big) / base;
 }
+// Partial-record slot (tile position within the unit) of CTA c's share of
+// the unit whose first tile is ut0: the position of c's first tile in it.
+__device__ __forceinline__ long long rec_slot(const AttnParams& p, long long c, long long ut0) {
+  const long long t = cta_first_tile(c, p.base, p.rem);
+  return t > ut0 ? t - ut0 : 0;
+}
 
 // Unit coordinates of the tile at a position of the flattened (unit, j)
 // order, advanced one tile at a time so that the main loop does no integer
@@ -362,18 +373,50 @@ __device__ __forceinline__ SeqState seq_state(const AttnParams& p, long long pos
   return q;
 }
 
-// Producer warp: everything for one tile -- its K/V loads, the header the
-// consumers read (rows that may hold keys, rows with a bad index, the new
-// token's row), the unit's query rows and, in the fused step, the new token's
-// K/V rows -- and the arrive that, once the bytes have landed, releases the
-// stage to the consumers.
-template <int D, int G, bool FUSED>
-__device__ __forceinline__ void produce_tile(const AttnParams& p, const AttnMaps& maps,
-                                             uint8_t* stage, uint8_t* aux, const TileCursor& c,
-                                             const TileMeta& meta, const SeqState& sq, int lane,
-                                             uint64_t* full) {
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;\n" ::"r"(smem_addr(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+// Producer lane 0, box tiles: what does not depend on pos -- the K/V boxes and
+// the unit's query rows -- issued as soon as the stage is free.  Two-
+// dimensional boxes of 64 consecutive rows of the ring, or of the Tier-1
+// tensor under identity selection; rows past the unit's keys are masked later,
+// rows past the tensor are zero-filled by the TMA unit.
+template <int D, int G>
+__device__ __forceinline__ void issue_box_loads(const AttnParams& p, const AttnMaps& maps,
+                                                uint8_t* stage, uint8_t* aux, const TileCursor& c,
+                                                uint64_t* full) {
   using S = Stage<D, G>;
   constexpr int H = S::kHalves;
+  const bool t1 = c.lt < p.t1_tiles;
+  const int row = t1 ? c.u * p.N + c.lt * kTileKeys : c.u * p.W + (c.lt - p.t1_tiles) * kTileKeys;
+  const CUtensorMap* mk = t1 ? &maps.t1k_box : &maps.rk_box;
+  const CUtensorMap* mv = t1 ? &maps.t1v_box : &maps.rv_box;
+  const uint32_t sK = smem_addr(stage + S::kK);
+  const uint32_t sV = smem_addr(stage + S::kV);
+  mbar_expect_tx(full, 2 * H * kHalfBytes + G * D * 2);
+#pragma unroll
+  for (int h = 0; h < H; ++h) {
+    tma_box(sK + h * kHalfBytes, mk, h * 64, row, full);
+    tma_box(sV + h * kHalfBytes, mv, h * 64, row, full);
+  }
+  const uint16_t* qsrc =
+      p.q + ((static_cast<long long>(c.b) * p.L + c.l) * p.Hq + static_cast<long long>(c.g) * G) * D;
+  bulk_copy(smem_addr(aux + S::kQ), qsrc, G * D * 2, full);
+}
+
+// Producer warp, once pos (and, for a gathered tile, its idx entries) is
+// known: the tile's header (rows that may hold keys, rows with a bad index,
+// the new token's row), the new token's K/V rows in the fused step, the loads
+// of a gathered tile, and the arrive that, once every byte has landed,
+// releases the stage to the consumers.
+template <int D, int G, bool FUSED>
+__device__ __forceinline__ void finish_tile(const AttnParams& p, uint8_t* stage, uint8_t* aux,
+                                            const TileCursor& c, const TileMeta& meta,
+                                            const SeqState& sq, int lane, uint64_t* full) {
+  using S = Stage<D, G>;
   const bool t1 = c.lt < p.t1_tiles;
   int n_rows, new_row = -1;
   if (t1) {
@@ -383,8 +426,6 @@ __device__ __forceinline__ void produce_tile(const AttnParams& p, const AttnMaps
     n_rows = min(max(sq.count - slot0, 0), kTileKeys);
     if (FUSED && sq.new_slot >= slot0 && sq.new_slot - slot0 < n_rows) new_row = sq.new_slot - slot0;
   }
-  const uint32_t sK = smem_addr(stage + S::kK);
-  const uint32_t sV = smem_addr(stage + S::kV);
   uint32_t bad_lo = 0, bad_hi = 0;  // rows with an out-of-range index (gathered tiles)
   const bool gath = t1 && p.idx != nullptr;
   if (gath) {
@@ -394,6 +435,8 @@ __device__ __forceinline__ void produce_tile(const AttnParams& p, const AttnMaps
     // reach the full barrier through cp.async.mbarrier.arrive.
     constexpr int LPR = D / 8;     // lanes per row
     constexpr int RPP = 32 / LPR;  // rows per pass
+    const uint32_t sK = smem_addr(stage + S::kK);
+    const uint32_t sV = smem_addr(stage + S::kV);
     const int chunk = lane % LPR;
     const int rsub = lane / LPR;
     const long long ubase = static_cast<long long>(c.u) * p.N * D + chunk * 8;
@@ -422,26 +465,15 @@ __device__ __forceinline__ void produce_tile(const AttnParams& p, const AttnMaps
     hw[H_MASKED] = (n_rows < kTileKeys || (bad_lo | bad_hi)) ? 1 : 0;
     hw[H_BADLO] = static_cast<int>(bad_lo);
     hw[H_BADHI] = static_cast<int>(bad_hi);
-    uint32_t tx = G * D * 2;  // query rows
+    uint32_t tx = 0;
+    if (gath) tx += G * D * 2;  // query rows (box tiles: issued with the boxes)
     if (new_row >= 0) tx += 2 * D * 2;
-    if (!gath) tx += 2 * H * kHalfBytes;
-    mbar_arrive_expect_tx(full, tx);  // releases the header; completes when the bytes land
-    if (!gath) {
-      // Two-dimensional boxes of 64 consecutive rows of the ring, or of the
-      // Tier-1 tensor under identity selection.  Rows past the unit's keys
-      // are masked; rows past the tensor are zero-filled by the TMA unit.
-      const int row = t1 ? c.u * p.N + c.lt * kTileKeys : c.u * p.W + (c.lt - p.t1_tiles) * kTileKeys;
-      const CUtensorMap* mk = t1 ? &maps.t1k_box : &maps.rk_box;
-      const CUtensorMap* mv = t1 ? &maps.t1v_box : &maps.rv_box;
-#pragma unroll
-      for (int h = 0; h < H; ++h) {
-        tma_box(sK + h * kHalfBytes, mk, h * 64, row, full);
-        tma_box(sV + h * kHalfBytes, mv, h * 64, row, full);
-      }
+    mbar_arrive_expect_tx(full, tx);  // releases the header
+    if (gath) {
+      const uint16_t* qsrc =
+          p.q + ((static_cast<long long>(c.b) * p.L + c.l) * p.Hq + static_cast<long long>(c.g) * G) * D;
+      bulk_copy(smem_addr(aux + S::kQ), qsrc, G * D * 2, full);
     }
-    const uint16_t* qsrc =
-        p.q + ((static_cast<long long>(c.b) * p.L + c.l) * p.Hq + static_cast<long long>(c.g) * G) * D;
-    bulk_copy(smem_addr(aux + S::kQ), qsrc, G * D * 2, full);
     if (new_row >= 0) {
       bulk_copy(smem_addr(aux + S::kNew), p.k_new + static_cast<long long>(c.u) * D, D * 2, full);
       bulk_copy(smem_addr(aux + S::kNew + D * 2), p.v_new + static_cast<long long>(c.u) * D, D * 2, full);
@@ -524,6 +556,16 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
       prefetch_meta(p, cm, m < n_tiles, lane, &slots[m]);
       cm.next(p);
     }
+    {
+      // The box tiles of the first NST stages: their loads do not depend on
+      // pos, so they go out before any metadata has arrived.
+      TileCursor cl = ci;
+      for (int i = 0; i < NST && i < n_tiles; ++i) {
+        if (lane == 0 && !gathered_tile(p, cl))
+          issue_box_loads<D, G>(p, maps, smem + i * S::kBytes, aux0 + i * S::kAuxBytes, cl, &full_bar[i]);
+        cl.next(p);
+      }
+    }
     int issued = 0;
     int run_b = -1;           // sequence of the current run of tiles
     long long run_tiles = 0;  // tiles in that run so far
@@ -531,9 +573,13 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     sq.pos = 0; sq.count = 0; sq.new_slot = -1; sq.bad = true;
     for (int i = 0; i < n_tiles; ++i) {
       const int s = i % NST;
-      if (i >= NST && !mbar_wait(&empty_bar[s], static_cast<uint32_t>((i / NST - 1) & 1))) {
-        if (lane == 0) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
-        break;
+      if (i >= NST) {
+        if (!mbar_wait(&empty_bar[s], static_cast<uint32_t>((i / NST - 1) & 1))) {
+          if (lane == 0) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
+          break;
+        }
+        if (lane == 0 && !gathered_tile(p, ci))
+          issue_box_loads<D, G>(p, maps, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, &full_bar[s]);
       }
       MetaSlot* ms = &slots[i % kMetaSlots];
       cp_async_wait<kMetaSlots - 1>();  // this tile's metadata has landed
@@ -552,8 +598,8 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
         sq = seq_state<FUSED>(p, meta.pos);
       }
       ++run_tiles;
-      produce_tile<D, G, FUSED>(p, maps, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, meta, sq,
-                                lane, &full_bar[s]);
+      finish_tile<D, G, FUSED>(p, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, meta, sq, lane,
+                               &full_bar[s]);
       ci.next(p);
       issued = i + 1;
       __syncwarp();
@@ -724,58 +770,61 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     // ---- end of a unit within this CTA: merge warps, write out or a partial ----
     const bool unit_end = (i + 1 == n_tiles) || (cc.j == p.tpu - 1);
     if (unit_end) {
+      // Merge the four warps' states of each head: every warp rescales its
+      // output and sum to the heads' common running max, then each thread
+      // adds four columns across the warps in a fixed order.
       l_run += __shfl_xor_sync(0xffffffffu, l_run, 1);
       l_run += __shfl_xor_sync(0xffffffffu, l_run, 2);
+      if (gq < G && tq == 0) merge_m[warp * 8 + gq] = m_run;
+      consumer_sync();
       if (gq < G) {
-        if (tq == 0) {
-          merge_m[warp * 8 + gq] = m_run;
-          merge_l[warp * 8 + gq] = l_run;
-        }
+        float M = merge_m[gq];
+#pragma unroll
+        for (int w = 1; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + gq]);
+        const float f = (M == -INFINITY) ? 0.f : ex2(m_run - M);
         float* ow = merge_o + (warp * G + gq) * D;
 #pragma unroll
-        for (int j = 0; j < NT; ++j) {
-          *reinterpret_cast<float2*>(ow + 8 * j + 2 * tq) = make_float2(o[j][0], o[j][1]);
-        }
+        for (int j = 0; j < NT; ++j)
+          *reinterpret_cast<float2*>(ow + 8 * j + 2 * tq) = make_float2(o[j][0] * f, o[j][1] * f);
+        if (tq == 0) merge_l[warp * 8 + gq] = l_run * f;
       }
       consumer_sync();
 
-      const long long c0 = cta_of_tile(static_cast<long long>(u) * p.tpu, p.base, p.rem);
-      const long long c1 = cta_of_tile(static_cast<long long>(u) * p.tpu + p.tpu - 1, p.base, p.rem);
-      const bool whole = (c0 == c1);
-      const int PW = G * (D + 2);
-      float* rec = p.partials + (static_cast<long long>(u) * p.tpu + (cta - c0)) * PW;
+      // The unit is whole in this CTA unless the CTA's tile range cuts it; a
+      // cut unit's record goes to the slot of this CTA's first tile in it.
+      const long long ut0 = static_cast<long long>(u) * p.tpu;
+      const bool whole = ut0 >= t_begin && ut0 + p.tpu <= t_end;
       const long long out_base =
           ((static_cast<long long>(cc.b) * p.L + cc.l) * p.Hq + static_cast<long long>(cc.g) * G) * D;
-      constexpr int PAIRS = G * D / 2;
-      for (int x = tid; x < PAIRS; x += kThreads) {
-        const int hh = (2 * x) / D;
-        const int c = (2 * x) % D;
-        float M = -INFINITY;
+      for (int x = tid; x < G * D / 4; x += kThreads) {
+        const int hh = (4 * x) / D;
+        const int c = (4 * x) % D;
+        float4 acc = *reinterpret_cast<const float4*>(merge_o + hh * D + c);
+        float Ls = merge_l[hh];
 #pragma unroll
-        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + hh]);
-        float Ls = 0.f, O0 = 0.f, O1 = 0.f;
-        if (M != -INFINITY) {
-#pragma unroll
-          for (int w = 0; w < kWarps; ++w) {
-            const float f = ex2(merge_m[w * 8 + hh] - M);
-            const float2 ow = *reinterpret_cast<const float2*>(merge_o + (w * G + hh) * D + c);
-            Ls = fmaf(f, merge_l[w * 8 + hh], Ls);
-            O0 = fmaf(f, ow.x, O0);
-            O1 = fmaf(f, ow.y, O1);
-          }
+        for (int w = 1; w < kWarps; ++w) {
+          const float4 v = *reinterpret_cast<const float4*>(merge_o + (w * G + hh) * D + c);
+          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+          Ls += merge_l[w * 8 + hh];
         }
         if (whole) {
-          const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-          *reinterpret_cast<uint32_t*>(p.out + out_base + hh * D + c) = pack_bf16x2(O0 * inv, O1 * inv);
+          const float inv = Ls > 0.f ? __frcp_rn(Ls) : 0.f;
+          *reinterpret_cast<uint2*>(p.out + out_base + hh * D + c) =
+              make_uint2(pack_bf16_rn(acc.x * inv, acc.y * inv), pack_bf16_rn(acc.z * inv, acc.w * inv));
         } else {  // merged by two_tier_combine_kernel
+          constexpr int PW = rec_floats(G, D);
+          float* rec = p.partials + (ut0 + (ut0 > t_begin ? 0 : t_begin - ut0)) * PW;
           if (c == 0) {
+            float M = merge_m[hh];
+#pragma unroll
+            for (int w = 1; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + hh]);
             rec[hh] = M;
             rec[G + hh] = Ls;
           }
-          *reinterpret_cast<float2*>(rec + 2 * G + hh * D + c) = make_float2(O0, O1);
+          *reinterpret_cast<float4*>(rec + rec_out_offset(G) + hh * D + c) = acc;
         }
       }
-      consumer_sync();  // merge buffers are reused by the next unit
+      if (i + 1 < n_tiles) consumer_sync();  // merge buffers are reused by the next unit
     }
     cc.next(p);
   }
@@ -796,25 +845,28 @@ two_tier_combine_kernel(const AttnParams p) {
   const int lg = u - b * LH;
   const int l = lg / p.Hkv;
   const int g = lg - l * p.Hkv;
-  const long long c0 = cta_of_tile(static_cast<long long>(u) * p.tpu, p.base, p.rem);
-  const long long c1 = cta_of_tile(static_cast<long long>(u) * p.tpu + p.tpu - 1, p.base, p.rem);
+  const long long ut0 = static_cast<long long>(u) * p.tpu;
+  const long long c0 = cta_of_tile(ut0, p.base, p.rem);
+  const long long c1 = cta_of_tile(ut0 + p.tpu - 1, p.base, p.rem);
   if (c0 == c1) return;  // written by the attention kernel
+  // one record per CTA that holds part of the unit, at the slot of that
+  // CTA's first tile in the unit (slot 0 for c0)
   const int nrec = static_cast<int>(c1 - c0 + 1);
-  const int PW = G * (D + 2);
-  const float* recs = p.partials + static_cast<long long>(u) * p.tpu * PW;
+  constexpr int PW = rec_floats(G, D);
+  const float* recs = p.partials + ut0 * PW;
   const long long out_base =
       ((static_cast<long long>(b) * p.L + l) * p.Hq + static_cast<long long>(g) * G) * D;
   for (int x = threadIdx.x; x < G * D / 2; x += blockDim.x) {
     const int hh = (2 * x) / D;
     const int c = (2 * x) % D;
     float M = -INFINITY;
-    for (int r = 0; r < nrec; ++r) M = fmaxf(M, recs[r * PW + hh]);
+    for (int r = 0; r < nrec; ++r) M = fmaxf(M, recs[rec_slot(p, c0 + r, ut0) * PW + hh]);
     float Ls = 0.f, O0 = 0.f, O1 = 0.f;
     if (M != -INFINITY) {
       for (int r = 0; r < nrec; ++r) {
-        const float* pr = recs + r * PW;
+        const float* pr = recs + rec_slot(p, c0 + r, ut0) * PW;
         const float f = ex2(pr[hh] - M);
-        const float2 o2 = *reinterpret_cast<const float2*>(pr + 2 * G + hh * D + c);
+        const float2 o2 = *reinterpret_cast<const float2*>(pr + rec_out_offset(G) + hh * D + c);
         Ls = fmaf(f, pr[G + hh], Ls);
         O0 = fmaf(f, o2.x, O0);
         O1 = fmaf(f, o2.y, O1);
@@ -906,14 +958,15 @@ static int tier1_tiles(const cmc_dims& m) { return (m.k + kTileKeys - 1) / kTile
 static int tiles_per_unit(const cmc_dims& m) { return tier1_tiles(m) + (m.W + kTileKeys - 1) / kTileKeys; }
 
 // [0, 256): status word; then one 8-byte pos-read count per sequence (padded
-// to 256 bytes); then one partial record per (unit, tile) slot.
+// to 256 bytes); then one partial record per (unit, tile) slot (16-byte
+// aligned: rec_floats is a multiple of 4).
 static WsLayout ws_layout(const cmc_dims& m) {
   WsLayout w;
   const long long units = static_cast<long long>(m.B) * m.L * m.Hkv;
   const int G = m.Hq / m.Hkv;
   w.tickets_off = kWsHeader;
   w.partials_off = w.tickets_off + ((static_cast<size_t>(m.B) * 8 + 255) / 256) * 256;
-  w.total = w.partials_off + static_cast<size_t>(units) * tiles_per_unit(m) * G * (m.d + 2) * sizeof(float);
+  w.total = w.partials_off + static_cast<size_t>(units) * tiles_per_unit(m) * rec_floats(G, m.d) * sizeof(float);
   return w;
 }
 

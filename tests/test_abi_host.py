@@ -134,7 +134,8 @@ def test_window_append_argument_checks(L):
 
 def test_attention_workspace_size(L):
     # a 256-byte status header, 8 bytes per sequence padded to 256, then one
-    # fp32 partial record of G * (d + 2) floats per (unit, 64-key tile) slot;
+    # fp32 partial record per (unit, 64-key tile) slot: max and sum per head
+    # (2G floats, padded to a multiple of 4) and the output, G * d floats;
     # a unit has ceil(k / 64) Tier-1 tiles and ceil(W / 64) ring tiles
     d = _dims()
     units = 2 * 3 * 2
@@ -149,7 +150,7 @@ def test_attention_workspace_size(L):
         256 + 256 + units * (0 + 1) * G * (128 + 2) * 4)
     many = _dims(B=40, Hkv=1, Hq=1, L=1, k=0, W=64)
     assert L.cmc_decode_attn_workspace_size(ctypes.byref(many)) == (
-        256 + 512 + 40 * 1 * 1 * (128 + 2) * 4)
+        256 + 512 + 40 * 1 * 1 * (4 + 128) * 4)
     assert L.cmc_decode_attn_workspace_size(ctypes.byref(_dims(d=80))) == 0
 
 
