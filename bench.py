@@ -441,6 +441,10 @@ def run_gpu(args, w, world, rank, local):
     value = tokens / (max_ms / 1000.0)
 
     launches_dec = K * R * T
+    # kernels per fused decode call (attention, plus combine if units are split)
+    step_launches = cmc.decode_attn_plan(
+        cmc.dims_of(reqs[0].out, reqs[0].t1k_dense if mode == "dense" else reqs[0].t1k,
+                    None if mode == "dense" else reqs[0].idx, reqs[0].ring_k), fused=True)[1]
     launch_us = 1000.0 * sum(dec_ms) / launches_dec
     nbytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W, gather=mode == "gather")
     achieved = nbytes / (launch_us * 1e-6) / 1e9
@@ -496,8 +500,9 @@ def run_gpu(args, w, world, rank, local):
         "variant": variant,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
-                     "kernel": ("fused decode step: two_tier_attn_kernel<128,4,fused,3> "
-                                "(one CTA per unit; no combine launch at this shape)"),
+                     "kernel": ("fused decode step: two_tier_attn_kernel<128,4,fused,3>"
+                                + (" (one CTA per unit, no combine launch)" if step_launches == 1
+                                   else " + two_tier_combine_kernel")),
                      "bytes_per_launch": nbytes, "traffic": profiled_traffic(),
                      "flops_per_launch": decode_step_flops(w.B, w.L, w.Hq, w.d, w.k, w.W)},
         "select_roofline": {"bound": "hbm", "bytes": select_bytes(w.B, w.N, w.D, w.k),
@@ -505,7 +510,7 @@ def run_gpu(args, w, world, rank, local):
                             / 1e9, "unit": "GB/s"},
         "e2e": e2e,
         "cpu_baseline": cpu,
-        "gpu_launches": K * R * (2 * T + (3 if mode == "dense" else 2)),
+        "gpu_launches": K * R * (T * step_launches + (3 if mode == "dense" else 2)),
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)
@@ -516,7 +521,9 @@ def run_e2e(args, w, reqs, dev, stream, world):
     """Same metric through the public Python API with host buffers: the
     question vector and CME bank of each request and, every decode step, q and
     the new token's K,V are copied in from pinned host memory and the output
-    copied back to pinned host memory."""
+    copied back to pinned host memory.  The per-step sequence (three copies
+    in, the decode call, one copy out) is captured in a CUDA graph of P rounds,
+    as a serving loop would; selection and compaction run eagerly."""
     import paper_2609_25537_gb300 as cmc
     R, T, P = args.requests, args.decode_steps, args.pool
     steps = max(1, min(args.steps, args.e2e_steps))
@@ -532,6 +539,25 @@ def run_e2e(args, w, reqs, dev, stream, world):
         }
         host.append(h)
 
+    def one_step_calls(p):
+        for r, h in zip(reqs, host):
+            h["q_d"].copy_(h["q"][p], non_blocking=True)
+            h["k_d"].copy_(h["k"][p], non_blocking=True)
+            h["v_d"].copy_(h["v"][p], non_blocking=True)
+            r.decode(p, q=h["q_d"], k_new=h["k_d"], v_new=h["v_d"], mode=args.tier1)
+            h["out"][p].copy_(r.out, non_blocking=True)
+
+    graph = None
+    try:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for p in range(P):
+                one_step_calls(p)
+        graph = g
+    except Exception as e:  # capture of host copies unsupported: run eagerly
+        print(f"e2e: graph capture failed ({type(e).__name__}: {e}); eager loop", file=sys.stderr)
+        torch.cuda.synchronize(dev)
+
     def step():
         with torch.cuda.stream(stream):
             for r, h in zip(reqs, host):
@@ -540,14 +566,12 @@ def run_e2e(args, w, reqs, dev, stream, world):
                 cmc.score_select(r.qemb, r.bank, w.k, idx_out=r.idx, workspace=r.sel_ws)
                 if args.tier1 == "dense":
                     r.gather()
-            for t in range(T):
-                p = t % P
-                for r, h in zip(reqs, host):
-                    h["q_d"].copy_(h["q"][p], non_blocking=True)
-                    h["k_d"].copy_(h["k"][p], non_blocking=True)
-                    h["v_d"].copy_(h["v"][p], non_blocking=True)
-                    r.decode(p, q=h["q_d"], k_new=h["k_d"], v_new=h["v_d"], mode=args.tier1)
-                    h["out"][p].copy_(r.out, non_blocking=True)
+            if graph is not None:
+                for _ in range(T // P):
+                    graph.replay()
+            else:
+                for t in range(T):
+                    one_step_calls(t % P)
         stream.synchronize()
 
     step()  # warm-up
@@ -562,7 +586,8 @@ def run_e2e(args, w, reqs, dev, stream, world):
                + T * 2 * (r0.q[0].numel() + r0.k_new[0].numel() + r0.v_new[0].numel()))
     d2h = R * T * r0.out.numel() * 2
     return {"value": world * steps * R * w.B * T / el, "unit": "tokens/s",
-            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps}
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
+            "per_step_graph": graph is not None}
 
 
 def main(argv=None):

@@ -211,6 +211,16 @@ CMC_API int cmc_tier1_gather(const void* bank_k, const void* bank_v, const int32
                              const cmc_dims* dims, void* tier1_k, void* tier1_v, uint32_t* status,
                              void* stream);
 
+/*
+ * Launch plan of cmc_two_tier_decode_attn (fused == 0) or cmc_decode_step
+ * (fused != 0) for `dims` on the current device: *ctas receives the grid size
+ * of the attention kernel and *launches the number of kernels one call
+ * enqueues (1, or 2 when some (sequence, layer, KV head) unit is split
+ * between CTAs and a combine kernel merges its partial results).  No work is
+ * enqueued.  Useful for sizing CUDA graphs and for counting launches.
+ */
+CMC_API int cmc_decode_attn_plan(const cmc_dims* dims, int fused, int* ctas, int* launches);
+
 /* Copies the device status word of an attention workspace (CMC_DEVFLAG_*
  * bits) into *flags, waiting for `stream`, and clears it when `clear` != 0. */
 CMC_API int cmc_read_status(void* workspace, int clear, uint32_t* flags, void* stream);

@@ -39,6 +39,7 @@ __all__ = [
     "decode_step",
     "tier1_gather",
     "decode_attn_workspace_size",
+    "decode_attn_plan",
     "dims_of",
     "DEVFLAG_BAD_INDEX",
     "DEVFLAG_BAD_POS",
@@ -130,6 +131,16 @@ def dims_of(q: torch.Tensor, tier1_k: torch.Tensor, idx: Optional[torch.Tensor],
 
 def decode_attn_workspace_size(dims: CmcDims) -> int:
     return int(lib().cmc_decode_attn_workspace_size(ctypes.byref(dims)))
+
+
+def decode_attn_plan(dims: CmcDims, fused: bool = True) -> Tuple[int, int]:
+    """(grid size, kernel launches per call) of the attention entry points for
+    `dims` on the current device; see cmc_decode_attn_plan."""
+    ctas, launches = ctypes.c_int(0), ctypes.c_int(0)
+    st = lib().cmc_decode_attn_plan(ctypes.byref(dims), 1 if fused else 0, ctypes.byref(ctas),
+                                    ctypes.byref(launches))
+    check(st, "cmc_decode_attn_plan")
+    return int(ctas.value), int(launches.value)
 
 
 class DecodeWorkspace:

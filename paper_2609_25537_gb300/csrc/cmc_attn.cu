@@ -902,10 +902,12 @@ __global__ void window_append_kernel(uint16_t* __restrict__ ring_k, uint16_t* __
 
 // Tier-1 compaction (the "M*" of Section 2.5, formed once per question):
 //   tier1[b, l, g, i] = bank[b, l, g, idx[b, i]]   for i < k.
-// A CTA copies a block of kGatherRows output rows of one unit; each row's d/8
-// 16-byte chunks are read by consecutive threads.  Out-of-range indices give a
-// zero row and CMC_DEVFLAG_BAD_INDEX.
+// A CTA copies a block of kGatherRows output rows of one unit: each thread
+// issues all of its 16-byte streaming loads (K and V) before its stores, so a
+// whole block is in flight at once.  Out-of-range indices give a zero row and
+// CMC_DEVFLAG_BAD_INDEX.
 constexpr int kGatherRows = 64;
+constexpr int kGatherThreads = 256;
 
 __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
   uint4 r;
@@ -915,32 +917,46 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
   return r;
 }
 
-__global__ void __launch_bounds__(256)
+template <int CPR>  // 16-byte chunks per row: d / 8
+__global__ void __launch_bounds__(kGatherThreads)
 tier1_gather_kernel(const uint4* __restrict__ bank_k, const uint4* __restrict__ bank_v,
                     const int32_t* __restrict__ idx, uint4* __restrict__ out_k,
                     uint4* __restrict__ out_v, uint32_t* status, long long blocks, int row_blocks,
-                    int LH, int N, int k, int cpr) {
+                    int LH, int N, int k) {
+  constexpr int kPer = kGatherRows * CPR / kGatherThreads;  // chunks per thread and tensor
+  pdl_wait();
+  pdl_trigger();
   bool bad = false;
   for (long long blk = blockIdx.x; blk < blocks; blk += gridDim.x) {
     const long long u = blk / row_blocks;
     const int i0 = static_cast<int>(blk - u * row_blocks) * kGatherRows;
-    const int nrow = min(kGatherRows, k - i0);
     const int32_t* irow = idx + (u / LH) * k;
-    for (int x = threadIdx.x; x < nrow * cpr; x += blockDim.x) {
-      const int i = i0 + x / cpr;
-      const int c = x % cpr;
-      const int j = __ldg(irow + i);
-      uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
-      if (static_cast<unsigned>(j) < static_cast<unsigned>(N)) {
-        const long long src = (u * N + j) * cpr + c;
-        kv = ld_stream(bank_k + src);
-        vv = ld_stream(bank_v + src);
-      } else {
-        bad = true;
+    uint4 kv[kPer], vv[kPer];
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+      const int x = threadIdx.x + e * kGatherThreads;
+      const int i = i0 + x / CPR;
+      kv[e] = vv[e] = make_uint4(0u, 0u, 0u, 0u);
+      if (i < k) {
+        const int j = __ldg(irow + i);
+        if (static_cast<unsigned>(j) < static_cast<unsigned>(N)) {
+          const long long src = (u * N + j) * CPR + x % CPR;
+          kv[e] = ld_stream(bank_k + src);
+          vv[e] = ld_stream(bank_v + src);
+        } else {
+          bad = true;
+        }
       }
-      const long long dst = (u * k + i) * cpr + c;
-      out_k[dst] = kv;
-      out_v[dst] = vv;
+    }
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) {
+      const int x = threadIdx.x + e * kGatherThreads;
+      const int i = i0 + x / CPR;
+      if (i < k) {
+        const long long dst = (u * k + i) * CPR + x % CPR;
+        out_k[dst] = kv[e];
+        out_v[dst] = vv[e];
+      }
     }
   }
   if (bad && status) atomicOr(status, CMC_DEVFLAG_BAD_INDEX);
@@ -1008,9 +1024,14 @@ static bool encode_rows(CUtensorMap* map, const void* base, long long rows, int 
 // ~110 KB of shared memory at d = 128, G <= 4, so two CTAs share an SM.
 constexpr int kStages = 3;
 
+// Launch plan of one attention call on the current device.
+struct AttnPlan {
+  long long ctas, base, rem;  // grid size; tiles per CTA (the first `rem` CTAs take one more)
+  bool split;                 // some unit is cut between CTAs: the combine kernel runs
+};
+
 template <int D, int G, bool FUSED>
-static int launch_attn(const AttnMaps& maps, const AttnParams& p0, long long total_tiles,
-                       cudaStream_t s) {
+static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
   constexpr size_t smem = attn_smem_bytes<D, G, kStages>();
   auto kern = two_tier_attn_kernel<D, G, FUSED, kStages>;
   static int configured[64] = {0};  // per device: attribute set and occupancy known
@@ -1027,43 +1048,60 @@ static int launch_attn(const AttnMaps& maps, const AttnParams& p0, long long tot
     if (per_sm < 1) per_sm = 1;
     if (dev >= 0 && dev < 64) configured[dev] = per_sm;
   }
-  AttnParams p = p0;
   // Grid: with no more units than resident CTAs, a whole number of CTAs per
   // unit (one per unit when they fit: no unit is split and no combine kernel
   // runs); otherwise one wave of resident CTAs, each taking an equal share of
   // the flattened tiles.
   const long long slots = static_cast<long long>(per_sm) * sm_count();
-  const long long units = total_tiles / p.tpu;
+  const long long units = total_tiles / tpu;
   long long ctas = units <= slots ? units * (slots / units) : slots;
   if (ctas > total_tiles) ctas = total_tiles;
   if (ctas < 1) ctas = 1;
-  p.base = total_tiles / ctas;
-  p.rem = total_tiles % ctas;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
-  cfg.blockDim = dim3(kThreads + 32);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  st = record_cuda_error(cudaLaunchKernelEx(&cfg, kern, maps, p));
-  if (st != CMC_OK) return st;
+  pl->ctas = ctas;
+  pl->base = total_tiles / ctas;
+  pl->rem = total_tiles % ctas;
   // Is any unit split between CTAs (a CTA boundary inside a unit)?
-  bool split = false;
-  for (long long c = 1; c < ctas && !split; ++c) {
-    const long long t = c * p.base + (c < p.rem ? c : p.rem);
-    split = (t % p.tpu) != 0;
+  pl->split = false;
+  for (long long c = 1; c < ctas && !pl->split; ++c) {
+    const long long t = c * pl->base + (c < pl->rem ? c : pl->rem);
+    pl->split = (t % tpu) != 0;
   }
-  if (split) {
-    cfg.gridDim = dim3(static_cast<unsigned>(units));
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = 0;
-    st = record_cuda_error(cudaLaunchKernelEx(&cfg, two_tier_combine_kernel<D, G>, p));
+  return CMC_OK;
+}
+
+template <int D, int G, bool FUSED>
+static int launch_attn(const AttnMaps& maps, const AttnParams& p0, long long total_tiles,
+                       cudaStream_t s) {
+  constexpr size_t smem = attn_smem_bytes<D, G, kStages>();
+  AttnPlan pl;
+  int st = plan_attn<D, G, FUSED>(total_tiles, p0.tpu, &pl);
+  if (st != CMC_OK) return st;
+  AttnParams p = p0;
+  p.base = pl.base;
+  p.rem = pl.rem;
+  st = launch_pdl(two_tier_attn_kernel<D, G, FUSED, kStages>, dim3(static_cast<unsigned>(pl.ctas)),
+                  dim3(kThreads + 32), smem, s, maps, p);
+  if (st != CMC_OK || !pl.split) return st;
+  return launch_pdl(two_tier_combine_kernel<D, G>, dim3(static_cast<unsigned>(total_tiles / p.tpu)),
+                    dim3(kThreads), 0, s, p);
+}
+
+template <bool FUSED>
+static int dispatch_plan(int d, int G, long long tiles, int tpu, AttnPlan* pl) {
+  if (d == 128) {
+    switch (G) {
+      case 1: return plan_attn<128, 1, FUSED>(tiles, tpu, pl);
+      case 2: return plan_attn<128, 2, FUSED>(tiles, tpu, pl);
+      case 4: return plan_attn<128, 4, FUSED>(tiles, tpu, pl);
+      default: return plan_attn<128, 8, FUSED>(tiles, tpu, pl);
+    }
   }
-  return st;
+  switch (G) {
+    case 1: return plan_attn<64, 1, FUSED>(tiles, tpu, pl);
+    case 2: return plan_attn<64, 2, FUSED>(tiles, tpu, pl);
+    case 4: return plan_attn<64, 4, FUSED>(tiles, tpu, pl);
+    default: return plan_attn<64, 8, FUSED>(tiles, tpu, pl);
+  }
 }
 
 template <bool FUSED>
@@ -1195,11 +1233,31 @@ int cmc_tier1_gather(const void* bank_k, const void* bank_v, const int32_t* idx,
   const int row_blocks = (m.k + kGatherRows - 1) / kGatherRows;
   const long long blocks = units * row_blocks;
   const long long grid = blocks < (1LL << 30) ? blocks : (1LL << 30);
-  tier1_gather_kernel<<<static_cast<unsigned>(grid), 256, 0, static_cast<cudaStream_t>(stream)>>>(
-      static_cast<const uint4*>(bank_k), static_cast<const uint4*>(bank_v), idx,
-      static_cast<uint4*>(tier1_k), static_cast<uint4*>(tier1_v), status, blocks, row_blocks,
-      m.L * m.Hkv, m.N, m.k, m.d / 8);
-  return check_launch();
+  auto kern = m.d == 128 ? tier1_gather_kernel<16> : tier1_gather_kernel<8>;
+  return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(kGatherThreads), 0,
+                    static_cast<cudaStream_t>(stream), static_cast<const uint4*>(bank_k),
+                    static_cast<const uint4*>(bank_v), idx, static_cast<uint4*>(tier1_k),
+                    static_cast<uint4*>(tier1_v), status, blocks, row_blocks, m.L * m.Hkv, m.N,
+                    m.k);
+}
+
+int cmc_decode_attn_plan(const cmc_dims* dims, int fused, int* ctas, int* launches) {
+  using namespace cmc;
+  int st = validate_dims(dims, true);
+  if (st != CMC_OK) return st;
+  if (!ctas || !launches) return CMC_ERR_NULL;
+  const cmc_dims& m = *dims;
+  const long long units = static_cast<long long>(m.B) * m.L * m.Hkv;
+  const int tpu = tiles_per_unit(m);
+  const long long tiles = units * tpu;
+  if (tiles >= (1LL << 31)) return CMC_ERR_SHAPE;
+  AttnPlan pl;
+  st = fused ? dispatch_plan<true>(m.d, m.Hq / m.Hkv, tiles, tpu, &pl)
+             : dispatch_plan<false>(m.d, m.Hq / m.Hkv, tiles, tpu, &pl);
+  if (st != CMC_OK) return st;
+  *ctas = static_cast<int>(pl.ctas);
+  *launches = pl.split ? 2 : 1;
+  return CMC_OK;
 }
 
 int cmc_window_append(void* ring_k, void* ring_v, int64_t* pos, const void* k_new,

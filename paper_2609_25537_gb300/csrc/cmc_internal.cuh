@@ -29,6 +29,25 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // Validates the shape fields of a cmc_dims that the attention path uses.
 int validate_dims(const cmc_dims* dims, bool need_bank);
 
+// Launches `kern` with programmatic stream serialization: the kernel may
+// start while the previous kernel on the stream is still running, so it must
+// execute griddepcontrol.wait before it reads anything that kernel writes.
+template <typename... KArgs, typename... Args>
+int launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+               Args... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return record_cuda_error(cudaLaunchKernelEx(&cfg, kern, args...));
+}
+
 // ---------------------------------------------------------------------------
 // Device side
 // ---------------------------------------------------------------------------
@@ -73,6 +92,11 @@ __device__ __forceinline__ float4 ld_stream_f4(const void* p) {
                : "l"(p));
   return r;
 }
+
+// Programmatic dependent launch: wait for the previous kernel on the stream
+// (and its memory) before reading its outputs; let the next kernel launch.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 // Order-preserving map of an fp32 score to uint32 (larger score -> larger key).
 __device__ __forceinline__ uint32_t orderable(float f) {

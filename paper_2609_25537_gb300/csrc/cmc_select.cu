@@ -2,15 +2,20 @@
 // top-K re-ordering by document position that follows it).
 //
 // Two kernels:
-//  1. cosine_scores_kernel -- one warp per CME row streams the row with 16-byte
-//     loads, accumulating m.q, m.m and q.q in fp32 in a fixed order, so equal
-//     rows produce bit-identical scores.  HBM-bound: 4*D bytes per row.
+//  1. cosine_scores_kernel -- one CTA of 256 threads per CME row (grid-stride
+//     over rows): every thread streams its share of the row with 16-byte loads
+//     issued four at a time, accumulating m.q, m.m and q.q in fp32; the
+//     partial sums meet in a fixed tree (warp shuffles, then the eight warps
+//     in order), so equal rows produce bit-identical scores.  HBM-bound:
+//     4*D bytes per row, with a whole row per CTA in flight.
 //  2. topk_select_kernel -- one CTA per sequence.  Scores are mapped to
 //     order-preserving uint32 keys; a 4-pass MSB radix select (8 bits a pass)
 //     finds the key T of the k-th largest score and how many of the keys equal
 //     to T are needed; an ordered compaction then writes the selected indices
 //     in ascending order (keys > T, plus the lowest-index keys == T), which is
 //     the document-order re-ordering and the lower-index tie rule at once.
+// Both launch with programmatic stream serialization, so the selection
+// kernel's launch overlaps the scoring kernel.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -21,28 +26,32 @@
 namespace cmc {
 
 constexpr int kScoreThreads = 256;
-constexpr int kScoreUnroll = 8;
+constexpr int kScoreUnroll = 4;
 constexpr int kSelectThreads = 1024;
 
 __global__ void __launch_bounds__(kScoreThreads)
 cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ bank, int N, int D,
                      long long rows, float* __restrict__ scores) {
-  const int lane = threadIdx.x & 31;
-  const long long warp0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const long long nwarps = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
+  constexpr int kWarpsPerCta = kScoreThreads / 32;
+  __shared__ float part[3][kWarpsPerCta];
+  const int tid = threadIdx.x;
+  const int lane = tid & 31;
+  const int warp = tid >> 5;
   const int D4 = D >> 2;
-  for (long long r = warp0; r < rows; r += nwarps) {
+  pdl_wait();
+  pdl_trigger();
+  for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
     const long long b = r / N;
     const float4* m = reinterpret_cast<const float4*>(bank + r * D);
     const float4* q = reinterpret_cast<const float4*>(qv + b * D);
     float dot = 0.f, mm = 0.f, qq = 0.f;
-    int i = lane;
-    for (; i + 32 * (kScoreUnroll - 1) < D4; i += 32 * kScoreUnroll) {
+    int i = tid;
+    for (; i + kScoreThreads * (kScoreUnroll - 1) < D4; i += kScoreThreads * kScoreUnroll) {
       float4 a[kScoreUnroll], c[kScoreUnroll];
 #pragma unroll
-      for (int u = 0; u < kScoreUnroll; ++u) a[u] = ld_stream_f4(m + i + 32 * u);
+      for (int u = 0; u < kScoreUnroll; ++u) a[u] = ld_stream_f4(m + i + kScoreThreads * u);
 #pragma unroll
-      for (int u = 0; u < kScoreUnroll; ++u) c[u] = __ldg(q + i + 32 * u);
+      for (int u = 0; u < kScoreUnroll; ++u) c[u] = __ldg(q + i + kScoreThreads * u);
 #pragma unroll
       for (int u = 0; u < kScoreUnroll; ++u) {
         dot = fmaf(a[u].x, c[u].x, dot); dot = fmaf(a[u].y, c[u].y, dot);
@@ -53,7 +62,7 @@ cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ ban
         qq = fmaf(c[u].z, c[u].z, qq); qq = fmaf(c[u].w, c[u].w, qq);
       }
     }
-    for (; i < D4; i += 32) {
+    for (; i < D4; i += kScoreThreads) {
       const float4 a = ld_stream_f4(m + i);
       const float4 c = __ldg(q + i);
       dot = fmaf(a.x, c.x, dot); dot = fmaf(a.y, c.y, dot);
@@ -70,11 +79,25 @@ cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ ban
       qq += __shfl_xor_sync(0xffffffffu, qq, off);
     }
     if (lane == 0) {
-      float s = 0.f;
-      if (mm > 0.f && qq > 0.f) s = dot / (sqrtf(mm) * sqrtf(qq));
-      if (s == 0.f) s = 0.f;  // -0 -> +0, so that -0 and +0 tie
-      scores[r] = s;
+      part[0][warp] = dot;
+      part[1][warp] = mm;
+      part[2][warp] = qq;
     }
+    __syncthreads();
+    if (tid == 0) {
+      float sd = part[0][0], sm = part[1][0], sq = part[2][0];
+#pragma unroll
+      for (int w = 1; w < kWarpsPerCta; ++w) {
+        sd += part[0][w];
+        sm += part[1][w];
+        sq += part[2][w];
+      }
+      float sc = 0.f;
+      if (sm > 0.f && sq > 0.f) sc = sd / (sqrtf(sm) * sqrtf(sq));
+      if (sc == 0.f) sc = 0.f;  // -0 -> +0, so that -0 and +0 tie
+      scores[r] = sc;
+    }
+    __syncthreads();  // part[] is reused by the next row
   }
 }
 
@@ -110,6 +133,8 @@ __global__ void __launch_bounds__(kSelectThreads)
 topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx_out) {
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
+  pdl_wait();  // the scores of the kernel before
+  pdl_trigger();
   const float* s = scores + static_cast<long long>(b) * N;
   int32_t* out = idx_out + static_cast<long long>(b) * k;
   if (k <= 0) return;
@@ -184,6 +209,20 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
   }
 }
 
+// The two selection kernels, scores written to `sc` (device, B * N floats).
+static int launch_score_select(const float* question_emb, const float* cme_bank, int B, int N,
+                               int D, int k, int32_t* idx_out, float* sc, cudaStream_t s) {
+  const long long rows = static_cast<long long>(B) * N;
+  long long blocks = rows;
+  const long long cap = static_cast<long long>(sm_count()) * (2048 / kScoreThreads);
+  if (blocks > cap) blocks = cap;
+  int st = launch_pdl(cosine_scores_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kScoreThreads),
+                      0, s, question_emb, cme_bank, N, D, rows, sc);
+  if (st != CMC_OK || k == 0) return st;
+  return launch_pdl(topk_select_kernel, dim3(B), dim3(kSelectThreads), 0, s,
+                    static_cast<const float*>(sc), N, k, idx_out);
+}
+
 }  // namespace cmc
 
 extern "C" {
@@ -213,18 +252,8 @@ int cmc_score_select(const float* question_emb, const float* cme_bank, int B, in
     if (reinterpret_cast<uintptr_t>(workspace) & 3) return CMC_ERR_ALIGN;
     sc = static_cast<float*>(workspace);
   }
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const long long rows = static_cast<long long>(B) * N;
-  const long long warps_per_block = kScoreThreads / 32;
-  long long blocks = (rows + warps_per_block - 1) / warps_per_block;
-  const long long cap = static_cast<long long>(sm_count()) * 16;
-  if (blocks > cap) blocks = cap;
-  cosine_scores_kernel<<<static_cast<unsigned>(blocks), kScoreThreads, 0, s>>>(
-      question_emb, cme_bank, N, D, rows, sc);
-  int st = check_launch();
-  if (st != CMC_OK || k == 0) return st;
-  topk_select_kernel<<<B, kSelectThreads, 0, s>>>(sc, N, k, idx_out);
-  return check_launch();
+  return launch_score_select(question_emb, cme_bank, B, N, D, k, idx_out, sc,
+                             static_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"
@@ -277,16 +306,6 @@ extern "C" int cmc_score_select_static(const float* question_emb, const float* c
   float* sc = nullptr;
   int st = static_scores_address(&sc);
   if (st != CMC_OK) return st;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const long long rows = static_cast<long long>(B) * N;
-  const long long warps_per_block = kScoreThreads / 32;
-  long long blocks = (rows + warps_per_block - 1) / warps_per_block;
-  const long long cap = static_cast<long long>(sm_count()) * 16;
-  if (blocks > cap) blocks = cap;
-  cosine_scores_kernel<<<static_cast<unsigned>(blocks), kScoreThreads, 0, s>>>(
-      question_emb, cme_bank, N, D, rows, sc);
-  st = check_launch();
-  if (st != CMC_OK || k == 0) return st;
-  topk_select_kernel<<<B, kSelectThreads, 0, s>>>(sc, N, k, idx_out);
-  return check_launch();
+  return launch_score_select(question_emb, cme_bank, B, N, D, k, idx_out, sc,
+                             static_cast<cudaStream_t>(stream));
 }

@@ -182,3 +182,13 @@ def test_tier1_gather_argument_checks(L):
     assert g(dims=_dims(Hq=3)) not in (SHAPE,)  # query heads are ignored
     assert g(bank=0, idx=0, out=0, dims=_dims(k=0)) == 0  # k = 0: nothing to do
     assert L.cmc_tier1_gather(FAKE, FAKE, FAKE, None, FAKE, FAKE, 0, None) == NULL
+
+
+def test_decode_attn_plan_argument_checks(L):
+    ctas, launches = ctypes.c_int(0), ctypes.c_int(0)
+    assert L.cmc_decode_attn_plan(None, 1, ctypes.byref(ctas), ctypes.byref(launches)) == NULL
+    assert L.cmc_decode_attn_plan(ctypes.byref(_dims()), 1, None, ctypes.byref(launches)) == NULL
+    assert L.cmc_decode_attn_plan(ctypes.byref(_dims(d=96)), 1, ctypes.byref(ctas),
+                                  ctypes.byref(launches)) == SHAPE
+    assert L.cmc_decode_attn_plan(ctypes.byref(_dims(k=101)), 0, ctypes.byref(ctas),
+                                  ctypes.byref(launches)) == RANGE

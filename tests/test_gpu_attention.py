@@ -374,3 +374,21 @@ def test_tier1_gather_bad_index_zero_row_and_flag(cuda_device):
             for i, j in enumerate(idx[b]):
                 want = host[b][:, :, j] if 0 <= j < w.N else 0
                 np.testing.assert_array_equal(got[b][:, :, i], want)
+
+
+def test_decode_attn_plan(cuda_device):
+    """One CTA per (layer, KV head) unit and a single launch per step at the
+    Llama-3-8B shape when 256 CTAs fit in one wave; split units (long-context
+    shape) add the combine launch."""
+    sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
+    w = WORKLOADS["llama3_8b"]
+    dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.k, w.W)
+    ctas, launches = cmc.decode_attn_plan(dims)
+    if 2 * sms >= 256:
+        assert (ctas, launches) == (256, 1)
+    w = WORKLOADS["long_context"]
+    dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.k, w.W)
+    ctas, launches = cmc.decode_attn_plan(dims, fused=False)
+    assert launches in (1, 2) and ctas >= 64
+    if 2 * sms >= 256:
+        assert (ctas, launches) == (256, 2)
