@@ -185,15 +185,34 @@ class ClockSampler:
 # Distributed plumbing (one process per GPU; replicas only)
 # ----------------------------------------------------------------------------
 
-def dist_setup():
+def dist_setup(backend: str = "nccl"):
+    """One process per GPU (torchrun env vars).  The ranks run independent
+    replicas of the workload (no data-path collective); the process group only
+    carries the start/stop barriers and the max-over-ranks of the elapsed
+    time.  `backend="gloo"` runs the same logic on CPU."""
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group(backend)
     return world, rank, local
+
+
+def request_seeds(w, rank: int, R: int):
+    """Seeds of the R requests rank `rank` runs: distinct across ranks, so N
+    ranks process N x R different requests (weak scaling)."""
+    return [1000 * w.seed + 100 * rank + r for r in range(R)]
+
+
+def job_tokens_per_s(world: int, K: int, R: int, B: int, T: int, max_ms: float) -> float:
+    """Whole-job decode tokens/s: every rank's K rounds of R requests x B
+    sequences x T steps, over the slowest rank's elapsed time."""
+    return world * K * R * B * T / (max_ms / 1000.0)
 
 
 def barrier(world):
@@ -365,8 +384,8 @@ def run_gpu(args, w, world, rank, local):
     if T % P:
         raise SystemExit(f"--decode-steps {T} must be a multiple of --pool {P}")
     sel0 = selection_inputs(w)
-    reqs = [Request(w, dev, 1000 * w.seed + 100 * rank + r, P,
-                    host_sel=sel0 if r == 0 else None) for r in range(R)]
+    reqs = [Request(w, dev, seed, P, host_sel=sel0 if (r == 0 and rank == 0) else None)
+            for r, seed in enumerate(request_seeds(w, rank, R))]
     torch.cuda.synchronize(dev)  # state was created on the default stream
     want_cpu = rank == 0 and world == 1 and not args.no_cpu_baseline
     # the oracle's copy of request 0, taken before any kernel of ours touches it
@@ -437,8 +456,7 @@ def run_gpu(args, w, world, rank, local):
     gat_ms = [e[1].elapsed_time(e[2]) for e in evs]
     dec_ms = [e[2].elapsed_time(e[3]) for e in evs]
     max_ms = max_over_ranks(elapsed_ms, world, dev)
-    tokens = world * K * R * w.B * T
-    value = tokens / (max_ms / 1000.0)
+    value = job_tokens_per_s(world, K, R, w.B, T, max_ms)
 
     launches_dec = K * R * T
     # kernels per fused decode call (attention, plus combine if units are split)
@@ -520,41 +538,74 @@ def run_gpu(args, w, world, rank, local):
 def run_e2e(args, w, reqs, dev, stream, world):
     """Same metric through the public Python API with host buffers: the
     question vector and CME bank of each request and, every decode step, q and
-    the new token's K,V are copied in from pinned host memory and the output
-    copied back to pinned host memory.  The per-step sequence (three copies
-    in, the decode call, one copy out) is captured in a CUDA graph of P rounds,
-    as a serving loop would; selection and compaction run eagerly."""
+    the new token's K,V (one packed pinned buffer per step) are copied in and
+    the output copied back to pinned host memory.  The per-step sequence is
+    captured in a CUDA graph of P rounds, as a serving loop would: copies in
+    run on one side stream and copies out on another, so they overlap the
+    decode kernels of the other requests; each request's decode waits for its
+    own inputs and for the previous read-back of its output buffer.
+    Selection and compaction run eagerly."""
     import paper_2609_25537_gb300 as cmc
     R, T, P = args.requests, args.decode_steps, args.pool
     steps = max(1, min(args.steps, args.e2e_steps))
+    nq, nk = reqs[0].q[0].numel(), reqs[0].k_new[0].numel()
     host = []
     for r in reqs:
+        packed = torch.cat([r.q.reshape(P, -1), r.k_new.reshape(P, -1), r.v_new.reshape(P, -1)],
+                           dim=1)
+        inp_d = torch.empty(packed.shape[1], dtype=torch.bfloat16, device=dev)
         h = {
             "qemb": r.qemb.cpu().pin_memory(), "bank": r.bank.cpu().pin_memory(),
-            "q": r.q.cpu().pin_memory(), "k": r.k_new.cpu().pin_memory(),
-            "v": r.v_new.cpu().pin_memory(),
+            "inp": packed.cpu().pin_memory(), "inp_d": inp_d,
+            "q_d": inp_d[:nq].view(r.q[0].shape),
+            "k_d": inp_d[nq:nq + nk].view(r.k_new[0].shape),
+            "v_d": inp_d[nq + nk:].view(r.v_new[0].shape),
             "out": torch.empty((P,) + tuple(r.out.shape), dtype=torch.bfloat16).pin_memory(),
-            "q_d": torch.empty_like(r.q[0]), "k_d": torch.empty_like(r.k_new[0]),
-            "v_d": torch.empty_like(r.v_new[0]),
         }
         host.append(h)
+    s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
 
-    def one_step_calls(p):
-        for r, h in zip(reqs, host):
-            h["q_d"].copy_(h["q"][p], non_blocking=True)
-            h["k_d"].copy_(h["k"][p], non_blocking=True)
-            h["v_d"].copy_(h["v"][p], non_blocking=True)
-            r.decode(p, q=h["q_d"], k_new=h["k_d"], v_new=h["v_d"], mode=args.tier1)
-            h["out"][p].copy_(r.out, non_blocking=True)
+    def rounds():
+        """P rounds of R decode steps with their copies; returns after joining
+        the side streams back into `stream`."""
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        s_in.wait_event(fork)
+        s_out.wait_event(fork)
+        done = [None] * R   # decode finished (its inputs and output are final)
+        freed = [None] * R  # read-back of the output finished
+        for p in range(P):
+            for i, (r, h) in enumerate(zip(reqs, host)):
+                with torch.cuda.stream(s_in):
+                    if done[i] is not None:
+                        s_in.wait_event(done[i])
+                    h["inp_d"].copy_(h["inp"][p], non_blocking=True)
+                    ready = torch.cuda.Event()
+                    ready.record(s_in)
+                stream.wait_event(ready)
+                if freed[i] is not None:
+                    stream.wait_event(freed[i])
+                with torch.cuda.stream(stream):
+                    r.decode(p, q=h["q_d"], k_new=h["k_d"], v_new=h["v_d"], mode=args.tier1)
+                done[i] = torch.cuda.Event()
+                done[i].record(stream)
+                with torch.cuda.stream(s_out):
+                    s_out.wait_event(done[i])
+                    h["out"][p].copy_(r.out, non_blocking=True)
+                    freed[i] = torch.cuda.Event()
+                    freed[i].record(s_out)
+        for side in (s_in, s_out):
+            j = torch.cuda.Event()
+            j.record(side)
+            stream.wait_event(j)
 
     graph = None
     try:
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            for p in range(P):
-                one_step_calls(p)
+            rounds()
         graph = g
-    except Exception as e:  # capture of host copies unsupported: run eagerly
+    except Exception as e:  # capture unsupported here: run the same calls eagerly
         print(f"e2e: graph capture failed ({type(e).__name__}: {e}); eager loop", file=sys.stderr)
         torch.cuda.synchronize(dev)
 
@@ -566,12 +617,11 @@ def run_e2e(args, w, reqs, dev, stream, world):
                 cmc.score_select(r.qemb, r.bank, w.k, idx_out=r.idx, workspace=r.sel_ws)
                 if args.tier1 == "dense":
                     r.gather()
-            if graph is not None:
-                for _ in range(T // P):
+            for _ in range(T // P):
+                if graph is not None:
                     graph.replay()
-            else:
-                for t in range(T):
-                    one_step_calls(t % P)
+                else:
+                    rounds()
         stream.synchronize()
 
     step()  # warm-up
@@ -581,10 +631,9 @@ def run_e2e(args, w, reqs, dev, stream, world):
         step()
     el = time.perf_counter() - t0
     el = max_over_ranks(el, world, dev)
-    r0 = reqs[0]
-    h2d = R * (r0.qemb.numel() * 4 + r0.bank.numel() * 4
-               + T * 2 * (r0.q[0].numel() + r0.k_new[0].numel() + r0.v_new[0].numel()))
-    d2h = R * T * r0.out.numel() * 2
+    h2d = R * (reqs[0].qemb.numel() * 4 + reqs[0].bank.numel() * 4
+               + T * 2 * host[0]["inp_d"].numel())
+    d2h = R * T * reqs[0].out.numel() * 2
     return {"value": world * steps * R * w.B * T / el, "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
             "per_step_graph": graph is not None}

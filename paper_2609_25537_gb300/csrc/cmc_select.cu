@@ -27,7 +27,7 @@ namespace cmc {
 
 constexpr int kScoreThreads = 256;
 constexpr int kScoreUnroll = 4;
-constexpr int kSelectThreads = 1024;
+constexpr int kSelectThreads = 512;
 
 __global__ void __launch_bounds__(kScoreThreads)
 cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ bank, int N, int D,
@@ -101,38 +101,45 @@ cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ ban
   }
 }
 
-// Exclusive block-wide prefix count of a per-thread flag (1024 threads).
-// `warp_sums` is a 32-entry shared scratch array; returns the exclusive count
-// for this thread and the block total in *total.
-__device__ __forceinline__ uint32_t block_exclusive_count(bool flag, uint32_t* warp_sums,
-                                                          uint32_t* total) {
+// Exclusive prefix sum of one value per thread over the block (kSelectThreads
+// threads, warps in order); `wsum` is a kSelectThreads/32-entry shared array
+// used by this call only.  Returns this thread's exclusive prefix; *total gets
+// the block total.
+__device__ __forceinline__ uint32_t block_exclusive_sum(uint32_t v, uint32_t* wsum, uint32_t* total) {
+  constexpr int kW = kSelectThreads / 32;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const uint32_t ballot = __ballot_sync(0xffffffffu, flag);
-  const uint32_t lane_ex = __popc(ballot & ((1u << lane) - 1u));
-  if (lane == 0) warp_sums[warp] = __popc(ballot);
-  __syncthreads();
-  if (warp == 0) {
-    const uint32_t v = (lane < (int)(blockDim.x >> 5)) ? warp_sums[lane] : 0u;
-    uint32_t inc = v;
+  uint32_t inc = v;
 #pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t t = __shfl_up_sync(0xffffffffu, inc, off);
-      if (lane >= off) inc += t;
-    }
-    warp_sums[lane] = inc - v;                       // exclusive
-    if (lane == 31) warp_sums[32] = inc;             // block total
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xffffffffu, inc, off);
+    if (lane >= off) inc += t;
   }
+  if (lane == 31) wsum[warp] = inc;
   __syncthreads();
-  const uint32_t r = warp_sums[warp] + lane_ex;
-  *total = warp_sums[32];
-  __syncthreads();  // warp_sums is reused by the next call
-  return r;
+  uint32_t before = 0, all = 0;
+#pragma unroll
+  for (int w = 0; w < kW; ++w) {
+    const uint32_t x = wsum[w];
+    before += (w < warp) ? x : 0u;
+    all += x;
+  }
+  *total = all;
+  return before + inc - v;
 }
+
+// Sequences of at most this many CMEs keep their keys in shared memory for
+// the radix passes and the compaction; longer ones re-read the scores.
+constexpr int kSelectSmemKeys = 16384;
 
 __global__ void __launch_bounds__(kSelectThreads)
 topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx_out) {
+  extern __shared__ uint32_t skeys[];
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t wsum[3][kSelectThreads / 32];
+  __shared__ uint32_t sh_prefix, sh_krem;
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
+  const int lane = tid & 31, warp = tid >> 5;
   pdl_wait();  // the scores of the kernel before
   pdl_trigger();
   const float* s = scores + static_cast<long long>(b) * N;
@@ -142,70 +149,99 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
     for (int j = tid; j < N; j += blockDim.x) out[j] = j;
     return;
   }
-  __shared__ uint32_t hist[256];
-  __shared__ uint32_t sh_prefix, sh_krem;
-  __shared__ uint32_t warp_sums[33];
+  const bool in_smem = N <= kSelectSmemKeys;
+  for (int j = tid; j < 256; j += blockDim.x) hist[j] = 0u;
+  if (in_smem)
+    for (int j = tid; j < N; j += blockDim.x) skeys[j] = orderable(s[j]);
+  __syncthreads();
+  auto key_at = [&](int j) -> uint32_t { return in_smem ? skeys[j] : orderable(s[j]); };
 
+  // Radix select, 8 bits a pass from the top: after the passes `prefix` is the
+  // key T of the k-th largest score and krem of the keys equal to T are kept.
   uint32_t prefix = 0u, mask = 0u, krem = static_cast<uint32_t>(k);
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
-    for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0u;
-    __syncthreads();
-    for (int j = tid; j < N; j += blockDim.x) {
-      const uint32_t key = orderable(s[j]);
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    // Scores cluster (cosines near 0 share their top bits), so lanes that hit
+    // the same bin add their count with one atomic (warp-aggregated).
+    for (int base = 0; base < N; base += blockDim.x) {
+      const int j = base + tid;
+      const uint32_t key = j < N ? key_at(j) : 0u;
+      const bool part = j < N && (key & mask) == prefix;
+      const uint32_t bin = part ? ((key >> shift) & 255u) : 0xFFFFFFFFu;
+      const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+      if (part && lane == __ffs(peers) - 1) atomicAdd(&hist[bin], __popc(peers));
     }
     __syncthreads();
-    if (tid < 32) {
-      // lane l owns digits 255-8l down to 248-8l; scan from the top digit down
-      const int lane = tid;
-      uint32_t c = 0;
-#pragma unroll
-      for (int t = 0; t < 8; ++t) c += hist[255 - 8 * lane - t];
-      uint32_t inc = c;
+    // Threads 0..255 own the digits from the top (255 - tid): an inclusive
+    // scan over them counts the matching keys at or above each digit; the one
+    // thread whose digit holds the krem-th key records it.  Reading a bin also
+    // clears it for the next pass.
+    uint32_t c = 0u, inc = 0u;
+    if (tid < 256) {
+      c = hist[255 - tid];
+      hist[255 - tid] = 0u;
+      inc = c;
 #pragma unroll
       for (int off = 1; off < 32; off <<= 1) {
         const uint32_t t = __shfl_up_sync(0xffffffffu, inc, off);
         if (lane >= off) inc += t;
       }
-      const uint32_t hit = __ballot_sync(0xffffffffu, inc >= krem);
-      const int first = __ffs(hit) - 1;  // krem <= count of matching keys, so hit != 0
-      if (lane == first) {
-        uint32_t above = inc - c;  // keys in digits above this lane's range
-        for (int t = 0; t < 8; ++t) {
-          const int digit = 255 - 8 * lane - t;
-          const uint32_t h = hist[digit];
-          if (above + h >= krem) {
-            sh_prefix = prefix | (static_cast<uint32_t>(digit) << shift);
-            sh_krem = krem - above;
-            break;
-          }
-          above += h;
-        }
+      if (lane == 31) wsum[0][warp] = inc;
+    }
+    __syncthreads();
+    if (tid < 256) {
+      for (int w = 0; w < warp; ++w) inc += wsum[0][w];
+      const uint32_t excl = inc - c;
+      if (excl < krem && inc >= krem) {
+        sh_prefix = prefix | (static_cast<uint32_t>(255 - tid) << shift);
+        sh_krem = krem - excl;
       }
     }
     __syncthreads();
     prefix = sh_prefix;
     krem = sh_krem;
     mask |= 0xFFu << shift;
-    __syncthreads();
   }
 
-  // prefix == T, the key of the k-th largest score; krem keys equal to T are needed.
+  // Ordered compaction: keys > T, and the first krem keys == T in index
+  // order, written in ascending index order.  Each thread owns a run of
+  // consecutive keys of a chunk; two block scans place its outputs.
   const uint32_t T = prefix;
-  uint32_t run_sel = 0u, run_eq = 0u;
-  for (int base = 0; base < N; base += blockDim.x) {
-    const int j = base + tid;
-    const uint32_t key = (j < N) ? orderable(s[j]) : 0u;
-    const bool gt = (j < N) && key > T;
-    const bool eq = (j < N) && key == T;
+  const int per = (N + static_cast<int>(blockDim.x) - 1) / static_cast<int>(blockDim.x);
+  const int C = per < 32 ? per : 32;  // keys per thread and chunk
+  const int chunk = C * static_cast<int>(blockDim.x);
+  uint32_t run_eq = 0u, run_sel = 0u;
+  for (int base = 0; base < N; base += chunk) {
+    const int j0 = base + tid * C;
+    uint32_t n_eq = 0u;
+    for (int e = 0; e < C; ++e) {
+      const int j = j0 + e;
+      if (j < N && key_at(j) == T) ++n_eq;
+    }
     uint32_t eq_total, sel_total;
-    const uint32_t eq_rank = run_eq + block_exclusive_count(eq, warp_sums, &eq_total);
-    const bool sel = gt || (eq && eq_rank < krem);
-    const uint32_t slot = run_sel + block_exclusive_count(sel, warp_sums, &sel_total);
-    if (sel && slot < static_cast<uint32_t>(k)) out[slot] = j;  // exactly k are selected
+    const uint32_t eq0 = run_eq + block_exclusive_sum(n_eq, wsum[1], &eq_total);
+    uint32_t n_sel = 0u, r = eq0;
+    for (int e = 0; e < C; ++e) {
+      const int j = j0 + e;
+      if (j < N) {
+        const uint32_t key = key_at(j);
+        if (key > T) ++n_sel;
+        else if (key == T) n_sel += (r++ < krem) ? 1u : 0u;
+      }
+    }
+    uint32_t slot = run_sel + block_exclusive_sum(n_sel, wsum[2], &sel_total);
+    r = eq0;
+    for (int e = 0; e < C; ++e) {
+      const int j = j0 + e;
+      if (j < N) {
+        const uint32_t key = key_at(j);
+        const bool sel = key > T || (key == T && r++ < krem);
+        if (sel && slot < static_cast<uint32_t>(k)) out[slot++] = j;  // exactly k are selected
+      }
+    }
     run_eq += eq_total;
     run_sel += sel_total;
+    __syncthreads();  // wsum[1], wsum[2] are reused by the next chunk
   }
 }
 
@@ -219,7 +255,20 @@ static int launch_score_select(const float* question_emb, const float* cme_bank,
   int st = launch_pdl(cosine_scores_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kScoreThreads),
                       0, s, question_emb, cme_bank, N, D, rows, sc);
   if (st != CMC_OK || k == 0) return st;
-  return launch_pdl(topk_select_kernel, dim3(B), dim3(kSelectThreads), 0, s,
+  static std::once_flag attr_once[64];
+  int dev = 0;
+  st = record_cuda_error(cudaGetDevice(&dev));
+  if (st != CMC_OK) return st;
+  if (dev >= 0 && dev < 64) {
+    std::call_once(attr_once[dev], [&] {
+      st = record_cuda_error(cudaFuncSetAttribute(topk_select_kernel,
+                                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                  static_cast<int>(kSelectSmemKeys * sizeof(uint32_t))));
+    });
+    if (st != CMC_OK) return st;
+  }
+  const size_t smem = (N <= kSelectSmemKeys && k < N) ? static_cast<size_t>(N) * sizeof(uint32_t) : 0;
+  return launch_pdl(topk_select_kernel, dim3(B), dim3(kSelectThreads), smem, s,
                     static_cast<const float*>(sc), N, k, idx_out);
 }
 
