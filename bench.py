@@ -518,7 +518,7 @@ def run_gpu(args, w, world, rank, local):
         "variant": variant,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
-                     "kernel": ("fused decode step: two_tier_attn_kernel<128,4,fused,3>"
+                     "kernel": (f"fused decode step: two_tier_attn_kernel<{w.d},{w.Hq // w.Hkv},fused,3>"
                                 + (" (one CTA per unit, no combine launch)" if step_launches == 1
                                    else " + two_tier_combine_kernel")),
                      "bytes_per_launch": nbytes, "traffic": profiled_traffic(),
