@@ -19,6 +19,10 @@ from .cmc_oracle import (
     two_tier_attention,
     decode_step,
     default_scale,
+    rope_angles,
+    rope_rotate,
+    f64_to_bf16_bits,
+    decode_step_rope,
 )
 
 __all__ = [
@@ -34,4 +38,8 @@ __all__ = [
     "two_tier_attention",
     "decode_step",
     "default_scale",
+    "rope_angles",
+    "rope_rotate",
+    "f64_to_bf16_bits",
+    "decode_step_rope",
 ]

@@ -33,6 +33,10 @@ Readings where the paper is silent (each is also listed in the design notes):
   encoded, so no rotary embedding is applied here; nothing is masked.
 * Query head h reads KV head h // (Hq / Hkv) (grouped-query attention).
 * An empty cache (no Tier-1 rows and no ring tokens) yields a zero output.
+* The decode step of a real GQA layer (decode_step_rope) rotates the new
+  query and key with rotary position embedding, which the paper's decoders
+  apply but the paper does not restate; its readings are listed above that
+  function.
 
 Parity status: every function here is pinned by the tests in
 tests/test_oracle_pins.py (closed forms, brute force, library routines,
@@ -216,3 +220,68 @@ def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new,
     ring_k, ring_v and pos are updated in place."""
     window_append(ring_k, ring_v, pos, k_new, v_new)
     return two_tier_attention(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, scale)
+
+
+# ----------------------------------------------------------------------------
+# Decode step of a real GQA layer: rotary position embedding, then the step
+# ----------------------------------------------------------------------------
+#
+# The paper runs frozen HuggingFace decoders (Llama-3, Mistral), which apply
+# rotary position embedding (RoPE) to queries and keys and cache the rotated
+# keys; it does not restate RoPE.  Readings used here:
+#   * the half-split pairing of those implementations: element i is paired
+#     with element i + d/2 and the pair is rotated by the angle
+#     p * theta^(-2i/d), i < d/2;
+#   * positions continue after the prefill input [M* || C_local || q]
+#     ("KV cache assembly"): the token appended as number pos[b] of the ring
+#     sits at position rope_offset + pos[b], where rope_offset counts the
+#     positions before the ring (k, the Tier-1 rows);
+#   * the rotated key is stored in the cache in bf16 (round to nearest even);
+#     the query is used unrounded.
+
+def rope_angles(d: int, p: float, theta: float) -> np.ndarray:
+    """Rotation angle of each of the d/2 pairs at position p: p * theta^(-2i/d)."""
+    i = np.arange(d // 2, dtype=np.float64)
+    return float(p) * np.power(float(theta), -2.0 * i / d)
+
+
+def rope_rotate(x: np.ndarray, p: float, theta: float) -> np.ndarray:
+    """Rotate the last axis of x (fp64 or bf16 bits) by position p: the pair
+    (x_i, x_{i+d/2}) becomes (x_i cos a_i - x_{i+d/2} sin a_i,
+    x_{i+d/2} cos a_i + x_i sin a_i).  Returns fp64."""
+    x = bf16_to_f64(x)
+    d = x.shape[-1]
+    a = rope_angles(d, p, theta)
+    c, s = np.cos(a), np.sin(a)
+    x1, x2 = x[..., : d // 2], x[..., d // 2:]
+    return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
+
+
+def f64_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """fp64 -> bf16 bit patterns, rounding to nearest even in one step (the
+    8 significant bits of bf16; finite values in bf16 range)."""
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)                         # x = m 2^e, 0.5 <= |m| < 1
+    y = np.ldexp(np.round(m * 256.0) / 256.0, e)  # np.round: half to even
+    return (y.astype(np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+
+
+def decode_step_rope(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new,
+                     theta: float, rope_offset: int, scale: Optional[float] = None
+                     ) -> np.ndarray:
+    """One decode step of a GQA layer with rotary position embedding.
+
+    q: [B, L, Hq, d] and k_new: [B, L, Hkv, d] are taken before rotation.  For
+    each sequence, position p = rope_offset + pos[b] (pos before the append):
+    the rotated key (bf16) and the value are appended to the ring, then the
+    rotated query attends over [Tier-1 | Tier-2].  ring_k, ring_v and pos are
+    updated in place.  Returns fp64 [B, L, Hq, d]."""
+    B = q.shape[0]
+    q_rot = np.empty(q.shape, dtype=np.float64)
+    k_rot = np.empty(np.shape(k_new), dtype=np.uint16)
+    for b in range(B):
+        p = rope_offset + int(pos[b])
+        q_rot[b] = rope_rotate(q[b], p, theta)
+        k_rot[b] = f64_to_bf16_bits(rope_rotate(k_new[b], p, theta))
+    window_append(ring_k, ring_v, pos, k_rot, v_new)
+    return two_tier_attention(q_rot, tier1_k, tier1_v, idx, ring_k, ring_v, pos, scale)

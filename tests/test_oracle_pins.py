@@ -379,3 +379,121 @@ def test_bf16_inputs_are_read_exactly():
     bits = f32_to_bf16_bits(x)
     t = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
     np.testing.assert_array_equal(oracle.bf16_to_f64(bits), t)
+
+
+# ----------------------------------------------------------------------------
+# Rotary position embedding of the GQA-layer decode step (decoders' RoPE)
+# ----------------------------------------------------------------------------
+
+def test_rope_closed_forms():
+    # d = 2: one pair rotated by angle p (theta^0 = 1)
+    for p in (0.0, 0.5, 3.0, 1000.0):
+        np.testing.assert_allclose(oracle.rope_rotate(np.array([1.0, 0.0]), p, 10000.0),
+                                   [math.cos(p), math.sin(p)], rtol=0, atol=1e-15)
+        np.testing.assert_allclose(oracle.rope_rotate(np.array([0.0, 1.0]), p, 10000.0),
+                                   [-math.sin(p), math.cos(p)], rtol=0, atol=1e-15)
+    # angle of pair i is p * theta^(-2i/d): d = 128, theta = 10^4 -> pair 32 is p / 100
+    a = oracle.rope_angles(128, 7.0, 10000.0)
+    assert a[0] == 7.0 and a[32] == pytest.approx(0.07, rel=1e-14)
+    assert a[63] == pytest.approx(7.0 * 10000.0 ** (-126 / 128), rel=1e-14)
+    # position 0 is the identity
+    x = np.random.default_rng(0).standard_normal((3, 64))
+    np.testing.assert_array_equal(oracle.rope_rotate(x, 0, 500000.0), x)
+
+
+def test_rope_matches_complex_rotation_of_half_split_pairs():
+    """Independent formulation: z_i = x_i + 1j * x_{i + d/2} times e^{1j a_i}."""
+    rng = np.random.default_rng(1)
+    d, theta = 128, 500000.0
+    x = rng.standard_normal((5, d))
+    for p in (1, 17, 3639, 131071):
+        i = np.arange(d // 2)
+        z = (x[:, : d // 2] + 1j * x[:, d // 2:]) * np.exp(1j * p * theta ** (-2.0 * i / d))
+        want = np.concatenate([z.real, z.imag], axis=1)
+        np.testing.assert_allclose(oracle.rope_rotate(x, p, theta), want, rtol=0, atol=1e-12)
+
+
+def test_rope_relative_position_and_composition():
+    rng = np.random.default_rng(2)
+    d, theta = 64, 10000.0
+    q, k = rng.standard_normal(d), rng.standard_normal(d)
+    for m, n in ((5, 3), (100, 7), (2000, 1999)):
+        lhs = oracle.rope_rotate(q, m, theta) @ oracle.rope_rotate(k, n, theta)
+        rhs = oracle.rope_rotate(q, m - n, theta) @ k
+        assert lhs == pytest.approx(rhs, rel=1e-10, abs=1e-10)
+    np.testing.assert_allclose(oracle.rope_rotate(oracle.rope_rotate(q, 30, theta), 12, theta),
+                               oracle.rope_rotate(q, 42, theta), rtol=0, atol=1e-12)
+    # rotation preserves every pair's length
+    r = oracle.rope_rotate(q, 77, theta)
+    np.testing.assert_allclose(r[: d // 2] ** 2 + r[d // 2:] ** 2,
+                               q[: d // 2] ** 2 + q[d // 2:] ** 2, rtol=1e-12)
+
+
+def test_f64_to_bf16_rounds_to_nearest_even():
+    # values exactly representable in fp32: torch's fp32 -> bf16 cast is RNE
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal(10000).astype(np.float32).astype(np.float64)
+    want = torch.from_numpy(x.astype(np.float32)).to(torch.bfloat16).view(torch.int16).numpy()
+    np.testing.assert_array_equal(oracle.f64_to_bf16_bits(x), want.view(np.uint16))
+    # exact midpoints between bf16 neighbours of 1: 1 + 2^-8 -> 1 (even), 1 + 3*2^-8 -> 1 + 2^-6
+    got = oracle.f64_to_bf16_bits(np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -1.0 - 2.0 ** -8]))
+    assert got.tolist() == [0x3F80, 0x3F82, 0xBF80]
+    # a value just above a midpoint (not representable in fp32) rounds up
+    assert oracle.f64_to_bf16_bits(np.array([1.0 + 2.0 ** -8 + 2.0 ** -40]))[0] == 0x3F81
+
+
+def test_rope_step_at_position_zero_is_the_plain_step():
+    w = WORKLOADS["tiny"].with_(B=2, W0=(0, 0), T=1)
+    kv = kv_inputs(w)
+    st = step_inputs(w, 0)
+    idx = np.tile(np.arange(w.k), (w.B, 1))
+    a = (kv.ring_k.copy(), kv.ring_v.copy(), kv.pos0.copy())
+    b = (kv.ring_k.copy(), kv.ring_v.copy(), kv.pos0.copy())
+    plain = oracle.decode_step(st.q, kv.tier1_k, kv.tier1_v, idx, *a, st.k_new, st.v_new)
+    rope = oracle.decode_step_rope(st.q, kv.tier1_k, kv.tier1_v, idx, *b, st.k_new, st.v_new,
+                                   theta=10000.0, rope_offset=0)
+    np.testing.assert_array_equal(plain, rope)
+    np.testing.assert_array_equal(a[0], b[0])
+
+
+def test_rope_step_scores_depend_on_relative_positions():
+    """Every key rotated at its own position and the query at the new
+    token's: shifting all positions by the same amount leaves the output
+    unchanged (the cache is built here, independently of the oracle's step)."""
+    rng = np.random.default_rng(4)
+    d, theta, n = 32, 10000.0, 9
+    keys = rng.standard_normal((n, d))
+    vals = rng.standard_normal((n, d))
+    q = rng.standard_normal(d)
+    outs = []
+    for shift in (0, 250, 4000):
+        K = np.stack([oracle.rope_rotate(keys[i], shift + i, theta) for i in range(n)])
+        qr = oracle.rope_rotate(q, shift + n - 1, theta)
+        outs.append(oracle.softmax_attention(qr, K, vals, 1 / math.sqrt(d)))
+    np.testing.assert_allclose(outs[1], outs[0], rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(outs[2], outs[0], rtol=1e-10, atol=1e-12)
+
+
+def test_rope_step_rotates_query_and_stored_key_at_offset_plus_pos():
+    w = WORKLOADS["tiny"].with_(B=2, W0=(5, 128), T=1)
+    kv = kv_inputs(w)
+    st = step_inputs(w, 0)
+    idx = np.tile(np.arange(w.k), (w.B, 1))
+    rk, rv, pos = kv.ring_k.copy(), kv.ring_v.copy(), kv.pos0.copy()
+    theta, off = 500000.0, w.k
+    out = oracle.decode_step_rope(st.q, kv.tier1_k, kv.tier1_v, idx, rk, rv, pos, st.k_new,
+                                  st.v_new, theta=theta, rope_offset=off)
+    for b, p0 in enumerate(kv.pos0):
+        slot = int(p0) % w.W
+        # the stored key is the bf16 rounding of the rotated key; the value is unchanged
+        want = oracle.f64_to_bf16_bits(oracle.rope_rotate(st.k_new[b], off + int(p0), theta))
+        np.testing.assert_array_equal(rk[b, :, :, slot], want)
+        np.testing.assert_array_equal(rv[b, :, :, slot], st.v_new[b])
+        # query head 3 of layer 0 against torch SDPA on the assembled keys
+        g = 3 // w.G
+        K, V = oracle.two_tier_kv(kv.tier1_k, kv.tier1_v, idx[b], rk, rv, int(pos[b]), b, 0, g)
+        qr = oracle.rope_rotate(st.q[b, 0, 3], off + int(p0), theta)
+        ref = F.scaled_dot_product_attention(
+            torch.from_numpy(qr)[None, None, None], torch.from_numpy(K)[None, None],
+            torch.from_numpy(V)[None, None])[0, 0, 0].numpy()
+        np.testing.assert_allclose(out[b, 0, 3], ref, rtol=1e-10, atol=1e-12)
