@@ -355,17 +355,21 @@ class Request:
         cmc.tier1_gather(self.t1k, self.t1v, self.idx, out_k=self.t1k_dense,
                          out_v=self.t1v_dense, workspace=self.ws_dense)
 
-    def decode(self, p, q=None, k_new=None, v_new=None, mode="dense"):
+    def decode(self, p, q=None, k_new=None, v_new=None, mode="dense", rope=False):
+        """One fused decode step; with `rope` the GQA-layer step that rotates
+        q and k_new (theta 5e5, the Llama-3 base; positions after the k
+        Tier-1 rows)."""
         import paper_2609_25537_gb300 as cmc
         q = self.q[p] if q is None else q
         k_new = self.k_new[p] if k_new is None else k_new
         v_new = self.v_new[p] if v_new is None else v_new
+        kw = dict(rope_theta=500000.0, rope_offset=self.idx.shape[1]) if rope else {}
         if mode == "dense":
             cmc.decode_step(q, self.t1k_dense, self.t1v_dense, None, self.ring_k, self.ring_v,
-                            self.pos, k_new, v_new, out=self.out, workspace=self.ws_dense)
+                            self.pos, k_new, v_new, out=self.out, workspace=self.ws_dense, **kw)
         else:
             cmc.decode_step(q, self.t1k, self.t1v, self.idx, self.ring_k, self.ring_v,
-                            self.pos, k_new, v_new, out=self.out, workspace=self.ws)
+                            self.pos, k_new, v_new, out=self.out, workspace=self.ws, **kw)
 
     def host_state(self):
         def bits(t):
@@ -401,15 +405,16 @@ def run_gpu(args, w, world, rank, local):
             r.gather()
             r.decode(0, mode=mode)
             r.decode(0, mode=other)
+            r.decode(0, mode=mode, rope=True)
     stream.synchronize()
 
     # one graph = P rounds of R decode launches; replayed T / P times per step
-    def capture(m):
+    def capture(m, rope=False):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             for p in range(P):
                 for r in reqs:
-                    r.decode(p, mode=m)
+                    r.decode(p, mode=m, rope=rope)
         return g
     graph = capture(mode)
     replays = T // P
@@ -470,24 +475,34 @@ def run_gpu(args, w, world, rank, local):
     select_us = 1000.0 * statistics.median(sel_ms) / R
     gather_us = 1000.0 * statistics.median(gat_ms) / R if mode == "dense" else 0.0
 
-    # the decode step with the other Tier-1 form (same state, same launch shape)
-    variant = None
-    if not args.no_variant:
-        g2 = capture(other)
+    def time_graph(g):
         with torch.cuda.stream(stream):
-            g2.replay()
+            g.replay()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             for _ in range(args.variant_replays):
-                g2.replay()
+                g.replay()
             e1.record(stream)
         stream.synchronize()
-        v_us = 1000.0 * e0.elapsed_time(e1) / (args.variant_replays * P * R)
+        return 1000.0 * e0.elapsed_time(e1) / (args.variant_replays * P * R)
+
+    # the decode step with the other Tier-1 form, and the GQA-layer step with
+    # rotary embedding (same state, same launch shape)
+    variant = rope_variant = None
+    if not args.no_variant:
+        g2 = capture(other)
+        v_us = time_graph(g2)
         v_bytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W,
                                     gather=other == "gather")
         variant = {"tier1": other, "us_per_launch": v_us,
                    "achieved_gbs": v_bytes / (v_us * 1e-6) / 1e9}
         del g2
+        g3 = capture(mode, rope=True)
+        r_us = time_graph(g3)
+        rope_variant = {"step": "GQA layer: rotary embedding of q and k_new + append + attention",
+                        "tier1": mode, "us_per_launch": r_us,
+                        "achieved_gbs": nbytes / (r_us * 1e-6) / 1e9}
+        del g3
 
     # e2e through the Python API with pinned host buffers
     e2e = run_e2e(args, w, reqs, dev, stream, world) if not args.no_e2e else None
@@ -516,6 +531,7 @@ def run_gpu(args, w, world, rank, local):
         "tier1_gather_gbs": (tier1_gather_bytes(w.B, w.L, w.Hkv, w.d, w.k) / (gather_us * 1e-6)
                              / 1e9 if gather_us > 0 else None),
         "variant": variant,
+        "rope_variant": rope_variant,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
                      "kernel": (f"fused decode step: two_tier_attn_kernel<{w.d},{w.Hq // w.Hkv},fused,3>"

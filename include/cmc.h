@@ -212,14 +212,41 @@ CMC_API int cmc_tier1_gather(const void* bank_k, const void* bank_v, const int32
                              void* stream);
 
 /*
- * Launch plan of cmc_two_tier_decode_attn (fused == 0) or cmc_decode_step
- * (fused != 0) for `dims` on the current device: *ctas receives the grid size
+ * Launch plan of cmc_two_tier_decode_attn (fused == 0), cmc_decode_step
+ * (fused == 1) or cmc_decode_step_rope (fused == 2) for `dims` on the
+ * current device: *ctas receives the grid size
  * of the attention kernel and *launches the number of kernels one call
  * enqueues (1, or 2 when some (sequence, layer, KV head) unit is split
  * between CTAs and a combine kernel merges its partial results).  No work is
  * enqueued.  Useful for sizing CUDA graphs and for counting launches.
  */
 CMC_API int cmc_decode_attn_plan(const cmc_dims* dims, int fused, int* ctas, int* launches);
+
+/*
+ * The decode step of a real GQA layer: cmc_decode_step with rotary position
+ * embedding applied inside the same launch.  The decoders of Section 2.5
+ * (Llama-3, Mistral) rotate queries and keys and cache the rotated keys; the
+ * paper does not restate the rotation, so it follows the half-split pairing
+ * of those decoders: element i pairs with element i + d/2 and the pair is
+ * rotated by the angle p * rope_theta^(-2i/d).
+ *
+ * q and k_new are taken BEFORE rotation.  For sequence b the new token's
+ * position is p = rope_offset + pos[b] (pos[b] before the append; rope_offset
+ * counts the positions that precede the ring, e.g. k for the Tier-1 rows of
+ * the prefill input [M* | C_local | q]).  The kernel rotates every query head
+ * and the new key at p, appends the rotated key (bf16, round to nearest even)
+ * and the value to the ring, and attends with the rotated query over
+ * [Tier-1 | Tier-2] exactly as cmc_decode_step.  Angles are formed in double
+ * precision.  Other arguments are those of cmc_decode_step.
+ *
+ * Errors: as cmc_decode_step; rope_theta must be positive and finite and
+ * 0 <= rope_offset <= 2^53 (else CMC_ERR_RANGE).
+ */
+CMC_API int cmc_decode_step_rope(const void* q, const void* tier1_k, const void* tier1_v,
+                                 const int32_t* idx, void* ring_k, void* ring_v, int64_t* pos,
+                                 const void* k_new, const void* v_new, const cmc_dims* dims,
+                                 float scale, double rope_theta, int64_t rope_offset, void* out,
+                                 void* workspace, size_t workspace_bytes, void* stream);
 
 /* Copies the device status word of an attention workspace (CMC_DEVFLAG_*
  * bits) into *flags, waiting for `stream`, and clears it when `clear` != 0. */

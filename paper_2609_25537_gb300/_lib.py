@@ -23,6 +23,7 @@ EXPORTS = (
     "cmc_decode_attn_workspace_size",
     "cmc_two_tier_decode_attn",
     "cmc_decode_step",
+    "cmc_decode_step_rope",
     "cmc_tier1_gather",
     "cmc_decode_attn_plan",
     "cmc_read_status",
@@ -81,6 +82,9 @@ _SIGNATURES = {
                                       ctypes.c_float, _vp, _vp, _sz, _vp]),
     "cmc_decode_step": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _dims_p,
                              ctypes.c_float, _vp, _vp, _sz, _vp]),
+    "cmc_decode_step_rope": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _dims_p,
+                                  ctypes.c_float, ctypes.c_double, ctypes.c_int64, _vp, _vp, _sz,
+                                  _vp]),
     "cmc_tier1_gather": (_i, [_vp, _vp, _vp, _dims_p, _vp, _vp, _vp, _vp]),
     "cmc_decode_attn_plan": (_i, [_dims_p, _i, ctypes.POINTER(_i), ctypes.POINTER(_i)]),
     "cmc_read_status": (_i, [_vp, _i, ctypes.POINTER(ctypes.c_uint32), _vp]),

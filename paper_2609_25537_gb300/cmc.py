@@ -133,11 +133,12 @@ def decode_attn_workspace_size(dims: CmcDims) -> int:
     return int(lib().cmc_decode_attn_workspace_size(ctypes.byref(dims)))
 
 
-def decode_attn_plan(dims: CmcDims, fused: bool = True) -> Tuple[int, int]:
+def decode_attn_plan(dims: CmcDims, fused: bool = True, rope: bool = False) -> Tuple[int, int]:
     """(grid size, kernel launches per call) of the attention entry points for
     `dims` on the current device; see cmc_decode_attn_plan."""
     ctas, launches = ctypes.c_int(0), ctypes.c_int(0)
-    st = lib().cmc_decode_attn_plan(ctypes.byref(dims), 1 if fused else 0, ctypes.byref(ctas),
+    mode = 2 if rope else (1 if fused else 0)
+    st = lib().cmc_decode_attn_plan(ctypes.byref(dims), mode, ctypes.byref(ctas),
                                     ctypes.byref(launches))
     check(st, "cmc_decode_attn_plan")
     return int(ctas.value), int(launches.value)
@@ -221,9 +222,14 @@ def two_tier_decode_attn(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, *,
 
 def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, *,
                 scale: Optional[float] = None, out: Optional[torch.Tensor] = None,
-                workspace: Optional[DecodeWorkspace] = None) -> torch.Tensor:
+                workspace: Optional[DecodeWorkspace] = None,
+                rope_theta: Optional[float] = None, rope_offset: int = 0) -> torch.Tensor:
     """Fused decode step: append (k_new, v_new) to the ring, then attend; see
-    cmc_decode_step.  Updates ring_k, ring_v and pos in place."""
+    cmc_decode_step.  Updates ring_k, ring_v and pos in place.
+
+    With ``rope_theta`` the step is that of a real GQA layer (see
+    cmc_decode_step_rope): q and k_new are given before rotary embedding and
+    are rotated at position ``rope_offset + pos[b]`` inside the launch."""
     dims, dev, out = _attn_args(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, out)
     _need(k_new, "k_new", torch.bfloat16, 4, dev)
     _need(v_new, "v_new", torch.bfloat16, 4, dev)
@@ -231,11 +237,18 @@ def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, *,
     if tuple(k_new.shape) != want or tuple(v_new.shape) != want:
         raise ValueError(f"k_new/v_new must be {want}")
     ws = workspace if workspace is not None else _workspace_for(dims, dev)
-    st = lib().cmc_decode_step(
-        _p(q), _p(tier1_k), _p(tier1_v), _p(idx), _p(ring_k), _p(ring_v), _p(pos),
-        _p(k_new), _p(v_new), ctypes.byref(dims), _scale(scale), _p(out), _p(ws.buf),
-        ws.nbytes, _stream(dev))
-    check(st, "cmc_decode_step")
+    if rope_theta is None:
+        st = lib().cmc_decode_step(
+            _p(q), _p(tier1_k), _p(tier1_v), _p(idx), _p(ring_k), _p(ring_v), _p(pos),
+            _p(k_new), _p(v_new), ctypes.byref(dims), _scale(scale), _p(out), _p(ws.buf),
+            ws.nbytes, _stream(dev))
+        check(st, "cmc_decode_step")
+    else:
+        st = lib().cmc_decode_step_rope(
+            _p(q), _p(tier1_k), _p(tier1_v), _p(idx), _p(ring_k), _p(ring_v), _p(pos),
+            _p(k_new), _p(v_new), ctypes.byref(dims), _scale(scale), float(rope_theta),
+            int(rope_offset), _p(out), _p(ws.buf), ws.nbytes, _stream(dev))
+        check(st, "cmc_decode_step_rope")
     return out
 
 

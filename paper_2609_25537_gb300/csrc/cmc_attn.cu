@@ -96,6 +96,8 @@ struct AttnParams {
   long long base;         // tiles per CTA (CTAs below `rem` take one more)
   long long rem;
   float scale_log2;       // softmax scale * log2(e)
+  long long rope_offset;  // rotary embedding (GQA-layer step): position of ring token 0
+  double rope_inv_freq[64];  // theta^(-2i/d) for the d/2 pairs, computed on the host
 };
 
 // ---------------------------------------------------------------------------
@@ -208,7 +210,7 @@ __device__ __forceinline__ void consumer_sync() {
 // Shared-memory layout of one pipeline stage (1024-byte aligned)
 // ---------------------------------------------------------------------------
 
-template <int D, int G>
+template <int D, int G, bool ROPE = false>
 struct Stage {
   static constexpr int kHalves = D / 64;               // 128-byte column boxes per row
   static constexpr int kK = 0;                         // K boxes [half][64 rows][128 B]
@@ -218,7 +220,8 @@ struct Stage {
   static constexpr int kQ = 0;                         // query rows [G][D] bf16
   static constexpr int kNew = G * D * 2;               // new token K row, V row (fused step)
   static constexpr int kHdr = kNew + 2 * D * 2;        // header words (H_*)
-  static constexpr int kAuxBytes = kHdr + 128;
+  static constexpr int kRope = kHdr + 128;             // rotary table: d/2 (cos, sin) pairs
+  static constexpr int kAuxBytes = kRope + (ROPE ? D * 4 : 0);
 };
 
 // Per-stage header words: rows of the tile that may hold a key, the new
@@ -227,9 +230,10 @@ struct Stage {
 // bit masks of rows 0-31 / 32-63 whose Tier-1 index is out of range.
 enum { H_NROWS = 0, H_NEWSLOT = 1, H_NEWROW = 2, H_MASKED = 3, H_BADLO = 4, H_BADHI = 5 };
 
-template <int D, int G, int NST>
+template <int D, int G, int NST, bool ROPE>
 constexpr size_t attn_smem_bytes() {
-  return 1024 /* alignment slack */ + static_cast<size_t>(NST) * (Stage<D, G>::kBytes + Stage<D, G>::kAuxBytes) +
+  return 1024 /* alignment slack */ +
+         static_cast<size_t>(NST) * (Stage<D, G, ROPE>::kBytes + Stage<D, G, ROPE>::kAuxBytes) +
          kMetaSlots * (kTileKeys * 4 + 16) +
          static_cast<size_t>(kWarps) * (2 * 8 + G * D) * sizeof(float);
 }
@@ -379,6 +383,33 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
                : "memory");
 }
 
+// Rotary embedding of a GQA-layer step: (cos, sin) of the angle
+// p * theta^(-2i/d) of pairs i = lane and lane + 32 (i < d/2) at the new
+// token's position p = rope_offset + pos.  Angles reach 10^5 rad and more, so
+// the product and its reduction to [-pi, pi] (2 pi split into a high and a
+// low part) are done in double; sine and cosine of the reduced angle in float.
+template <int D>
+__device__ __forceinline__ void rope_pairs(const AttnParams& p, long long pos, int lane,
+                                           float2 (&cs)[2]) {
+  constexpr double kTwoPiHi = 6.283185307179586;      // 2 pi rounded to double
+  constexpr double kTwoPiLo = 2.4492935982947064e-16;  // 2 pi - kTwoPiHi
+  constexpr double kInvTwoPi = 0.15915494309189535;
+  const double pp = static_cast<double>(p.rope_offset + pos);
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const int i = lane + 32 * e;
+    cs[e] = make_float2(1.f, 0.f);
+    if (i < D / 2) {
+      const double a = pp * p.rope_inv_freq[i];
+      const double n = rint(a * kInvTwoPi);
+      const double r = fma(-n, kTwoPiLo, fma(-n, kTwoPiHi, a));
+      float sn, cn;
+      sincosf(static_cast<float>(r), &sn, &cn);
+      cs[e] = make_float2(cn, sn);
+    }
+  }
+}
+
 // Producer lane 0, box tiles: what does not depend on pos -- the K/V boxes and
 // the unit's query rows -- issued as soon as the stage is free.  Two-
 // dimensional boxes of 64 consecutive rows of the ring, or of the Tier-1
@@ -412,11 +443,18 @@ __device__ __forceinline__ void issue_box_loads(const AttnParams& p, const AttnM
 // the new token's row), the new token's K/V rows in the fused step, the loads
 // of a gathered tile, and the arrive that, once every byte has landed,
 // releases the stage to the consumers.
-template <int D, int G, bool FUSED>
+template <int D, int G, bool FUSED, bool ROPE>
 __device__ __forceinline__ void finish_tile(const AttnParams& p, uint8_t* stage, uint8_t* aux,
                                             const TileCursor& c, const TileMeta& meta,
-                                            const SeqState& sq, int lane, uint64_t* full) {
-  using S = Stage<D, G>;
+                                            const SeqState& sq, const float2 (&rope)[2], int lane,
+                                            uint64_t* full) {
+  using S = Stage<D, G, ROPE>;
+  if (ROPE) {  // the sequence's rotary table travels with every tile
+    float2* tab = reinterpret_cast<float2*>(aux + S::kRope);
+    tab[lane] = rope[0];
+    if (lane + 32 < D / 2) tab[lane + 32] = rope[1];
+    __syncwarp();
+  }
   const bool t1 = c.lt < p.t1_tiles;
   int n_rows, new_row = -1;
   if (t1) {
@@ -498,10 +536,10 @@ __device__ __forceinline__ void seq_run_done(const AttnParams& p, int b, long lo
 // the CTA's tiles through NST shared-memory stages; stage s is handed over by
 // full[s] (its bytes have landed and its header is written) and handed back
 // by empty[s] (every consumer warp is done with it).
-template <int D, int G, bool FUSED, int NST>
+template <int D, int G, bool FUSED, int NST, bool ROPE>
 __global__ void __launch_bounds__(kThreads + 32)
 two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) {
-  using S = Stage<D, G>;
+  using S = Stage<D, G, ROPE>;
   constexpr int KS = D / 16;  // k-steps of the Q K^T product
   constexpr int NT = D / 8;   // n8 tiles of the output
   extern __shared__ uint8_t smem_raw[];
@@ -571,6 +609,7 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     long long run_tiles = 0;  // tiles in that run so far
     SeqState sq;
     sq.pos = 0; sq.count = 0; sq.new_slot = -1; sq.bad = true;
+    float2 rope[2] = {make_float2(1.f, 0.f), make_float2(1.f, 0.f)};
     for (int i = 0; i < n_tiles; ++i) {
       const int s = i % NST;
       if (i >= NST) {
@@ -596,10 +635,11 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
         run_b = ci.b;
         run_tiles = 0;
         sq = seq_state<FUSED>(p, meta.pos);
+        if (ROPE && !sq.bad) rope_pairs<D>(p, meta.pos, lane, rope);
       }
       ++run_tiles;
-      finish_tile<D, G, FUSED>(p, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, meta, sq, lane,
-                               &full_bar[s]);
+      finish_tile<D, G, FUSED, ROPE>(p, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, meta, sq,
+                                     rope, lane, &full_bar[s]);
       ci.next(p);
       issued = i + 1;
       __syncwarp();
@@ -653,7 +693,26 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
       if (warp == 0 && lane < 2 * (D / 8)) {
         const int which = lane / (D / 8);  // 0: K, 1: V
         const int c = lane - which * (D / 8);
-        const uint4 v = *reinterpret_cast<const uint4*>(aux + S::kNew + which * D * 2 + c * 16);
+        uint4 v = *reinterpret_cast<const uint4*>(aux + S::kNew + which * D * 2 + c * 16);
+        if (ROPE && which == 0) {
+          // rotate the new key: columns 8c .. 8c+7 with their partners in the
+          // other half (chunk c ^ d/16), round to bf16
+          const uint4 pv = *reinterpret_cast<const uint4*>(aux + S::kNew + (c ^ (D / 16)) * 16);
+          const float2* tab = reinterpret_cast<const float2*>(aux + S::kRope);
+          const int i0 = (8 * c) & (D / 2 - 1);
+          const float sg = (8 * c < D / 2) ? -1.f : 1.f;
+          const uint32_t xs[4] = {v.x, v.y, v.z, v.w};
+          const uint32_t ps[4] = {pv.x, pv.y, pv.z, pv.w};
+          uint32_t r[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float2 t0 = tab[i0 + 2 * e], t1 = tab[i0 + 2 * e + 1];
+            const float lo = fmaf(bf16lo_to_f32(xs[e]), t0.x, sg * bf16lo_to_f32(ps[e]) * t0.y);
+            const float hi = fmaf(bf16hi_to_f32(xs[e]), t1.x, sg * bf16hi_to_f32(ps[e]) * t1.y);
+            r[e] = pack_bf16_rn(lo, hi);
+          }
+          v = make_uint4(r[0], r[1], r[2], r[3]);
+        }
         *reinterpret_cast<uint4*>(stage + (which ? S::kV : S::kK) + swz(new_row, c)) = v;
         uint16_t* ring = which ? p.ring_v : p.ring_k;
         *reinterpret_cast<uint4*>(ring + (static_cast<long long>(u) * p.W + hw[H_NEWSLOT]) * D + c * 8) = v;
@@ -668,8 +727,25 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
 #pragma unroll
       for (int ks = 0; ks < KS; ++ks) {
         if (gq < G && !dead) {
-          qa[ks][0] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq) * 2);
-          qa[ks][1] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq + 8) * 2);
+          if (ROPE) {
+            // rotate the query: column c pairs with c ^ d/2 (the other half)
+            const float2* tab = reinterpret_cast<const float2*>(aux + S::kRope);
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf) {
+              const int c = 16 * ks + 2 * tq + 8 * hf;
+              const uint32_t xv = *reinterpret_cast<const uint32_t*>(qs + (gq * D + c) * 2);
+              const uint32_t pv = *reinterpret_cast<const uint32_t*>(qs + (gq * D + (c ^ (D / 2))) * 2);
+              const int i = c & (D / 2 - 1);
+              const float sg = (c < D / 2) ? -1.f : 1.f;
+              const float2 t0 = tab[i], t1 = tab[i + 1];
+              const float lo = fmaf(bf16lo_to_f32(xv), t0.x, sg * bf16lo_to_f32(pv) * t0.y);
+              const float hi = fmaf(bf16hi_to_f32(xv), t1.x, sg * bf16hi_to_f32(pv) * t1.y);
+              qa[ks][hf] = pack_bf16_rn(lo, hi);
+            }
+          } else {
+            qa[ks][0] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq) * 2);
+            qa[ks][1] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq + 8) * 2);
+          }
         }
       }
       m_run = -INFINITY;
@@ -1030,10 +1106,10 @@ struct AttnPlan {
   bool split;                 // some unit is cut between CTAs: the combine kernel runs
 };
 
-template <int D, int G, bool FUSED>
+template <int D, int G, bool FUSED, bool ROPE>
 static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
-  constexpr size_t smem = attn_smem_bytes<D, G, kStages>();
-  auto kern = two_tier_attn_kernel<D, G, FUSED, kStages>;
+  constexpr size_t smem = attn_smem_bytes<D, G, kStages, ROPE>();
+  auto kern = two_tier_attn_kernel<D, G, FUSED, kStages, ROPE>;
   static int configured[64] = {0};  // per device: attribute set and occupancy known
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
@@ -1069,57 +1145,57 @@ static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
   return CMC_OK;
 }
 
-template <int D, int G, bool FUSED>
+template <int D, int G, bool FUSED, bool ROPE>
 static int launch_attn(const AttnMaps& maps, const AttnParams& p0, long long total_tiles,
                        cudaStream_t s) {
-  constexpr size_t smem = attn_smem_bytes<D, G, kStages>();
+  constexpr size_t smem = attn_smem_bytes<D, G, kStages, ROPE>();
   AttnPlan pl;
-  int st = plan_attn<D, G, FUSED>(total_tiles, p0.tpu, &pl);
+  int st = plan_attn<D, G, FUSED, ROPE>(total_tiles, p0.tpu, &pl);
   if (st != CMC_OK) return st;
   AttnParams p = p0;
   p.base = pl.base;
   p.rem = pl.rem;
-  st = launch_pdl(two_tier_attn_kernel<D, G, FUSED, kStages>, dim3(static_cast<unsigned>(pl.ctas)),
+  st = launch_pdl(two_tier_attn_kernel<D, G, FUSED, kStages, ROPE>, dim3(static_cast<unsigned>(pl.ctas)),
                   dim3(kThreads + 32), smem, s, maps, p);
   if (st != CMC_OK || !pl.split) return st;
   return launch_pdl(two_tier_combine_kernel<D, G>, dim3(static_cast<unsigned>(total_tiles / p.tpu)),
                     dim3(kThreads), 0, s, p);
 }
 
-template <bool FUSED>
+template <bool FUSED, bool ROPE>
 static int dispatch_plan(int d, int G, long long tiles, int tpu, AttnPlan* pl) {
   if (d == 128) {
     switch (G) {
-      case 1: return plan_attn<128, 1, FUSED>(tiles, tpu, pl);
-      case 2: return plan_attn<128, 2, FUSED>(tiles, tpu, pl);
-      case 4: return plan_attn<128, 4, FUSED>(tiles, tpu, pl);
-      default: return plan_attn<128, 8, FUSED>(tiles, tpu, pl);
+      case 1: return plan_attn<128, 1, FUSED, ROPE>(tiles, tpu, pl);
+      case 2: return plan_attn<128, 2, FUSED, ROPE>(tiles, tpu, pl);
+      case 4: return plan_attn<128, 4, FUSED, ROPE>(tiles, tpu, pl);
+      default: return plan_attn<128, 8, FUSED, ROPE>(tiles, tpu, pl);
     }
   }
   switch (G) {
-    case 1: return plan_attn<64, 1, FUSED>(tiles, tpu, pl);
-    case 2: return plan_attn<64, 2, FUSED>(tiles, tpu, pl);
-    case 4: return plan_attn<64, 4, FUSED>(tiles, tpu, pl);
-    default: return plan_attn<64, 8, FUSED>(tiles, tpu, pl);
+    case 1: return plan_attn<64, 1, FUSED, ROPE>(tiles, tpu, pl);
+    case 2: return plan_attn<64, 2, FUSED, ROPE>(tiles, tpu, pl);
+    case 4: return plan_attn<64, 4, FUSED, ROPE>(tiles, tpu, pl);
+    default: return plan_attn<64, 8, FUSED, ROPE>(tiles, tpu, pl);
   }
 }
 
-template <bool FUSED>
+template <bool FUSED, bool ROPE>
 static int dispatch_attn(const AttnMaps& maps, const AttnParams& p, int d, int G, long long tiles,
                          cudaStream_t s) {
   if (d == 128) {
     switch (G) {
-      case 1: return launch_attn<128, 1, FUSED>(maps, p, tiles, s);
-      case 2: return launch_attn<128, 2, FUSED>(maps, p, tiles, s);
-      case 4: return launch_attn<128, 4, FUSED>(maps, p, tiles, s);
-      default: return launch_attn<128, 8, FUSED>(maps, p, tiles, s);
+      case 1: return launch_attn<128, 1, FUSED, ROPE>(maps, p, tiles, s);
+      case 2: return launch_attn<128, 2, FUSED, ROPE>(maps, p, tiles, s);
+      case 4: return launch_attn<128, 4, FUSED, ROPE>(maps, p, tiles, s);
+      default: return launch_attn<128, 8, FUSED, ROPE>(maps, p, tiles, s);
     }
   }
   switch (G) {
-    case 1: return launch_attn<64, 1, FUSED>(maps, p, tiles, s);
-    case 2: return launch_attn<64, 2, FUSED>(maps, p, tiles, s);
-    case 4: return launch_attn<64, 4, FUSED>(maps, p, tiles, s);
-    default: return launch_attn<64, 8, FUSED>(maps, p, tiles, s);
+    case 1: return launch_attn<64, 1, FUSED, ROPE>(maps, p, tiles, s);
+    case 2: return launch_attn<64, 2, FUSED, ROPE>(maps, p, tiles, s);
+    case 4: return launch_attn<64, 4, FUSED, ROPE>(maps, p, tiles, s);
+    default: return launch_attn<64, 8, FUSED, ROPE>(maps, p, tiles, s);
   }
 }
 
@@ -1127,12 +1203,15 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
                          const int32_t* idx, void* ring_k, void* ring_v, int64_t* pos,
                          const void* k_new, const void* v_new, const cmc_dims* dims, float scale,
                          void* out, void* workspace, size_t workspace_bytes, void* stream,
-                         bool fused) {
+                         bool fused, bool rope = false, double rope_theta = 0.0,
+                         long long rope_offset = 0) {
   int st = validate_dims(dims, true);
   if (st != CMC_OK) return st;
   const cmc_dims& m = *dims;
   if (!q || !tier1_k || !tier1_v || !ring_k || !ring_v || !pos || !out) return CMC_ERR_NULL;
   if (fused && (!k_new || !v_new)) return CMC_ERR_NULL;
+  if (rope && !(rope_theta > 0.0 && rope_theta < 1e300)) return CMC_ERR_RANGE;
+  if (rope && (rope_offset < 0 || rope_offset > (1LL << 53))) return CMC_ERR_RANGE;
   if (!aligned16(q) || !aligned16(tier1_k) || !aligned16(tier1_v) || !aligned16(ring_k) ||
       !aligned16(ring_v) || !aligned16(out))
     return CMC_ERR_ALIGN;
@@ -1183,10 +1262,14 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   p.rem = 0;
   const float sc = scale > 0.f ? scale : 1.0f / sqrtf(static_cast<float>(m.d));
   p.scale_log2 = sc * 1.4426950408889634f;
+  p.rope_offset = rope ? rope_offset : 0;
+  for (int i = 0; i < 64; ++i)
+    p.rope_inv_freq[i] = (rope && i < m.d / 2) ? pow(rope_theta, -2.0 * i / m.d) : 0.0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int G = m.Hq / m.Hkv;
-  return fused ? dispatch_attn<true>(maps, p, m.d, G, tiles, s)
-               : dispatch_attn<false>(maps, p, m.d, G, tiles, s);
+  if (rope) return dispatch_attn<true, true>(maps, p, m.d, G, tiles, s);
+  return fused ? dispatch_attn<true, false>(maps, p, m.d, G, tiles, s)
+               : dispatch_attn<false, false>(maps, p, m.d, G, tiles, s);
 }
 
 }  // namespace cmc
@@ -1213,6 +1296,16 @@ int cmc_decode_step(const void* q, const void* tier1_k, const void* tier1_v, con
                     size_t workspace_bytes, void* stream) {
   return cmc::run_attention(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, dims,
                             scale, out, workspace, workspace_bytes, stream, true);
+}
+
+int cmc_decode_step_rope(const void* q, const void* tier1_k, const void* tier1_v,
+                         const int32_t* idx, void* ring_k, void* ring_v, int64_t* pos,
+                         const void* k_new, const void* v_new, const cmc_dims* dims, float scale,
+                         double rope_theta, int64_t rope_offset, void* out, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  return cmc::run_attention(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, dims,
+                            scale, out, workspace, workspace_bytes, stream, true, true, rope_theta,
+                            rope_offset);
 }
 
 int cmc_tier1_gather(const void* bank_k, const void* bank_v, const int32_t* idx,
@@ -1252,8 +1345,10 @@ int cmc_decode_attn_plan(const cmc_dims* dims, int fused, int* ctas, int* launch
   const long long tiles = units * tpu;
   if (tiles >= (1LL << 31)) return CMC_ERR_SHAPE;
   AttnPlan pl;
-  st = fused ? dispatch_plan<true>(m.d, m.Hq / m.Hkv, tiles, tpu, &pl)
-             : dispatch_plan<false>(m.d, m.Hq / m.Hkv, tiles, tpu, &pl);
+  if (fused < 0 || fused > 2) return CMC_ERR_RANGE;
+  st = fused == 2 ? dispatch_plan<true, true>(m.d, m.Hq / m.Hkv, tiles, tpu, &pl)
+       : fused    ? dispatch_plan<true, false>(m.d, m.Hq / m.Hkv, tiles, tpu, &pl)
+                  : dispatch_plan<false, false>(m.d, m.Hq / m.Hkv, tiles, tpu, &pl);
   if (st != CMC_OK) return st;
   *ctas = static_cast<int>(pl.ctas);
   *launches = pl.split ? 2 : 1;

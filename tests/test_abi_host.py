@@ -192,3 +192,19 @@ def test_decode_attn_plan_argument_checks(L):
                                   ctypes.byref(launches)) == SHAPE
     assert L.cmc_decode_attn_plan(ctypes.byref(_dims(k=101)), 0, ctypes.byref(ctas),
                                   ctypes.byref(launches)) == RANGE
+
+
+@host_only
+def test_decode_step_rope_argument_checks(L):
+    d = _dims()
+    def r(theta=10000.0, off=0, k_new=FAKE, dims=d, wsb=1 << 30):
+        return L.cmc_decode_step_rope(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, k_new, FAKE,
+                                      ctypes.byref(dims), 0.0, theta, off, FAKE, FAKE, wsb, None)
+    assert r(theta=0.0) == RANGE
+    assert r(theta=-5.0) == RANGE
+    assert r(theta=float("inf")) == RANGE
+    assert r(theta=float("nan")) == RANGE
+    assert r(off=-1) == RANGE
+    assert r(k_new=0) == NULL
+    assert r(dims=_dims(d=96)) == SHAPE
+    assert r(wsb=16) == WORKSPACE

@@ -392,3 +392,88 @@ def test_decode_attn_plan(cuda_device):
     assert launches in (1, 2) and ctas >= 64
     if 2 * sms >= 256:
         assert (ctas, launches) == (256, 2)
+
+
+# ----------------------------------------------------------------------------
+# Decode step of a GQA layer with rotary position embedding
+# ----------------------------------------------------------------------------
+
+def _ring_close_bf16(got_bits, want_bits, what, max_frac=2e-3):
+    """Rotated keys are rounded to bf16 on both sides, from fp32 (GPU) and fp64
+    (oracle) values.  They may round to neighbouring bf16 values (one unit in
+    the last place: 2^-7 relative), and where the rotation cancels to almost 0
+    the fp32 error (~1e-7 of the inputs) shows; both rarely."""
+    a = oracle.bf16_to_f64(got_bits)
+    b = oracle.bf16_to_f64(want_bits)
+    err = np.abs(a - b)
+    bound = 2.0 ** -7 * np.abs(b) + 1e-6 * np.abs(b).max()
+    assert np.all(err <= bound), f"{what}: max excess {(err - bound).max():.3e}"
+    assert (err != 0).mean() <= max_frac, f"{what}: {(err != 0).mean():.2e} of elements differ"
+
+
+def _rope_run(w, dev, mode, theta, offset, compare_steps=None, q_std=None):
+    P = Problem(w, dev, mode=mode)
+    steps = range(w.T) if compare_steps is None else compare_steps
+    for t in range(w.T):
+        st = step_inputs(w, t, q_std=q_std)
+        out = cmc.decode_step(dev_bf16(st.q, dev), P.t1k, P.t1v, P.idx, P.ring_k, P.ring_v, P.pos,
+                              dev_bf16(st.k_new, dev), dev_bf16(st.v_new, dev), workspace=P.ws,
+                              rope_theta=theta, rope_offset=offset)
+        ref = oracle.decode_step_rope(st.q, P.kv.tier1_k, P.kv.tier1_v, P.idx_host, P.o_ring_k,
+                                      P.o_ring_v, P.o_pos, st.k_new, st.v_new, theta=theta,
+                                      rope_offset=offset)
+        if t in steps:
+            assert_attn_close(to_f64(out), ref, f"{w.name} rope step {t}")
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(P.pos.cpu().numpy(), P.o_pos)
+    np.testing.assert_array_equal(host_bits(P.ring_v), P.o_ring_v)
+    _ring_close_bf16(host_bits(P.ring_k), P.o_ring_k, f"{w.name} rotated keys")
+    assert P.ws.status() == 0
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_rope_tiny_every_step(cuda_device, mode):
+    w = WORKLOADS["tiny"]
+    _rope_run(w, cuda_device, mode, theta=10000.0, offset=w.k)
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_rope_llama_shape(cuda_device, mode):
+    w = WORKLOADS["llama3_8b"].with_(L=4, T=6)
+    _rope_run(w, cuda_device, mode, theta=500000.0, offset=w.k)
+
+
+def test_rope_large_positions_and_peaked_queries(cuda_device):
+    """Positions past 10^5 (long contexts): the angles need double precision."""
+    w = WORKLOADS["tiny"].with_(B=2, T=4, kv_std=0.3)
+    _rope_run(w, cuda_device, "dense", theta=10000.0, offset=123457, q_std=3.0 / 0.3)
+
+
+@pytest.mark.parametrize("G,d", [(1, 64), (2, 128), (8, 64), (8, 128)])
+def test_rope_head_shapes_ragged(cuda_device, G, d):
+    Hkv = 2
+    w = WORKLOADS["tiny"].with_(B=3, L=2, Hq=G * Hkv, Hkv=Hkv, d=d, N=70, k=9, W=33, T=5,
+                                kv_std=1.0, q_std=1.0 / np.sqrt(d), W0=(33, 5, 0))
+    _rope_run(w, cuda_device, "gather", theta=1e6, offset=w.k)
+
+
+def test_rope_at_position_zero_equals_the_plain_step(cuda_device):
+    """p = 0 rotates by nothing: the output and ring are bit-identical to the
+    fused step without rotary embedding."""
+    w = WORKLOADS["llama3_8b"].with_(L=2, T=1, B=2, W0=(0, 0))
+    A = Problem(w, cuda_device, mode="dense")
+    Bp = Problem(w, cuda_device, mode="dense")
+    st = step_inputs(w, 0)
+    args = lambda P: (dev_bf16(st.q, cuda_device), P.t1k, P.t1v, P.idx, P.ring_k, P.ring_v, P.pos,
+                      dev_bf16(st.k_new, cuda_device), dev_bf16(st.v_new, cuda_device))
+    out_a = cmc.decode_step(*args(A), workspace=A.ws)
+    out_b = cmc.decode_step(*args(Bp), workspace=Bp.ws, rope_theta=500000.0, rope_offset=0)
+    torch.cuda.synchronize()
+    assert torch.equal(out_a.view(torch.int16), out_b.view(torch.int16))
+    assert torch.equal(A.ring_k, Bp.ring_k) and torch.equal(A.pos, Bp.pos)
+
+
+def test_rope_plan_matches_the_fused_step(cuda_device):
+    w = WORKLOADS["llama3_8b"]
+    dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.k, w.W)
+    assert cmc.decode_attn_plan(dims, rope=True) == cmc.decode_attn_plan(dims)
