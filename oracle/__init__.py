@@ -11,6 +11,10 @@ from .cmc_oracle import (
     cosine_scores,
     select_top_k,
     score_select,
+    question_vector,
+    tier2_start,
+    cme_locate,
+    question_select,
     window_append,
     window_slots,
     softmax_attention,
@@ -30,6 +34,10 @@ __all__ = [
     "cosine_scores",
     "select_top_k",
     "score_select",
+    "question_vector",
+    "tier2_start",
+    "cme_locate",
+    "question_select",
     "window_append",
     "window_slots",
     "softmax_attention",

@@ -121,6 +121,66 @@ def score_select(question_emb: np.ndarray, cme_bank: np.ndarray, k: int
 
 
 # ----------------------------------------------------------------------------
+# Question-side prologue (Section 2.5 and the appendix on localisation
+# without annotations)
+# ----------------------------------------------------------------------------
+
+def question_vector(tokens: np.ndarray, q_len: np.ndarray) -> np.ndarray:
+    """q_vec: the mean of the question tokens' input embeddings (Section 2.5,
+    Tier-1).  tokens: [B, Lq, D]; q_len: [B] tokens per question (rows past it
+    are ignored; an empty question gives the zero vector).  Returns fp64
+    [B, D]."""
+    tokens = np.asarray(tokens)
+    B, _, D = tokens.shape
+    out = np.zeros((B, D), dtype=np.float64)
+    for b in range(B):
+        n = int(q_len[b])
+        if n > 0:
+            out[b] = tokens[b, :n].astype(np.float64).sum(axis=0) / n
+    return out
+
+
+def tier2_start(alpha: int, ctx_len: int, W: int) -> int:
+    """Start of the W-token local window centred on alpha (Section 2.5,
+    Tier-2): max(0, min(|C| - W, alpha - W/2)), W/2 rounded down."""
+    return max(0, min(int(ctx_len) - W, int(alpha) - W // 2))
+
+
+def cme_locate(cme_bank: np.ndarray, chunk_offset: np.ndarray, ctx_len: np.ndarray, W: int
+               ) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
+    """CME-guided localisation (appendix on deployment without annotations):
+    alpha = offset of the chunk that produced the highest-norm CME, and the
+    Tier-2 start derived from it.  The argmax is decided on the squared norms
+    rounded to float32 (the kernels' precision); equal norms go to the lower
+    index.  Returns (alpha [B], start [B], j_max [B]) as int64."""
+    m = np.asarray(cme_bank)
+    B, N, D = m.shape
+    alpha = np.empty(B, dtype=np.int64)
+    start = np.empty(B, dtype=np.int64)
+    jmax = np.empty(B, dtype=np.int64)
+    for b in range(B):
+        sq = np.empty(N, dtype=np.float64)
+        for j0 in range(0, N, 4096):
+            rows = m[b, j0:j0 + 4096].astype(np.float64)
+            sq[j0:j0 + 4096] = np.einsum("ij,ij->i", rows, rows)
+        sq32 = sq.astype(np.float32)
+        j = int(np.flatnonzero(sq32 == sq32.max())[0])
+        jmax[b] = j
+        alpha[b] = int(chunk_offset[b, j])
+        start[b] = tier2_start(alpha[b], ctx_len[b], W)
+    return alpha, start, jmax
+
+
+def question_select(tokens, q_len, cme_bank, k: int, chunk_offset, ctx_len, W: int):
+    """The question-side prologue: q_vec, the Tier-1 selection and the Tier-2
+    window start.  Returns (q_vec, idx, scores, alpha, start)."""
+    q = question_vector(tokens, q_len)
+    idx, scores = score_select(q, cme_bank, k)
+    alpha, start, _ = cme_locate(cme_bank, chunk_offset, ctx_len, W)
+    return q, idx, scores, alpha, start
+
+
+# ----------------------------------------------------------------------------
 # Tier-2: local-window ring (Section 2.5, Tier-2 and KV cache assembly)
 # ----------------------------------------------------------------------------
 

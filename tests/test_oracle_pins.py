@@ -497,3 +497,78 @@ def test_rope_step_rotates_query_and_stored_key_at_offset_plus_pos():
             torch.from_numpy(qr)[None, None, None], torch.from_numpy(K)[None, None],
             torch.from_numpy(V)[None, None])[0, 0, 0].numpy()
         np.testing.assert_allclose(out[b, 0, 3], ref, rtol=1e-10, atol=1e-12)
+
+
+# ----------------------------------------------------------------------------
+# Question-side prologue: q_vec, CME-guided localisation, Tier-2 start
+# ----------------------------------------------------------------------------
+
+def test_question_vector_closed_forms():
+    tok = np.zeros((3, 4, 2), dtype=np.float32)
+    tok[0, :3] = [[1.0, 2.0], [1.0, 2.0], [1.0, 2.0]]   # constant rows -> that row
+    tok[1, :2] = [[1.0, -3.0], [3.0, 5.0]]             # two rows -> their midpoint
+    tok[0, 3] = tok[1, 2:] = np.nan                     # padding is never read
+    q = oracle.question_vector(tok, np.array([3, 2, 0]))
+    np.testing.assert_array_equal(q, [[1.0, 2.0], [2.0, 1.0], [0.0, 0.0]])
+
+
+def test_question_vector_matches_torch_mean():
+    rng = np.random.default_rng(5)
+    tok = rng.standard_normal((4, 9, 33)).astype(np.float32)
+    qlen = np.array([9, 1, 5, 7])
+    q = oracle.question_vector(tok, qlen)
+    for b in range(4):
+        want = torch.from_numpy(tok[b, :qlen[b]]).double().mean(dim=0).numpy()
+        np.testing.assert_allclose(q[b], want, rtol=1e-15, atol=1e-15)
+
+
+def test_tier2_start_formula_cases():
+    # start = max(0, min(|C| - W, alpha - W/2))
+    assert oracle.tier2_start(100, 1000, 64) == 68
+    assert oracle.tier2_start(10, 1000, 64) == 0        # clamped at the context start
+    assert oracle.tier2_start(990, 1000, 64) == 936     # clamped so the window ends at |C|
+    assert oracle.tier2_start(500, 40, 64) == 0         # context shorter than the window
+    assert oracle.tier2_start(77, 1000, 63) == 46       # W/2 rounded down
+
+
+def test_cme_locate_argmax_norm_and_ties():
+    bank = np.zeros((2, 5, 3), dtype=np.float32)
+    bank[0] = [[1, 0, 0], [0, 3, 0], [2, 0, 0], [0, 0, -2.5], [1, 1, 1]]   # norms 1,3,2,2.5,1.73
+    bank[1] = [[0, 2, 0], [2, 0, 0], [0, 0, 2], [1, 1, 1], [0, 0, 0]]      # three rows tie at 2
+    offs = np.array([[0, 256, 512, 768, 1024], [0, 10, 20, 30, 40]], dtype=np.int32)
+    alpha, start, j = oracle.cme_locate(bank, offs, np.array([4096, 50]), 64)
+    assert j.tolist() == [1, 0]                         # ties -> lower index
+    assert alpha.tolist() == [256, 0]
+    assert start.tolist() == [224, 0]
+    # brute force on random banks: the row of largest Euclidean norm
+    rng = np.random.default_rng(6)
+    bank = rng.standard_normal((3, 50, 16)).astype(np.float32)
+    _, _, j = oracle.cme_locate(bank, np.tile(np.arange(50, dtype=np.int32), (3, 1)),
+                                np.full(3, 100), 8)
+    for b in range(3):
+        norms = [math.sqrt(sum(float(x) ** 2 for x in row)) for row in bank[b]]
+        assert j[b] == max(range(50), key=lambda i: (norms[i], -i))
+
+
+def test_cme_locate_decides_in_float32():
+    # two squared norms that differ in fp64 but round to the same float32:
+    # the decision is a tie and goes to the lower index
+    bank = np.zeros((1, 2, 2), dtype=np.float32)
+    bank[0, 0] = [1.0, 0.0]
+    bank[0, 1] = [1.0, 2.0 ** -13]    # squared norm 1 + 2^-26 rounds to 1 in float32
+    _, _, j = oracle.cme_locate(bank, np.zeros((1, 2), dtype=np.int32), np.array([10]), 4)
+    assert j[0] == 0
+
+
+def test_question_inputs_carry_the_planted_selection():
+    """The generated tokens average to the planted question vector, so the
+    selection of the pooled vector is the planted set (margin 2e-4)."""
+    from workloads import question_inputs
+    w = WORKLOADS["tiny"].with_(B=3)
+    si = selection_inputs(w)
+    qi = question_inputs(w, si)
+    q, idx, _, alpha, start = oracle.question_select(qi.tokens, qi.q_len, si.cme_bank, w.k,
+                                                     qi.chunk_offset, qi.ctx_len, w.W)
+    np.testing.assert_allclose(q, si.question_emb, rtol=0, atol=1e-6)
+    np.testing.assert_array_equal(idx, si.planted_idx)
+    assert np.all((0 <= start) & (start <= qi.ctx_len - w.W))

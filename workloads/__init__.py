@@ -8,9 +8,11 @@ method's arithmetic (no cosine scoring, no top-k selection, no attention).
 from .configs import Workload, WORKLOADS, ablation_workloads, get_workload
 from .generate import (
     SelectionInputs,
+    QuestionInputs,
     KVInputs,
     StepInputs,
     selection_inputs,
+    question_inputs,
     kv_inputs,
     step_inputs,
     random_tier1_indices,
@@ -24,9 +26,11 @@ __all__ = [
     "ablation_workloads",
     "get_workload",
     "SelectionInputs",
+    "QuestionInputs",
     "KVInputs",
     "StepInputs",
     "selection_inputs",
+    "question_inputs",
     "kv_inputs",
     "step_inputs",
     "random_tier1_indices",

@@ -46,6 +46,7 @@ _TAGS = {
     "step_k": 10,
     "step_v": 11,
     "idx": 12,
+    "question_tokens": 13,
 }
 
 
@@ -159,6 +160,43 @@ def selection_inputs(w: Workload, attempt: int = 0, batch: Optional[range] = Non
         question_emb=q_out, cme_bank=bank,
         planted_idx=None if planted is None else np.stack(planted),
     )
+
+
+@dataclass
+class QuestionInputs:
+    tokens: np.ndarray        # float32 [B, Lq, D]: input embeddings of the question tokens
+    q_len: np.ndarray         # int32 [B]: tokens of each question (rows past it are padding)
+    chunk_offset: np.ndarray  # int32 [B, N]: context position of the chunk behind CME j
+    ctx_len: np.ndarray       # int32 [B]: context length |C| in tokens
+
+
+def question_inputs(w: Workload, si: SelectionInputs, Lq: int = 24, chunk: int = 256,
+                    ratio: int = 4, batch: Optional[range] = None) -> QuestionInputs:
+    """Question-side inputs around the question vectors of `si`.
+
+    Each question has q_len tokens (24, 22, 20, ... ragged across sequences):
+    the planted question vector plus noise of zero mean, so that the tokens'
+    mean is that vector and the planted top-k margin carries over; padding
+    rows hold other noise.  The context is cut into chunks of `chunk` tokens,
+    each giving chunk / ratio consecutive CMEs, so CME j comes from the chunk
+    at (j // (chunk / ratio)) * chunk and |C| = N * ratio."""
+    seqs = range(w.B) if batch is None else batch
+    nb = len(seqs)
+    tokens = np.empty((nb, Lq, w.D), dtype=np.float32)
+    q_len = np.empty(nb, dtype=np.int32)
+    per_chunk = chunk // ratio
+    offs = ((np.arange(w.N) // per_chunk) * chunk).astype(np.int32)
+    for i, b in enumerate(seqs):
+        n = max(1, Lq - 2 * (b % 5))
+        rng = _rng(w.seed, "question_tokens", b)
+        noise = rng.standard_normal((n, w.D)) * w.emb_std
+        noise -= noise.mean(axis=0)
+        tokens[i, :n] = (si.question_emb[i].astype(np.float64) + noise).astype(np.float32)
+        tokens[i, n:] = (rng.standard_normal((Lq - n, w.D)) * w.emb_std).astype(np.float32)
+        q_len[i] = n
+    return QuestionInputs(tokens=tokens, q_len=q_len,
+                          chunk_offset=np.tile(offs, (nb, 1)),
+                          ctx_len=np.full(nb, w.N * ratio, dtype=np.int32))
 
 
 # ----------------------------------------------------------------------------
