@@ -58,7 +58,8 @@ sys.path.insert(0, ROOT)
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-from workloads import WORKLOADS, kv_inputs, selection_inputs, step_inputs  # noqa: E402
+from workloads import (WORKLOADS, kv_inputs, question_inputs, selection_inputs,  # noqa: E402
+                       step_inputs)
 
 METRIC = ("two-tier decode-attn tokens/s and % of 8 TB/s HBM; CME top-k select µs")
 NOMINAL_HBM_GBS = 8000.0
@@ -419,17 +420,26 @@ def run_gpu(args, w, world, rank, local):
     graph = capture(mode)
     replays = T // P
 
+    # the once-per-request kernels, also as graphs (so that their times are
+    # GPU times, not Python launch rates)
+    def capture_calls(fn):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for r in reqs:
+                fn(r)
+        return g
+    g_sel = capture_calls(lambda r: r.select())
+    g_gat = capture_calls(lambda r: r.gather()) if mode == "dense" else None
+
     def one_step(ev=None):
         with torch.cuda.stream(stream):
             if ev is not None:
                 ev[0].record(stream)
-            for r in reqs:
-                r.select()
+            g_sel.replay()
             if ev is not None:
                 ev[1].record(stream)
-            if mode == "dense":
-                for r in reqs:
-                    r.gather()
+            if g_gat is not None:
+                g_gat.replay()
             if ev is not None:
                 ev[2].record(stream)
             for _ in range(replays):
@@ -504,6 +514,33 @@ def run_gpu(args, w, world, rank, local):
                         "achieved_gbs": nbytes / (r_us * 1e-6) / 1e9}
         del g3
 
+    # the question-side prologue per request (pool q_vec, score + select,
+    # CME-guided window start), L2-cold like select_us
+    prologue_us = None
+    if not args.no_variant:
+        qi = question_inputs(w, sel0, ratio=8 if w.N >= 16384 else 4)
+        tok = torch.from_numpy(qi.tokens).to(dev)
+        qlen = torch.from_numpy(qi.q_len).to(dev)
+        offs = torch.from_numpy(qi.chunk_offset).to(dev)
+        clen = torch.from_numpy(qi.ctx_len).to(dev)
+        ws_q = torch.empty(cmc.score_select_workspace_size(w.B, w.N) * 2, dtype=torch.uint8,
+                           device=dev)
+
+        g_pro = capture_calls(lambda r: cmc.question_select(
+            tok, r.bank, w.k, q_len=qlen, chunk_offset=offs, ctx_len=clen, W=w.W, workspace=ws_q))
+        with torch.cuda.stream(stream):
+            g_pro.replay()
+            times = []
+            for _ in range(5):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                g_pro.replay()
+                e1.record(stream)
+                times.append((e0, e1))
+        stream.synchronize()
+        prologue_us = 1000.0 * statistics.median(a.elapsed_time(b) for a, b in times) / R
+        del g_pro
+
     # e2e through the Python API with pinned host buffers
     e2e = run_e2e(args, w, reqs, dev, stream, world) if not args.no_e2e else None
 
@@ -527,6 +564,7 @@ def run_gpu(args, w, world, rank, local):
         "decode_us_per_launch": launch_us,
         "hbm_pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
         "select_us": select_us,
+        "question_prologue_us": prologue_us,
         "tier1_gather_us": gather_us,
         "tier1_gather_gbs": (tier1_gather_bytes(w.B, w.L, w.Hkv, w.d, w.k) / (gather_us * 1e-6)
                              / 1e9 if gather_us > 0 else None),

@@ -113,6 +113,46 @@ CMC_API int cmc_score_select(const float* question_emb, const float* cme_bank, i
                              int k, int32_t* idx_out, float* scores_out, void* workspace,
                              size_t workspace_bytes, void* stream);
 
+/* Bytes of workspace cmc_question_select needs for B sequences of N CMEs. */
+CMC_API size_t cmc_question_select_workspace_size(int B, int N);
+
+/*
+ * The question-side prologue of a request, on the device:
+ *   q_vec[b]  = mean of the first q_len[b] rows of question_tokens[b] (the
+ *               question tokens' input embeddings, mean-pooled: Section 2.5,
+ *               Tier-1); an empty question gives the zero vector;
+ *   idx[b]    = the Tier-1 selection of cmc_score_select for q_vec;
+ *   alpha[b]  = chunk_offset[b, j*] where j* is the CME of largest norm
+ *               (CME-guided localisation, the appendix on deployment without
+ *               annotations; norms compared in fp32, ties to the lower index);
+ *   start[b]  = max(0, min(ctx_len[b] - W, alpha[b] - W/2)) (W/2 rounded
+ *               down), the first context token of the W-token Tier-2 window
+ *               (Section 2.5, Tier-2).
+ *
+ *   question_tokens  fp32 [B, Lq, D]
+ *   q_len            int32 [B] tokens per question, or NULL for Lq each;
+ *                    values are clamped to [0, Lq]
+ *   cme_bank         fp32 [B, N, D]
+ *   chunk_offset     int32 [B, N] context position of the chunk behind each
+ *                    CME (same unit as ctx_len and W)
+ *   ctx_len          int32 [B] context length |C|
+ *   q_vec_out        fp32 [B, D] (required)
+ *   idx_out          int32 [B, k] ascending (may be NULL when k == 0)
+ *   alpha_out, start_out  int32 [B]; either may be NULL; when both are NULL
+ *                    chunk_offset, ctx_len and W are not used
+ *   workspace        >= cmc_question_select_workspace_size(B, N) bytes, any
+ *                    content, 16-byte aligned
+ *
+ * Limits: those of cmc_score_select, Lq >= 1, Lq * D <= 2^31, W >= 1 when
+ * localising.
+ */
+CMC_API int cmc_question_select(const float* question_tokens, const int32_t* q_len, int Lq,
+                                const float* cme_bank, int B, int N, int D, int k,
+                                const int32_t* chunk_offset, const int32_t* ctx_len, int W,
+                                float* q_vec_out, int32_t* idx_out, int32_t* alpha_out,
+                                int32_t* start_out, void* workspace, size_t workspace_bytes,
+                                void* stream);
+
 /* ------------------------------------------------------------------------ *
  * Tier-2: local-window ring append (Section 2.5, Tier-2 and the K + W + |q| *
  * bound of "KV cache assembly")                                             *

@@ -15,6 +15,7 @@ from .cmc import (  # noqa: F401
     decode_attn_workspace_size,
     decode_step,
     dims_of,
+    question_select,
     score_select,
     score_select_workspace_size,
     tier1_gather,

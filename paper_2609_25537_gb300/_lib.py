@@ -19,6 +19,8 @@ EXPORTS = (
     "cmc_last_cuda_error",
     "cmc_score_select_workspace_size",
     "cmc_score_select",
+    "cmc_question_select_workspace_size",
+    "cmc_question_select",
     "cmc_window_append",
     "cmc_decode_attn_workspace_size",
     "cmc_two_tier_decode_attn",
@@ -76,6 +78,9 @@ _SIGNATURES = {
     "cmc_last_cuda_error": (_i, []),
     "cmc_score_select_workspace_size": (_sz, [_i, _i]),
     "cmc_score_select": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _sz, _vp]),
+    "cmc_question_select_workspace_size": (_sz, [_i, _i]),
+    "cmc_question_select": (_i, [_vp, _vp, _i, _vp, _i, _i, _i, _i, _vp, _vp, _i, _vp, _vp, _vp,
+                                 _vp, _vp, _sz, _vp]),
     "cmc_window_append": (_i, [_vp, _vp, _vp, _vp, _vp, _dims_p, _vp]),
     "cmc_decode_attn_workspace_size": (_sz, [_dims_p]),
     "cmc_two_tier_decode_attn": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _dims_p,

@@ -34,6 +34,7 @@ __all__ = [
     "DecodeWorkspace",
     "score_select",
     "score_select_workspace_size",
+    "question_select",
     "window_append",
     "two_tier_decode_attn",
     "decode_step",
@@ -109,6 +110,47 @@ def score_select(question_emb: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
                                 _p(scores_out), _p(workspace), ws_bytes, _stream(dev))
     check(st, "cmc_score_select")
     return idx_out
+
+
+def question_select(question_tokens: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
+                    q_len: Optional[torch.Tensor] = None,
+                    chunk_offset: Optional[torch.Tensor] = None,
+                    ctx_len: Optional[torch.Tensor] = None, W: Optional[int] = None,
+                    workspace: Optional[torch.Tensor] = None):
+    """The question-side prologue; see cmc_question_select.  Returns
+    (q_vec fp32 [B, D], idx int32 [B, k], alpha int32 [B] or None,
+    start int32 [B] or None); alpha and start when chunk_offset, ctx_len
+    and W are given."""
+    _need(cme_bank, "cme_bank", torch.float32, 3)
+    dev = cme_bank.device
+    _need(question_tokens, "question_tokens", torch.float32, 3, dev)
+    B, N, D = cme_bank.shape
+    Bq, Lq, Dq = question_tokens.shape
+    if (Bq, Dq) != (B, D):
+        raise ValueError(f"question_tokens shape {tuple(question_tokens.shape)} != ({B}, Lq, {D})")
+    if q_len is not None:
+        _need(q_len, "q_len", torch.int32, 1, dev)
+        if int(q_len.shape[0]) != B:
+            raise ValueError("q_len must be [B]")
+    locate = chunk_offset is not None
+    if locate:
+        _need(chunk_offset, "chunk_offset", torch.int32, 2, dev)
+        _need(ctx_len, "ctx_len", torch.int32, 1, dev)
+        if tuple(chunk_offset.shape) != (B, N) or int(ctx_len.shape[0]) != B or W is None:
+            raise ValueError("chunk_offset [B, N], ctx_len [B] and W are needed together")
+    q_vec = torch.empty((B, D), dtype=torch.float32, device=dev)
+    idx = torch.empty((B, k), dtype=torch.int32, device=dev)
+    alpha = torch.empty(B, dtype=torch.int32, device=dev) if locate else None
+    start = torch.empty(B, dtype=torch.int32, device=dev) if locate else None
+    need = int(lib().cmc_question_select_workspace_size(B, N))
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    st = lib().cmc_question_select(
+        _p(question_tokens), _p(q_len), Lq, _p(cme_bank), B, N, D, k, _p(chunk_offset),
+        _p(ctx_len), int(W or 0), _p(q_vec), _p(idx), _p(alpha), _p(start), _p(workspace),
+        workspace.numel() * workspace.element_size(), _stream(dev))
+    check(st, "cmc_question_select")
+    return q_vec, idx, alpha, start
 
 
 # ----------------------------------------------------------------------------

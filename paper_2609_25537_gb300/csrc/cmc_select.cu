@@ -31,7 +31,7 @@ constexpr int kSelectThreads = 512;
 
 __global__ void __launch_bounds__(kScoreThreads)
 cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ bank, int N, int D,
-                     long long rows, float* __restrict__ scores) {
+                     long long rows, float* __restrict__ scores, float* __restrict__ sqnorm) {
   constexpr int kWarpsPerCta = kScoreThreads / 32;
   __shared__ float part[3][kWarpsPerCta];
   const int tid = threadIdx.x;
@@ -96,9 +96,39 @@ cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ ban
       if (sm > 0.f && sq > 0.f) sc = sd / (sqrtf(sm) * sqrtf(sq));
       if (sc == 0.f) sc = 0.f;  // -0 -> +0, so that -0 and +0 tie
       scores[r] = sc;
+      if (sqnorm) sqnorm[r] = sm;  // for the CME-guided localisation
     }
     __syncthreads();  // part[] is reused by the next row
   }
+}
+
+// q_vec[b] = mean of the first q_len[b] question-token embeddings (Section
+// 2.5, Tier-1): one thread per 4 columns sums the tokens in order and divides
+// by the count; an empty question gives the zero vector.
+constexpr int kPoolThreads = 256;
+
+__global__ void __launch_bounds__(kPoolThreads)
+question_pool_kernel(const float* __restrict__ tokens, const int32_t* __restrict__ q_len, int Lq,
+                     int D, float* __restrict__ q_vec) {
+  pdl_wait();
+  pdl_trigger();
+  const int b = blockIdx.y;
+  const int c4 = blockIdx.x * kPoolThreads + threadIdx.x;
+  const int D4 = D >> 2;
+  if (c4 >= D4) return;
+  int n = q_len ? q_len[b] : Lq;
+  n = n < 0 ? 0 : (n > Lq ? Lq : n);
+  const float4* t = reinterpret_cast<const float4*>(tokens + static_cast<long long>(b) * Lq * D) + c4;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i = 0; i < n; ++i) {
+    const float4 v = __ldg(t + static_cast<long long>(i) * D4);
+    acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+  }
+  if (n > 0) {
+    const float fn = static_cast<float>(n);
+    acc.x /= fn; acc.y /= fn; acc.z /= fn; acc.w /= fn;
+  }
+  reinterpret_cast<float4*>(q_vec + static_cast<long long>(b) * D)[c4] = acc;
 }
 
 // Exclusive prefix sum of one value per thread over the block (kSelectThreads
@@ -131,8 +161,54 @@ __device__ __forceinline__ uint32_t block_exclusive_sum(uint32_t v, uint32_t* ws
 // the radix passes and the compaction; longer ones re-read the scores.
 constexpr int kSelectSmemKeys = 16384;
 
+// CME-guided localisation for the Tier-2 window (optional part of the
+// selection CTA): alpha = offset of the chunk behind the CME of largest norm
+// (the argmax over the squared norms the scoring kernel wrote, ties to the
+// lower index), start = max(0, min(|C| - W, alpha - W/2)).
+struct LocateArgs {
+  float* sqnorm;                // [B, N], or NULL: no localisation
+  const int32_t* chunk_offset;  // [B, N]
+  const int32_t* ctx_len;       // [B]
+  int W;
+  int32_t* alpha_out;           // [B] (nullable)
+  int32_t* start_out;           // [B] (nullable)
+};
+
+__device__ __forceinline__ void locate_window(const LocateArgs& la, int b, int N) {
+  __shared__ float wbest[kSelectThreads / 32];
+  __shared__ int wbidx[kSelectThreads / 32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* sq = la.sqnorm + static_cast<long long>(b) * N;
+  float best = -1.f;
+  int bi = 0x7fffffff;
+  for (int j = tid; j < N; j += blockDim.x) {  // ascending j: strict > keeps the lowest index
+    const float v = sq[j];
+    if (v > best) { best = v; bi = j; }
+  }
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, best, off);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+    if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
+  }
+  if (lane == 0) { wbest[warp] = best; wbidx[warp] = bi; }
+  __syncthreads();
+  if (tid == 0) {
+    for (int w = 1; w < static_cast<int>(blockDim.x >> 5); ++w)
+      if (wbest[w] > best || (wbest[w] == best && wbidx[w] < bi)) { best = wbest[w]; bi = wbidx[w]; }
+    const long long alpha = la.chunk_offset[static_cast<long long>(b) * N + bi];
+    long long st = static_cast<long long>(la.ctx_len[b]) - la.W;
+    const long long centred = alpha - la.W / 2;
+    if (centred < st) st = centred;
+    if (st < 0) st = 0;
+    if (la.alpha_out) la.alpha_out[b] = static_cast<int32_t>(alpha);
+    if (la.start_out) la.start_out[b] = static_cast<int32_t>(st);
+  }
+}
+
 __global__ void __launch_bounds__(kSelectThreads)
-topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx_out) {
+topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx_out,
+                   const LocateArgs la) {
   extern __shared__ uint32_t skeys[];
   __shared__ uint32_t hist[256];
   __shared__ uint32_t wsum[3][kSelectThreads / 32];
@@ -142,6 +218,7 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
   const int lane = tid & 31, warp = tid >> 5;
   pdl_wait();  // the scores of the kernel before
   pdl_trigger();
+  if (la.sqnorm) locate_window(la, b, N);
   const float* s = scores + static_cast<long long>(b) * N;
   int32_t* out = idx_out + static_cast<long long>(b) * k;
   if (k <= 0) return;
@@ -245,16 +322,20 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
   }
 }
 
-// The two selection kernels, scores written to `sc` (device, B * N floats).
+// The two selection kernels, scores written to `sc` (device, B * N floats);
+// with la.sqnorm set, the squared norms too and the localisation runs in the
+// selection kernel.
 static int launch_score_select(const float* question_emb, const float* cme_bank, int B, int N,
-                               int D, int k, int32_t* idx_out, float* sc, cudaStream_t s) {
+                               int D, int k, int32_t* idx_out, float* sc, cudaStream_t s,
+                               const LocateArgs& la = LocateArgs{nullptr, nullptr, nullptr, 0,
+                                                                 nullptr, nullptr}) {
   const long long rows = static_cast<long long>(B) * N;
   long long blocks = rows;
   const long long cap = static_cast<long long>(sm_count()) * (2048 / kScoreThreads);
   if (blocks > cap) blocks = cap;
   int st = launch_pdl(cosine_scores_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kScoreThreads),
-                      0, s, question_emb, cme_bank, N, D, rows, sc);
-  if (st != CMC_OK || k == 0) return st;
+                      0, s, question_emb, cme_bank, N, D, rows, sc, la.sqnorm);
+  if (st != CMC_OK || (k == 0 && !la.sqnorm)) return st;
   static std::once_flag attr_once[64];
   int dev = 0;
   st = record_cuda_error(cudaGetDevice(&dev));
@@ -267,9 +348,10 @@ static int launch_score_select(const float* question_emb, const float* cme_bank,
     });
     if (st != CMC_OK) return st;
   }
-  const size_t smem = (N <= kSelectSmemKeys && k < N) ? static_cast<size_t>(N) * sizeof(uint32_t) : 0;
+  const size_t smem =
+      (N <= kSelectSmemKeys && k > 0 && k < N) ? static_cast<size_t>(N) * sizeof(uint32_t) : 0;
   return launch_pdl(topk_select_kernel, dim3(B), dim3(kSelectThreads), smem, s,
-                    static_cast<const float*>(sc), N, k, idx_out);
+                    static_cast<const float*>(sc), N, k, idx_out, la);
 }
 
 }  // namespace cmc
@@ -303,6 +385,46 @@ int cmc_score_select(const float* question_emb, const float* cme_bank, int B, in
   }
   return launch_score_select(question_emb, cme_bank, B, N, D, k, idx_out, sc,
                              static_cast<cudaStream_t>(stream));
+}
+
+size_t cmc_question_select_workspace_size(int B, int N) {
+  if (B < 1 || N < 1) return 0;
+  return 2 * cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256);
+}
+
+int cmc_question_select(const float* question_tokens, const int32_t* q_len, int Lq,
+                        const float* cme_bank, int B, int N, int D, int k,
+                        const int32_t* chunk_offset, const int32_t* ctx_len, int W,
+                        float* q_vec_out, int32_t* idx_out, int32_t* alpha_out,
+                        int32_t* start_out, void* workspace, size_t workspace_bytes,
+                        void* stream) {
+  using namespace cmc;
+  if (B < 1 || B > 65535 || N < 1 || N > (1 << 20) || D < 4 || D > 65536 || (D & 3) || Lq < 1 ||
+      static_cast<long long>(Lq) * D > (1LL << 31))
+    return CMC_ERR_SHAPE;
+  if (k < 0 || k > N) return CMC_ERR_RANGE;
+  const bool locate = alpha_out || start_out;
+  if (locate && W < 1) return CMC_ERR_RANGE;
+  if (!question_tokens || !cme_bank || !q_vec_out || !workspace) return CMC_ERR_NULL;
+  if (k > 0 && !idx_out) return CMC_ERR_NULL;
+  if (locate && (!chunk_offset || !ctx_len)) return CMC_ERR_NULL;
+  if (!aligned16(question_tokens) || !aligned16(cme_bank) || !aligned16(q_vec_out) ||
+      !aligned16(workspace))
+    return CMC_ERR_ALIGN;
+  for (const void* ptr : {static_cast<const void*>(q_len), static_cast<const void*>(idx_out),
+                          static_cast<const void*>(chunk_offset), static_cast<const void*>(ctx_len),
+                          static_cast<const void*>(alpha_out), static_cast<const void*>(start_out)})
+    if (reinterpret_cast<uintptr_t>(ptr) & 3) return CMC_ERR_ALIGN;
+  if (workspace_bytes < cmc_question_select_workspace_size(B, N)) return CMC_ERR_WORKSPACE;
+  float* sc = static_cast<float*>(workspace);
+  float* sq = sc + align_up(static_cast<size_t>(B) * N * sizeof(float), 256) / sizeof(float);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int D4 = D / 4;
+  int st = launch_pdl(question_pool_kernel, dim3((D4 + kPoolThreads - 1) / kPoolThreads, B),
+                      dim3(kPoolThreads), 0, s, question_tokens, q_len, Lq, D, q_vec_out);
+  if (st != CMC_OK) return st;
+  LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out};
+  return launch_score_select(q_vec_out, cme_bank, B, N, D, k, idx_out, sc, s, la);
 }
 
 }  // extern "C"

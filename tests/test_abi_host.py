@@ -208,3 +208,30 @@ def test_decode_step_rope_argument_checks(L):
     assert r(k_new=0) == NULL
     assert r(dims=_dims(d=96)) == SHAPE
     assert r(wsb=16) == WORKSPACE
+
+
+def test_question_select_workspace_size(L):
+    assert L.cmc_question_select_workspace_size(3, 100) == 2 * 1280
+    assert L.cmc_question_select_workspace_size(0, 100) == 0
+
+
+@host_only
+def test_question_select_argument_checks(L):
+    def q(tok=FAKE, qlen=0, Lq=8, bank=FAKE, B=2, N=64, D=16, k=8, offs=FAKE, clen=FAKE, W=32,
+          qv=FAKE, idx=FAKE, alpha=FAKE, start=FAKE, ws=FAKE, wsb=1 << 20):
+        return L.cmc_question_select(tok, qlen, Lq, bank, B, N, D, k, offs, clen, W, qv, idx,
+                                     alpha, start, ws, wsb, None)
+    assert q(Lq=0) == SHAPE
+    assert q(D=18) == SHAPE
+    assert q(k=65) == RANGE
+    assert q(W=0) == RANGE                       # localising needs a window
+    assert q(tok=0) == NULL
+    assert q(qv=0) == NULL
+    assert q(idx=0) == NULL
+    assert q(offs=0) == NULL                     # alpha/start requested without offsets
+    assert q(ws=0) == NULL
+    assert q(tok=FAKE + 4) == ALIGN
+    assert q(alpha=FAKE + 2) == ALIGN
+    assert q(wsb=100) == WORKSPACE
+    # no localisation asked: offsets, lengths and W are not needed
+    assert q(offs=0, clen=0, W=0, alpha=0, start=0) not in (NULL, RANGE, SHAPE, ALIGN, WORKSPACE)
