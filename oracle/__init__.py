@@ -11,6 +11,7 @@ from .cmc_oracle import (
     cosine_scores,
     select_top_k,
     score_select,
+    bridge_epilogue,
     question_vector,
     tier2_start,
     cme_locate,
@@ -34,6 +35,7 @@ __all__ = [
     "cosine_scores",
     "select_top_k",
     "score_select",
+    "bridge_epilogue",
     "question_vector",
     "tier2_start",
     "cme_locate",

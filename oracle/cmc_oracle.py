@@ -121,6 +121,28 @@ def score_select(question_emb: np.ndarray, cme_bank: np.ndarray, k: int
 
 
 # ----------------------------------------------------------------------------
+# MemoryBridge output (Section 2.2, the norm-calibrated tanh equation)
+# ----------------------------------------------------------------------------
+
+def bridge_epilogue(x: np.ndarray, gamma: np.ndarray, beta: np.ndarray, nu: float,
+                    eps: float = 1e-5) -> np.ndarray:
+    """The decoder-ready CMEs from the MemoryBridge MLP output x [rows, H_d]:
+    m_hat = LayerNorm(x) (mean and biased variance over the features, eps,
+    per-feature gamma and beta: PyTorch's default, as the hyperparameter
+    appendix states), then m = nu tanh(m_hat) min(1, 2 nu / ||nu tanh(m_hat)||)
+    (Section 2.2), so that ||m|| <= 2 nu.  Returns fp64 [rows, H_d]."""
+    x = np.asarray(x, dtype=np.float64)
+    mu = x.mean(axis=-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=-1, keepdims=True)
+    m_hat = np.asarray(gamma, np.float64) * (x - mu) / np.sqrt(var + eps) + np.asarray(beta, np.float64)
+    t = nu * np.tanh(m_hat)
+    n = np.sqrt((t * t).sum(axis=-1, keepdims=True))
+    with np.errstate(divide="ignore"):
+        f = np.minimum(1.0, np.where(n > 0, 2.0 * nu / n, np.inf))
+    return t * f
+
+
+# ----------------------------------------------------------------------------
 # Question-side prologue (Section 2.5 and the appendix on localisation
 # without annotations)
 # ----------------------------------------------------------------------------

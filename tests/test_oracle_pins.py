@@ -572,3 +572,45 @@ def test_question_inputs_carry_the_planted_selection():
     np.testing.assert_allclose(q, si.question_emb, rtol=0, atol=1e-6)
     np.testing.assert_array_equal(idx, si.planted_idx)
     assert np.all((0 <= start) & (start <= qi.ctx_len - w.W))
+
+
+# ----------------------------------------------------------------------------
+# MemoryBridge output: LayerNorm, norm-calibrated tanh, norm cap (Section 2.2)
+# ----------------------------------------------------------------------------
+
+def test_bridge_epilogue_closed_forms():
+    nu = 0.7
+    # (a, -a): LayerNorm gives (a, -a)/sqrt(a^2 + eps); 1.077 nu < 2 nu: no cap
+    a = 3.0
+    z = a / math.sqrt(a * a + 1e-5)
+    got = oracle.bridge_epilogue(np.array([[a, -a]]), np.ones(2), np.zeros(2), nu)
+    np.testing.assert_allclose(got, [[nu * math.tanh(z), -nu * math.tanh(z)]], rtol=1e-14)
+    # 16 features of +-a: ||nu tanh|| = 4 nu tanh(z) > 2 nu: scaled to norm 2 nu exactly
+    x = np.array([[a, -a] * 8])
+    got = oracle.bridge_epilogue(x, np.ones(16), np.zeros(16), nu)
+    np.testing.assert_allclose(np.linalg.norm(got), 2 * nu, rtol=1e-14)
+    np.testing.assert_allclose(got, 2 * nu * np.sign(x) / 4.0, rtol=1e-14)
+    # a constant row has zero variance: LayerNorm gives beta; zero beta -> zero vector
+    got = oracle.bridge_epilogue(np.full((1, 8), 5.0), np.ones(8), np.zeros(8), nu)
+    np.testing.assert_array_equal(got, np.zeros((1, 8)))
+
+
+def test_bridge_epilogue_against_torch_and_the_norm_bound():
+    rng = np.random.default_rng(8)
+    rows, D, nu = 37, 256, 0.9
+    x = rng.standard_normal((rows, D)) * 3 + 1
+    gamma = 1 + 0.1 * rng.standard_normal(D)
+    beta = 0.1 * rng.standard_normal(D)
+    ln = F.layer_norm(torch.from_numpy(x), (D,), torch.from_numpy(gamma), torch.from_numpy(beta),
+                      eps=1e-5)
+    t = nu * torch.tanh(ln)
+    cap = torch.clamp(2 * nu / t.norm(dim=-1, keepdim=True), max=1.0)
+    got = oracle.bridge_epilogue(x, gamma, beta, nu)
+    np.testing.assert_allclose(got, (t * cap).numpy(), rtol=1e-12, atol=1e-14)
+    norms = np.linalg.norm(got, axis=-1)
+    assert np.all(norms <= 2 * nu * (1 + 1e-12))
+    # rows under the cap are exactly nu tanh(LayerNorm(x)): shrink them below it
+    small = oracle.bridge_epilogue(x, gamma * 0.01, beta * 0.01, nu)
+    np.testing.assert_allclose(small, nu * np.tanh(F.layer_norm(
+        torch.from_numpy(x), (D,), torch.from_numpy(gamma * 0.01),
+        torch.from_numpy(beta * 0.01), eps=1e-5).numpy()), rtol=1e-12, atol=1e-15)
