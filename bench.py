@@ -516,7 +516,7 @@ def run_gpu(args, w, world, rank, local):
 
     # the question-side prologue per request (pool q_vec, score + select,
     # CME-guided window start), L2-cold like select_us
-    prologue_us = None
+    prologue_us = bridge_us = None
     if not args.no_variant:
         qi = question_inputs(w, sel0, ratio=8 if w.N >= 16384 else 4)
         tok = torch.from_numpy(qi.tokens).to(dev)
@@ -540,6 +540,22 @@ def run_gpu(args, w, world, rank, local):
         stream.synchronize()
         prologue_us = 1000.0 * statistics.median(a.elapsed_time(b) for a, b in times) / R
         del g_pro
+        # MemoryBridge output (LayerNorm, nu tanh, norm cap) on a bank-sized
+        # MLP output per request, out of place
+        scratch = torch.empty_like(reqs[0].bank)
+        g_br = capture_calls(lambda r: cmc.bridge_epilogue(r.bank, 0.8, out=scratch))
+        with torch.cuda.stream(stream):
+            g_br.replay()
+            times = []
+            for _ in range(5):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                g_br.replay()
+                e1.record(stream)
+                times.append((e0, e1))
+        stream.synchronize()
+        bridge_us = 1000.0 * statistics.median(a.elapsed_time(b) for a, b in times) / R
+        del g_br, scratch
 
     # e2e through the Python API with pinned host buffers
     e2e = run_e2e(args, w, reqs, dev, stream, world) if not args.no_e2e else None
@@ -565,6 +581,9 @@ def run_gpu(args, w, world, rank, local):
         "hbm_pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
         "select_us": select_us,
         "question_prologue_us": prologue_us,
+        "bridge_epilogue_us": bridge_us,
+        "bridge_epilogue_gbs": (8 * w.B * w.N * w.D / (bridge_us * 1e-6) / 1e9
+                                if bridge_us else None),
         "tier1_gather_us": gather_us,
         "tier1_gather_gbs": (tier1_gather_bytes(w.B, w.L, w.Hkv, w.d, w.k) / (gather_us * 1e-6)
                              / 1e9 if gather_us > 0 else None),

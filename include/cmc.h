@@ -83,6 +83,29 @@ CMC_API const char* cmc_status_string(int status);
 CMC_API int cmc_last_cuda_error(void);
 
 /* ------------------------------------------------------------------------ *
+ * MemoryBridge output (Section 2.2, the norm-calibrated tanh equation)       *
+ * ------------------------------------------------------------------------ */
+
+/*
+ * Turns the output x of the MemoryBridge MLP into decoder-ready CMEs:
+ *     m_hat = gamma * (x - mean(x)) / sqrt(var(x) + eps) + beta
+ *             (LayerNorm over the D features, biased variance: PyTorch's
+ *             default, as the paper's hyperparameter appendix states)
+ *     m     = nu tanh(m_hat) * min(1, 2 nu / ||nu tanh(m_hat)||_2)
+ * row by row, so every CME's norm is at most 2 nu (nu = s * mean embedding
+ * norm of the decoder, a scalar the caller passes).  The MLP's matrix
+ * products are plain GEMMs left to the caller.
+ *
+ *   x      fp32 [rows, D]      out  fp32 [rows, D] (may be x: in place)
+ *   gamma, beta  fp32 [D], or NULL for ones / zeros
+ *
+ * Limits: rows >= 1, 4 <= D <= 16384, D % 4 == 0; eps > 0 and nu > 0 finite.
+ */
+CMC_API int cmc_bridge_epilogue(const float* x, const float* gamma, const float* beta,
+                                int64_t rows, int D, float eps, float nu, float* out,
+                                void* stream);
+
+/* ------------------------------------------------------------------------ *
  * Tier-1: question-guided scoring and top-K selection                       *
  * (Section 2.5, the score_j equation and the top-K re-ordering after it)    *
  * ------------------------------------------------------------------------ */

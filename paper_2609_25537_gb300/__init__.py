@@ -11,6 +11,7 @@ from .cmc import (  # noqa: F401
     DEVFLAG_BAD_INDEX,
     DEVFLAG_BAD_POS,
     DEVFLAG_TIMEOUT,
+    bridge_epilogue,
     decode_attn_plan,
     decode_attn_workspace_size,
     decode_step,

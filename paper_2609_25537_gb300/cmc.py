@@ -32,6 +32,7 @@ from ._lib import CmcDims, check, lib, DEVFLAG_BAD_INDEX, DEVFLAG_BAD_POS, DEVFL
 __all__ = [
     "CmcDims",
     "DecodeWorkspace",
+    "bridge_epilogue",
     "score_select",
     "score_select_workspace_size",
     "question_select",
@@ -69,6 +70,35 @@ def _need(t: torch.Tensor, name: str, dtype: torch.dtype, ndim: int, device=None
         raise ValueError(f"{name} must be contiguous")
     if device is not None and t.device != device:
         raise ValueError(f"{name} is on {t.device}, expected {device}")
+
+
+# ----------------------------------------------------------------------------
+# MemoryBridge output
+# ----------------------------------------------------------------------------
+
+def bridge_epilogue(x: torch.Tensor, nu: float, *, gamma: Optional[torch.Tensor] = None,
+                    beta: Optional[torch.Tensor] = None, eps: float = 1e-5,
+                    out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Decoder-ready CMEs from the MemoryBridge MLP output x (fp32 [..., D]):
+    LayerNorm, nu tanh, and the 2 nu norm cap; see cmc_bridge_epilogue."""
+    _need(x, "x", torch.float32, x.dim())
+    dev = x.device
+    D = int(x.shape[-1])
+    rows = x.numel() // D if D else 0
+    for t, name in ((gamma, "gamma"), (beta, "beta")):
+        if t is not None:
+            _need(t, name, torch.float32, 1, dev)
+            if int(t.shape[0]) != D:
+                raise ValueError(f"{name} must be [{D}]")
+    if out is None:
+        out = torch.empty_like(x)
+    _need(out, "out", torch.float32, x.dim(), dev)
+    if out.shape != x.shape:
+        raise ValueError("out must have the shape of x")
+    st = lib().cmc_bridge_epilogue(_p(x), _p(gamma), _p(beta), rows, D, float(eps), float(nu),
+                                   _p(out), _stream(dev))
+    check(st, "cmc_bridge_epilogue")
+    return out
 
 
 # ----------------------------------------------------------------------------

@@ -235,3 +235,19 @@ def test_question_select_argument_checks(L):
     assert q(wsb=100) == WORKSPACE
     # no localisation asked: offsets, lengths and W are not needed
     assert q(offs=0, clen=0, W=0, alpha=0, start=0) not in (NULL, RANGE, SHAPE, ALIGN, WORKSPACE)
+
+
+@host_only
+def test_bridge_epilogue_argument_checks(L):
+    def b(x=FAKE, g=0, be=0, rows=4, D=64, eps=1e-5, nu=1.0, out=FAKE):
+        return L.cmc_bridge_epilogue(x, g, be, rows, D, eps, nu, out, None)
+    assert b(rows=0) == SHAPE
+    assert b(D=66) == SHAPE
+    assert b(D=16388) == SHAPE
+    assert b(eps=0.0) == RANGE
+    assert b(nu=-1.0) == RANGE
+    assert b(nu=float("inf")) == RANGE
+    assert b(x=0) == NULL
+    assert b(out=0) == NULL
+    assert b(x=FAKE + 4) == ALIGN
+    assert b(g=FAKE + 8) == ALIGN
