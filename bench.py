@@ -58,8 +58,8 @@ sys.path.insert(0, ROOT)
 import numpy as np  # noqa: E402
 import torch  # noqa: E402
 
-from workloads import (WORKLOADS, kv_inputs, question_inputs, selection_inputs,  # noqa: E402
-                       step_inputs)
+from workloads import (WORKLOADS, context_inputs, kv_inputs, question_inputs,  # noqa: E402
+                       selection_inputs, step_inputs)
 
 METRIC = ("two-tier decode-attn tokens/s and % of 8 TB/s HBM; CME top-k select µs")
 NOMINAL_HBM_GBS = 8000.0
@@ -516,7 +516,8 @@ def run_gpu(args, w, world, rank, local):
 
     # the question-side prologue per request (pool q_vec, score + select,
     # CME-guided window start), L2-cold like select_us
-    prologue_us = bridge_us = None
+    prologue_us = bridge_us = denoise_us = None
+    denoise_bytes = 0
     if not args.no_variant:
         qi = question_inputs(w, sel0, ratio=8 if w.N >= 16384 else 4)
         tok = torch.from_numpy(qi.tokens).to(dev)
@@ -556,6 +557,27 @@ def run_gpu(args, w, world, rank, local):
         stream.synchronize()
         bridge_us = 1000.0 * statistics.median(a.elapsed_time(b) for a, b in times) / R
         del g_br, scratch
+        # graph-based denoising of one context of |C| = N * r tokens (H = 1280,
+        # GPT2-Large's width; g = 3, tau = 0.05, keep-minimum 16)
+        ratio = 8 if w.N >= 16384 else 4
+        ci = context_inputs(w.with_(B=1), H=1280, ratio=ratio)
+        emb = torch.from_numpy(ci.emb).to(dev)
+        ws_d = torch.empty(cmc.lib().cmc_denoise_workspace_size(1, emb.shape[1]),
+                           dtype=torch.uint8, device=dev)
+        g_dn = capture_calls(lambda r: cmc.denoise(emb, workspace=ws_d))
+        with torch.cuda.stream(stream):
+            g_dn.replay()
+            times = []
+            for _ in range(5):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                g_dn.replay()
+                e1.record(stream)
+                times.append((e0, e1))
+        stream.synchronize()
+        denoise_us = 1000.0 * statistics.median(a.elapsed_time(b) for a, b in times) / R
+        denoise_bytes = emb.numel() * 4
+        del g_dn, emb
 
     # e2e through the Python API with pinned host buffers
     e2e = run_e2e(args, w, reqs, dev, stream, world) if not args.no_e2e else None
@@ -584,6 +606,8 @@ def run_gpu(args, w, world, rank, local):
         "bridge_epilogue_us": bridge_us,
         "bridge_epilogue_gbs": (8 * w.B * w.N * w.D / (bridge_us * 1e-6) / 1e9
                                 if bridge_us else None),
+        "denoise_us": denoise_us,
+        "denoise_gbs": denoise_bytes / (denoise_us * 1e-6) / 1e9 if denoise_us else None,
         "tier1_gather_us": gather_us,
         "tier1_gather_gbs": (tier1_gather_bytes(w.B, w.L, w.Hkv, w.d, w.k) / (gather_us * 1e-6)
                              / 1e9 if gather_us > 0 else None),

@@ -83,6 +83,39 @@ CMC_API const char* cmc_status_string(int status);
 CMC_API int cmc_last_cuda_error(void);
 
 /* ------------------------------------------------------------------------ *
+ * Graph-based context denoising (Section 2.1)                               *
+ * ------------------------------------------------------------------------ */
+
+/* Bytes of workspace cmc_denoise needs for B contexts of n_max tokens. */
+CMC_API size_t cmc_denoise_workspace_size(int B, int n_max);
+
+/*
+ * Keeps token i of context b when its cosine similarity to at least one of
+ * its g following tokens j = i+1 .. min(i+g, n-1) is at least tau (the last
+ * token has no follower and fails); the keep-minimum of the paper's
+ * threshold appendix then forces one kept token into every run of
+ * keep_every consecutive positions (walking left to right, a token is also
+ * kept when the previous kept token is keep_every positions back, or, before
+ * any, when it is token keep_every - 1; keep_every == 0 disables it).
+ * Cosines with a zero vector are 0; the comparison is taken in fp32.
+ *
+ *   emb         fp32 [B, n_max, H]  token embeddings of each context
+ *   n_tokens    int32 [B] tokens per context (clamped to [0, n_max]), or NULL
+ *   kept_idx    int32 [B, n_max] output: the kept positions in ascending
+ *               order, then -1
+ *   kept_count  int32 [B] output: how many were kept
+ *   workspace   >= cmc_denoise_workspace_size(B, n_max) bytes, any content;
+ *               on completion its first B * n_max bytes hold each token's
+ *               threshold-test result (1 passed, 0 not or past n_tokens)
+ *
+ * Limits: 1 <= B <= 65535, 1 <= n_max <= 2^24, 4 <= H <= 65536, H % 4 == 0,
+ * 1 <= g <= 8, keep_every >= 0, tau finite.
+ */
+CMC_API int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int H, int g,
+                        float tau, int keep_every, int32_t* kept_idx, int32_t* kept_count,
+                        void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------ *
  * MemoryBridge output (Section 2.2, the norm-calibrated tanh equation)       *
  * ------------------------------------------------------------------------ */
 

@@ -11,6 +11,10 @@ from .cmc_oracle import (
     cosine_scores,
     select_top_k,
     score_select,
+    denoise_pass,
+    keep_minimum,
+    denoise_keep,
+    denoise,
     bridge_epilogue,
     question_vector,
     tier2_start,
@@ -35,6 +39,10 @@ __all__ = [
     "cosine_scores",
     "select_top_k",
     "score_select",
+    "denoise_pass",
+    "keep_minimum",
+    "denoise_keep",
+    "denoise",
     "bridge_epilogue",
     "question_vector",
     "tier2_start",

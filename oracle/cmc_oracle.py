@@ -121,6 +121,70 @@ def score_select(question_emb: np.ndarray, cme_bank: np.ndarray, k: int
 
 
 # ----------------------------------------------------------------------------
+# Graph-based context denoising (Section 2.1)
+# ----------------------------------------------------------------------------
+
+def denoise_pass(emb: np.ndarray, n_tokens: int, g: int, tau: float) -> np.ndarray:
+    """The threshold test of the graph-based denoising (Section 2.1): token i
+    passes when its cosine similarity to at least one of its g following
+    tokens (j = i+1 .. min(i+g, n)) is at least tau; the last token has no
+    follower and fails.  Cosines of zero vectors are 0; the comparison with
+    tau is taken on the cosine rounded to float32 (the kernels' precision).
+    emb: [>= n_tokens, H].  Returns bool [n_tokens]."""
+    e = np.asarray(emb[:n_tokens], dtype=np.float64)
+    n = e.shape[0]
+    norms = np.sqrt(np.einsum("ij,ij->i", e, e))
+    passed = np.zeros(n, dtype=bool)
+    for i in range(n):
+        best = -np.inf
+        for j in range(i + 1, min(i + g, n - 1) + 1):
+            den = norms[i] * norms[j]
+            c = float(e[i] @ e[j]) / den if den > 0 else 0.0
+            best = max(best, c)
+        passed[i] = bool(np.float32(best) >= np.float32(tau))
+    return passed
+
+
+def keep_minimum(passed: np.ndarray, keep_every: int) -> np.ndarray:
+    """The keep-minimum constraint of the threshold appendix: one kept token
+    in every run of `keep_every` consecutive positions.  Walking left to
+    right, a token is also kept when the previous kept token lies
+    `keep_every` positions back (or, before any, when it is token
+    keep_every - 1); keep_every == 0 keeps just the passing tokens."""
+    keep = np.array(passed, dtype=bool)
+    last = -1
+    for i in range(keep.size):
+        if not keep[i] and keep_every > 0 and i - last >= keep_every:
+            keep[i] = True
+        if keep[i]:
+            last = i
+    return keep
+
+
+def denoise_keep(emb: np.ndarray, n_tokens: int, g: int, tau: float, keep_every: int
+                 ) -> np.ndarray:
+    """Which tokens of one context survive the denoising: the threshold test
+    followed by the keep-minimum.  Returns bool [n_tokens]."""
+    return keep_minimum(denoise_pass(emb, n_tokens, g, tau), keep_every)
+
+
+def denoise(emb: np.ndarray, n_tokens: np.ndarray, g: int, tau: float, keep_every: int
+            ) -> Tuple[np.ndarray, np.ndarray]:
+    """Denoised contexts as index lists: for each context b, the positions of
+    the kept tokens in ascending order (int64 [B, max_n], -1 past the count)
+    and the counts (int64 [B])."""
+    emb = np.asarray(emb)
+    B, n_max = emb.shape[0], emb.shape[1]
+    idx = np.full((B, n_max), -1, dtype=np.int64)
+    cnt = np.zeros(B, dtype=np.int64)
+    for b in range(B):
+        kept = np.flatnonzero(denoise_keep(emb[b], int(n_tokens[b]), g, tau, keep_every))
+        idx[b, :len(kept)] = kept
+        cnt[b] = len(kept)
+    return idx, cnt
+
+
+# ----------------------------------------------------------------------------
 # MemoryBridge output (Section 2.2, the norm-calibrated tanh equation)
 # ----------------------------------------------------------------------------
 

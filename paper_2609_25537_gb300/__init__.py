@@ -15,6 +15,7 @@ from .cmc import (  # noqa: F401
     decode_attn_plan,
     decode_attn_workspace_size,
     decode_step,
+    denoise,
     dims_of,
     question_select,
     score_select,

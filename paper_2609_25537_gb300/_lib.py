@@ -17,6 +17,8 @@ LIB_PATH = os.path.join(PKG_DIR, "libcmc.so")
 EXPORTS = (
     "cmc_status_string",
     "cmc_last_cuda_error",
+    "cmc_denoise_workspace_size",
+    "cmc_denoise",
     "cmc_bridge_epilogue",
     "cmc_score_select_workspace_size",
     "cmc_score_select",
@@ -77,6 +79,8 @@ _dims_p = ctypes.POINTER(CmcDims)
 _SIGNATURES = {
     "cmc_status_string": (ctypes.c_char_p, [_i]),
     "cmc_last_cuda_error": (_i, []),
+    "cmc_denoise_workspace_size": (_sz, [_i, _i]),
+    "cmc_denoise": (_i, [_vp, _vp, _i, _i, _i, _i, ctypes.c_float, _i, _vp, _vp, _vp, _sz, _vp]),
     "cmc_bridge_epilogue": (_i, [_vp, _vp, _vp, ctypes.c_int64, _i, ctypes.c_float,
                                  ctypes.c_float, _vp, _vp]),
     "cmc_score_select_workspace_size": (_sz, [_i, _i]),

@@ -32,6 +32,7 @@ from ._lib import CmcDims, check, lib, DEVFLAG_BAD_INDEX, DEVFLAG_BAD_POS, DEVFL
 __all__ = [
     "CmcDims",
     "DecodeWorkspace",
+    "denoise",
     "bridge_epilogue",
     "score_select",
     "score_select_workspace_size",
@@ -70,6 +71,35 @@ def _need(t: torch.Tensor, name: str, dtype: torch.dtype, ndim: int, device=None
         raise ValueError(f"{name} must be contiguous")
     if device is not None and t.device != device:
         raise ValueError(f"{name} is on {t.device}, expected {device}")
+
+
+# ----------------------------------------------------------------------------
+# Graph-based context denoising
+# ----------------------------------------------------------------------------
+
+def denoise(emb: torch.Tensor, *, n_tokens: Optional[torch.Tensor] = None, g: int = 3,
+            tau: float = 0.05, keep_every: int = 16,
+            workspace: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """Positions of the tokens kept by the graph-based denoising, int32
+    [B, n_max] ascending then -1, and their counts int32 [B]; see
+    cmc_denoise.  Defaults: the paper's g = 3, tau = 0.05, keep-minimum 16."""
+    _need(emb, "emb", torch.float32, 3)
+    dev = emb.device
+    B, n_max, H = emb.shape
+    if n_tokens is not None:
+        _need(n_tokens, "n_tokens", torch.int32, 1, dev)
+        if int(n_tokens.shape[0]) != B:
+            raise ValueError("n_tokens must be [B]")
+    kept = torch.empty((B, n_max), dtype=torch.int32, device=dev)
+    count = torch.empty(B, dtype=torch.int32, device=dev)
+    need = int(lib().cmc_denoise_workspace_size(B, n_max))
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+    st = lib().cmc_denoise(_p(emb), _p(n_tokens), B, n_max, H, g, float(tau), keep_every,
+                           _p(kept), _p(count), _p(workspace),
+                           workspace.numel() * workspace.element_size(), _stream(dev))
+    check(st, "cmc_denoise")
+    return kept, count
 
 
 # ----------------------------------------------------------------------------

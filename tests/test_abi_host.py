@@ -251,3 +251,26 @@ def test_bridge_epilogue_argument_checks(L):
     assert b(out=0) == NULL
     assert b(x=FAKE + 4) == ALIGN
     assert b(g=FAKE + 8) == ALIGN
+
+
+def test_denoise_workspace_size(L):
+    assert L.cmc_denoise_workspace_size(2, 1000) == 2048
+    assert L.cmc_denoise_workspace_size(0, 10) == 0
+
+
+@host_only
+def test_denoise_argument_checks(L):
+    def d(emb=FAKE, nt=0, B=2, n=100, H=64, g=3, tau=0.05, every=16, idx=FAKE, cnt=FAKE,
+          ws=FAKE, wsb=1 << 20):
+        return L.cmc_denoise(emb, nt, B, n, H, g, tau, every, idx, cnt, ws, wsb, None)
+    assert d(H=66) == SHAPE
+    assert d(n=0) == SHAPE
+    assert d(g=0) == RANGE
+    assert d(g=9) == RANGE
+    assert d(every=-1) == RANGE
+    assert d(tau=float("nan")) == RANGE
+    assert d(emb=0) == NULL
+    assert d(idx=0) == NULL
+    assert d(emb=FAKE + 4) == ALIGN
+    assert d(cnt=FAKE + 2) == ALIGN
+    assert d(wsb=100) == WORKSPACE

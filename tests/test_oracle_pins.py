@@ -614,3 +614,65 @@ def test_bridge_epilogue_against_torch_and_the_norm_bound():
     np.testing.assert_allclose(small, nu * np.tanh(F.layer_norm(
         torch.from_numpy(x), (D,), torch.from_numpy(gamma * 0.01),
         torch.from_numpy(beta * 0.01), eps=1e-5).numpy()), rtol=1e-12, atol=1e-15)
+
+
+# ----------------------------------------------------------------------------
+# Graph-based context denoising (Section 2.1; keep-minimum from the appendix)
+# ----------------------------------------------------------------------------
+
+def test_denoise_closed_forms():
+    u, v = np.array([1.0, 0.0, 0.0]), np.array([0.0, 1.0, 0.0])
+    w = np.array([1.0, 1.0, 0.0])               # cos(u, w) = cos(v, w) = 1/sqrt(2)
+    e = np.stack([u, u, v, w, v, u, v])
+    # g = 1: cos to the next token: 1, 0, .707, .707, 0, 0, (none)
+    keep = oracle.denoise_keep(e, 7, 1, 0.5, 0)
+    assert keep.tolist() == [True, False, True, True, False, False, False]
+    # g = 2: token 1 sees v (0) and w (.707); token 4 sees u, v (0, 1); token 5 sees v (0)
+    keep = oracle.denoise_keep(e, 7, 2, 0.5, 0)
+    assert keep.tolist() == [True, True, True, True, True, False, False]
+    # a zero vector has cosine 0 with everything
+    e0 = np.stack([u, np.zeros(3), u])
+    assert oracle.denoise_keep(e0, 3, 1, 0.0, 0).tolist() == [True, True, False]
+    assert oracle.denoise_keep(e0, 3, 1, 0.1, 0).tolist() == [False, False, False]
+
+
+def test_denoise_thresholds_at_the_extremes():
+    rng = np.random.default_rng(12)
+    e = rng.standard_normal((100, 8))
+    # tau = -1: every token with a follower passes; the last has none
+    keep = oracle.denoise_keep(e, 100, 3, -1.0, 16)
+    assert keep.sum() == 99 and not keep[-1]
+    # tau > 1: nothing passes; the keep-minimum alone keeps 15, 31, 47, ...
+    keep = oracle.denoise_keep(e, 100, 3, 1.5, 16)
+    assert np.flatnonzero(keep).tolist() == [15, 31, 47, 63, 79, 95]
+
+
+def test_denoise_against_an_independent_formulation():
+    """Threshold test from torch's pairwise cosines over shifted copies; the
+    keep-minimum from its closed form: a token that fails the test is kept
+    exactly when its distance to the last token that passed it (or to
+    position -1) is a multiple of keep_every."""
+    rng = np.random.default_rng(13)
+    n, H, g, tau, every = 700, 16, 3, 0.35, 16
+    steps = rng.standard_normal((n, H)) * 0.6
+    steps[rng.random(n) < 0.3] *= 6.0              # isolated tokens
+    e = np.cumsum(steps, axis=0)                    # neighbours correlate
+    et = torch.from_numpy(e)
+    best = torch.full((n,), -math.inf, dtype=torch.float64)
+    for s in range(1, g + 1):
+        c = F.cosine_similarity(et[:-s], et[s:], dim=1, eps=0.0)
+        best[:-s] = torch.maximum(best[:-s], c)
+    passed = (best >= tau).numpy()
+    last, want = -1, np.zeros(n, dtype=bool)
+    for i in range(n):
+        want[i] = passed[i] or (i - last) % every == 0
+        if passed[i]:
+            last = i
+    got = oracle.denoise_keep(e, n, g, tau, every)
+    np.testing.assert_array_equal(got, want)
+    kept = np.flatnonzero(got)
+    assert np.all(np.diff(np.concatenate([[-1], kept])) <= every)   # no gap above 16
+    assert 0 < kept.size < n
+    idx, cnt = oracle.denoise(e[None], np.array([n]), g, tau, every)
+    assert cnt[0] == kept.size and idx[0, :kept.size].tolist() == kept.tolist()
+    assert np.all(idx[0, kept.size:] == -1)

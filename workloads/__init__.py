@@ -9,10 +9,12 @@ from .configs import Workload, WORKLOADS, ablation_workloads, get_workload
 from .generate import (
     SelectionInputs,
     QuestionInputs,
+    ContextInputs,
     KVInputs,
     StepInputs,
     selection_inputs,
     question_inputs,
+    context_inputs,
     kv_inputs,
     step_inputs,
     random_tier1_indices,
@@ -27,10 +29,12 @@ __all__ = [
     "get_workload",
     "SelectionInputs",
     "QuestionInputs",
+    "ContextInputs",
     "KVInputs",
     "StepInputs",
     "selection_inputs",
     "question_inputs",
+    "context_inputs",
     "kv_inputs",
     "step_inputs",
     "random_tier1_indices",

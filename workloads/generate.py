@@ -47,6 +47,8 @@ _TAGS = {
     "step_v": 11,
     "idx": 12,
     "question_tokens": 13,
+    "context_vocab": 14,
+    "context_ids": 15,
 }
 
 
@@ -197,6 +199,36 @@ def question_inputs(w: Workload, si: SelectionInputs, Lq: int = 24, chunk: int =
     return QuestionInputs(tokens=tokens, q_len=q_len,
                           chunk_offset=np.tile(offs, (nb, 1)),
                           ctx_len=np.full(nb, w.N * ratio, dtype=np.int32))
+
+
+@dataclass
+class ContextInputs:
+    emb: np.ndarray       # float32 [B, n, H]: input embeddings of the context tokens
+    n_tokens: np.ndarray  # int32 [B]: tokens per context (rows past it are padding)
+
+
+def context_inputs(w: Workload, H: int = 1280, ratio: int = 4, vocab: int = 4096,
+                   batch: Optional[range] = None) -> ContextInputs:
+    """Context token embeddings for the denoising filter: |C| = N * ratio
+    tokens per context (the last context of a batch is 3/4 as long), each the
+    embedding of a token id drawn with Zipf-like frequencies (p ~ 1/rank)
+    from a vocabulary of independent Gaussian vectors, so that distinct
+    tokens are nearly orthogonal and repeats of frequent tokens are close."""
+    seqs = range(w.B) if batch is None else batch
+    nb = len(seqs)
+    n = w.N * ratio
+    table = (_rng(w.seed, "context_vocab").standard_normal((vocab, H)) / np.sqrt(H)
+             ).astype(np.float32)
+    p = 1.0 / np.arange(1, vocab + 1)
+    p /= p.sum()
+    emb = np.zeros((nb, n, H), dtype=np.float32)
+    n_tok = np.empty(nb, dtype=np.int32)
+    for i, b in enumerate(seqs):
+        nt = n if b + 1 < w.B or w.B == 1 else (3 * n) // 4
+        ids = _rng(w.seed, "context_ids", b).choice(vocab, size=nt, p=p)
+        emb[i, :nt] = table[ids]
+        n_tok[i] = nt
+    return ContextInputs(emb=emb, n_tokens=n_tok)
 
 
 # ----------------------------------------------------------------------------
