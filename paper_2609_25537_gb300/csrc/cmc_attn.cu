@@ -97,6 +97,7 @@ struct AttnParams {
   long long rem;
   float scale_log2;       // softmax scale * log2(e)
   long long rope_offset;  // rotary embedding (GQA-layer step): position of ring token 0
+  int l2_prefetch;        // box tiles per CTA prefetched into L2 before the grid dependency wait
   double rope_inv_freq[64];  // theta^(-2i/d) for the d/2 pairs, computed on the host
 };
 
@@ -199,6 +200,19 @@ __device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_
           dst),
       "l"(src), "r"(bytes), "r"(smem_addr(bar))
       : "memory");
+}
+
+// L2 prefetch of one TMA box and of a contiguous byte range.  These are hints:
+// no data reaches the issuing thread and the L2 stays coherent with the
+// previous kernel's writes, so they may be issued before the grid dependency
+// wait.
+__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap* map, int col, int row) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];\n" ::"l"(map),
+               "r"(col), "r"(row)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(src), "r"(bytes) : "memory");
 }
 
 // Named barrier over the consumer warps only (the producer warp never joins).
@@ -438,6 +452,31 @@ __device__ __forceinline__ void issue_box_loads(const AttnParams& p, const AttnM
   bulk_copy(smem_addr(aux + S::kQ), qsrc, G * D * 2, full);
 }
 
+// Producer lane 0, before the grid dependency wait: the boxes of a box tile
+// (and, for the first tile of a unit, the unit's query rows) prefetched into
+// L2.  A CTA that becomes resident while the previous kernel on the stream is
+// still running (a free slot, or one that kernel's exiting CTAs freed) thus
+// pulls its first tile from HBM during that kernel's tail; its loads after
+// the wait then hit L2.
+template <int D, int G>
+__device__ __forceinline__ void prefetch_box_tile(const AttnParams& p, const AttnMaps& maps,
+                                                  const TileCursor& c, bool with_q) {
+  constexpr int H = D / 64;
+  const bool t1 = c.lt < p.t1_tiles;
+  const int row = t1 ? c.u * p.N + c.lt * kTileKeys : c.u * p.W + (c.lt - p.t1_tiles) * kTileKeys;
+  const CUtensorMap* mk = t1 ? &maps.t1k_box : &maps.rk_box;
+  const CUtensorMap* mv = t1 ? &maps.t1v_box : &maps.rv_box;
+#pragma unroll
+  for (int h = 0; h < H; ++h) {
+    tma_prefetch_l2(mk, h * 64, row);
+    tma_prefetch_l2(mv, h * 64, row);
+  }
+  if (with_q)
+    bulk_prefetch_l2(p.q + ((static_cast<long long>(c.b) * p.L + c.l) * p.Hq +
+                            static_cast<long long>(c.g) * G) * D,
+                     G * D * 2);
+}
+
 // Producer warp, once pos (and, for a gathered tile, its idx entries) is
 // known: the tile's header (rows that may hold keys, rows with a bad index,
 // the new token's row), the new token's K/V rows in the fused step, the loads
@@ -569,6 +608,21 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
   __syncthreads();
+  if (warp == kWarps && lane == 0 && p.l2_prefetch > 0) {
+    asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.rk_box) : "memory");
+    asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.rv_box) : "memory");
+    if (p.idx == nullptr && p.k > 0) {
+      asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.t1k_box) : "memory");
+      asm volatile("prefetch.tensormap [%0];\n" ::"l"(&maps.t1v_box) : "memory");
+    }
+    TileCursor cp;
+    cp.init(t_begin, p);
+    const int npf = n_tiles < p.l2_prefetch ? n_tiles : p.l2_prefetch;
+    for (int i = 0; i < npf; ++i) {
+      if (!gathered_tile(p, cp)) prefetch_box_tile<D, G>(p, maps, cp, i == 0 || cp.j == 0);
+      cp.next(p);
+    }
+  }
   // Programmatic dependent launch: everything above overlapped the previous
   // kernel; inputs may be that kernel's outputs, so wait for it here.  Then let
   // the combine kernel that follows launch early.
@@ -1099,6 +1153,10 @@ static bool encode_rows(CUtensorMap* map, const void* base, long long rows, int 
 // Pipeline depth: stages of 64 keys per CTA.  Three stages keep a CTA at
 // ~110 KB of shared memory at d = 128, G <= 4, so two CTAs share an SM.
 constexpr int kStages = 3;
+// Box tiles per CTA prefetched into L2 before the grid dependency wait.  One
+// tile hides most of the HBM latency at the start of a launch; deeper
+// prefetch competes with the running kernel's stream and measured slower.
+constexpr int kL2PrefetchTiles = 1;
 
 // Launch plan of one attention call on the current device.
 struct AttnPlan {
@@ -1263,6 +1321,7 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   const float sc = scale > 0.f ? scale : 1.0f / sqrtf(static_cast<float>(m.d));
   p.scale_log2 = sc * 1.4426950408889634f;
   p.rope_offset = rope ? rope_offset : 0;
+  p.l2_prefetch = kL2PrefetchTiles;
   for (int i = 0; i < 64; ++i)
     p.rope_inv_freq[i] = (rope && i < m.d / 2) ? pow(rope_theta, -2.0 * i / m.d) : 0.0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
