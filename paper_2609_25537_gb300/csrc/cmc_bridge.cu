@@ -8,9 +8,17 @@
 // are plain library GEMMs and stay with the caller; this is the row-wise
 // epilogue that turns their output into the bank the Tier-1 scoring reads.
 //
-// One CTA per row (grid-stride): the row is streamed once into shared memory
-// with 16-byte loads, the three row reductions (sum, squared deviations,
-// squared norm of nu tanh) meet in a fixed tree, and the row is written once.
+// Rows of up to 4,096 features stay in registers (bridge_epilogue_reg_kernel,
+// below).  Longer rows: a CTA walks its rows (grid-stride) through three
+// shared-memory row buffers: while it reduces and writes row r, rows r + grid and r + 2 grid are
+// already on their way (16-byte cp.async copies), so each SM overlaps the HBM
+// reads of later rows with the arithmetic and the writes of the current one.
+// The three row reductions (sum, squared deviations, squared norm of
+// nu tanh) meet in a fixed tree; each thread touches only its own float4s of
+// the row, so the buffers need a barrier only when a buffer is refilled.
+// tanh(z) is evaluated as 1 - 2 / (1 + e^{2z}) with the hardware base-2
+// exponential (ex2.approx, relative error ~2^-22) and a fast division:
+// absolute error below 1e-6, saturating correctly to +-1.
 // HBM-bound: 8 * H_d bytes per row.
 #include <cuda_runtime.h>
 #include <math.h>
@@ -21,7 +29,9 @@
 namespace cmc {
 
 constexpr int kBridgeThreads = 256;
-constexpr int kBridgeMaxD = 16384;  // 64 KB of shared memory per row
+constexpr int kBridgeMaxD = 16384;  // 64 KB of shared memory per row buffer
+constexpr int kBridgeBufs = 3;      // the row being processed + two in flight
+constexpr int kBridgeCtasPerSm = 2;
 
 // Block-wide sum in a fixed order (warp shuffles, then the warps in order);
 // every thread receives the total.  `red` holds kBridgeThreads / 32 + 1 floats.
@@ -43,11 +53,30 @@ __device__ __forceinline__ float bridge_block_sum(float v, float* red) {
   return total;
 }
 
-__global__ void __launch_bounds__(kBridgeThreads)
-bridge_epilogue_kernel(const float* __restrict__ x, const float* __restrict__ gamma,
+// tanh(z) = 1 - 2 / (1 + 2^(2 z log2 e)).
+__device__ __forceinline__ float tanh_ex2(float z) {
+  float e;
+  asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(e) : "f"(z * 2.8853900817779268f));
+  return 1.f - __fdividef(2.f, 1.f + e);
+}
+
+__device__ __forceinline__ void br_cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(
+                   static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void br_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void br_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+__global__ void __launch_bounds__(kBridgeThreads, kBridgeCtasPerSm)
+bridge_epilogue_kernel(const float* x, const float* __restrict__ gamma,
                        const float* __restrict__ beta, long long rows, int D, float eps, float nu,
                        float* out) {
-  extern __shared__ float4 srow[];  // the row being processed, D / 4 vectors
+  extern __shared__ float4 sbuf[];  // kBridgeBufs row buffers of D / 4 vectors
   __shared__ float red[kBridgeThreads / 32 + 1];
   pdl_wait();
   pdl_trigger();
@@ -55,28 +84,35 @@ bridge_epilogue_kernel(const float* __restrict__ x, const float* __restrict__ ga
   const int D4 = D >> 2;
   const float4* g4 = reinterpret_cast<const float4*>(gamma);
   const float4* b4 = reinterpret_cast<const float4*>(beta);
-  for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
-    const float4* xr = reinterpret_cast<const float4*>(x + r * D);
+  const long long step = gridDim.x;
+  auto load = [&](long long r, int buf) {
+    const float4* src = reinterpret_cast<const float4*>(x + r * D);
+    float4* dst = sbuf + static_cast<long long>(buf) * D4;
+    for (int i = tid; i < D4; i += kBridgeThreads) br_cp_async16(dst + i, src + i);
+  };
+  // prologue: the first kBridgeBufs - 1 rows of this CTA (one group each)
+#pragma unroll
+  for (int k = 0; k < kBridgeBufs - 1; ++k) {
+    const long long r = blockIdx.x + k * step;
+    if (r < rows) load(r, k);
+    br_commit();
+  }
+  int k = 0;
+  for (long long r = blockIdx.x; r < rows; r += step, ++k) {
+    const long long ra = r + (kBridgeBufs - 1) * step;  // row whose load starts now
+    if (ra < rows) load(ra, (k + kBridgeBufs - 1) % kBridgeBufs);
+    br_commit();
+    br_wait<kBridgeBufs - 1>();  // this thread's copies of row r have landed
+    float4* row = sbuf + static_cast<long long>(k % kBridgeBufs) * D4;
     float s = 0.f;
-    // four 16-byte loads per thread in flight before any is used
-    for (int base = 0; base < D4; base += 4 * kBridgeThreads) {
-      float4 v[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int i = base + u * kBridgeThreads + tid;
-        v[u] = i < D4 ? ld_stream_f4(xr + i) : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int i = base + u * kBridgeThreads + tid;
-        if (i < D4) srow[i] = v[u];
-        s += (v[u].x + v[u].y) + (v[u].z + v[u].w);
-      }
+    for (int i = tid; i < D4; i += kBridgeThreads) {
+      const float4 v = row[i];
+      s += (v.x + v.y) + (v.z + v.w);
     }
     const float mean = bridge_block_sum(s, red) / static_cast<float>(D);
     float q = 0.f;
     for (int i = tid; i < D4; i += kBridgeThreads) {
-      const float4 v = srow[i];
+      const float4 v = row[i];
       const float a = v.x - mean, b = v.y - mean, c = v.z - mean, d = v.w - mean;
       q += (a * a + b * b) + (c * c + d * d);
     }
@@ -84,25 +120,113 @@ bridge_epilogue_kernel(const float* __restrict__ x, const float* __restrict__ ga
     const float rstd = 1.0f / sqrtf(var + eps);
     float n2 = 0.f;
     for (int i = tid; i < D4; i += kBridgeThreads) {
-      const float4 v = srow[i];
+      const float4 v = row[i];
       const float4 g = gamma ? __ldg(g4 + i) : make_float4(1.f, 1.f, 1.f, 1.f);
       const float4 b = beta ? __ldg(b4 + i) : make_float4(0.f, 0.f, 0.f, 0.f);
       float4 t;
-      t.x = nu * tanhf(fmaf(g.x, (v.x - mean) * rstd, b.x));
-      t.y = nu * tanhf(fmaf(g.y, (v.y - mean) * rstd, b.y));
-      t.z = nu * tanhf(fmaf(g.z, (v.z - mean) * rstd, b.z));
-      t.w = nu * tanhf(fmaf(g.w, (v.w - mean) * rstd, b.w));
-      srow[i] = t;
+      t.x = nu * tanh_ex2(fmaf(g.x, (v.x - mean) * rstd, b.x));
+      t.y = nu * tanh_ex2(fmaf(g.y, (v.y - mean) * rstd, b.y));
+      t.z = nu * tanh_ex2(fmaf(g.z, (v.z - mean) * rstd, b.z));
+      t.w = nu * tanh_ex2(fmaf(g.w, (v.w - mean) * rstd, b.w));
+      row[i] = t;
       n2 += (t.x * t.x + t.y * t.y) + (t.z * t.z + t.w * t.w);
     }
     const float norm = sqrtf(bridge_block_sum(n2, red));
     const float f = (norm > 2.f * nu) ? (2.f * nu) / norm : 1.f;
     float4* orow = reinterpret_cast<float4*>(out + r * D);
     for (int i = tid; i < D4; i += kBridgeThreads) {
-      const float4 t = srow[i];
+      const float4 t = row[i];
       orow[i] = make_float4(t.x * f, t.y * f, t.z * f, t.w * f);
     }
-    __syncthreads();  // srow is refilled by the next row
+    __syncthreads();  // this buffer is refilled at the next iteration
+  }
+  br_wait<0>();
+}
+
+// Rows of at most 4,096 features: a thread keeps its V float4s of the row in
+// registers and loads its share of the next row of the CTA (grid-stride)
+// before it works on the current one, so no shared-memory staging and no
+// refill barrier; each of the three reductions takes one barrier (its own
+// partials array, summed by every thread in the same order).
+constexpr int kBridgeRegMaxV = 4;  // float4s per thread: D <= 4 * 4 * kBridgeThreads
+constexpr int kBridgeRegCtasPerSm = 3;
+
+template <int V>
+__global__ void __launch_bounds__(kBridgeThreads, kBridgeRegCtasPerSm)
+bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
+                           const float* __restrict__ beta, long long rows, int D, float eps,
+                           float nu, float* out) {
+  constexpr int NW = kBridgeThreads / 32;
+  __shared__ float red[3][NW];
+  pdl_wait();
+  pdl_trigger();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int D4 = D >> 2;
+  const float4* g4 = reinterpret_cast<const float4*>(gamma);
+  const float4* b4 = reinterpret_cast<const float4*>(beta);
+  const long long step = gridDim.x;
+  auto block_sum = [&](float v, float* part) {
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == 0) part[warp] = v;
+    __syncthreads();
+    float t = part[0];
+#pragma unroll
+    for (int w = 1; w < NW; ++w) t += part[w];
+    return t;
+  };
+  auto load = [&](long long r, float4 (&v)[V]) {
+    const float4* src = reinterpret_cast<const float4*>(x + r * D);
+#pragma unroll
+    for (int e = 0; e < V; ++e) {
+      const int i = tid + e * kBridgeThreads;
+      v[e] = i < D4 ? __ldcs(src + i) : make_float4(0.f, 0.f, 0.f, 0.f);  // coherent: x may be out
+    }
+  };
+  float4 cur[V], nxt[V];
+  long long r = blockIdx.x;
+  if (r < rows) load(r, cur);
+  for (; r < rows; r += step) {
+    if (r + step < rows) load(r + step, nxt);
+    float s = 0.f;
+#pragma unroll
+    for (int e = 0; e < V; ++e) s += (cur[e].x + cur[e].y) + (cur[e].z + cur[e].w);
+    const float mean = block_sum(s, red[0]) / static_cast<float>(D);
+    float q = 0.f;
+#pragma unroll
+    for (int e = 0; e < V; ++e) {
+      if (tid + e * kBridgeThreads < D4) {
+        const float a = cur[e].x - mean, b = cur[e].y - mean, c = cur[e].z - mean, d = cur[e].w - mean;
+        q += (a * a + b * b) + (c * c + d * d);
+      }
+    }
+    const float var = block_sum(q, red[1]) / static_cast<float>(D);
+    const float rstd = 1.0f / sqrtf(var + eps);
+    float n2 = 0.f;
+#pragma unroll
+    for (int e = 0; e < V; ++e) {
+      const int i = tid + e * kBridgeThreads;
+      if (i < D4) {
+        const float4 g = gamma ? __ldg(g4 + i) : make_float4(1.f, 1.f, 1.f, 1.f);
+        const float4 b = beta ? __ldg(b4 + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+        float4& t = cur[e];
+        t.x = nu * tanh_ex2(fmaf(g.x, (t.x - mean) * rstd, b.x));
+        t.y = nu * tanh_ex2(fmaf(g.y, (t.y - mean) * rstd, b.y));
+        t.z = nu * tanh_ex2(fmaf(g.z, (t.z - mean) * rstd, b.z));
+        t.w = nu * tanh_ex2(fmaf(g.w, (t.w - mean) * rstd, b.w));
+        n2 += (t.x * t.x + t.y * t.y) + (t.z * t.z + t.w * t.w);
+      }
+    }
+    const float norm = sqrtf(block_sum(n2, red[2]));
+    const float f = (norm > 2.f * nu) ? (2.f * nu) / norm : 1.f;
+    float4* orow = reinterpret_cast<float4*>(out + r * D);
+#pragma unroll
+    for (int e = 0; e < V; ++e) {
+      const int i = tid + e * kBridgeThreads;
+      if (i < D4) orow[i] = make_float4(cur[e].x * f, cur[e].y * f, cur[e].z * f, cur[e].w * f);
+    }
+#pragma unroll
+    for (int e = 0; e < V; ++e) cur[e] = nxt[e];
   }
 }
 
@@ -118,7 +242,22 @@ int cmc_bridge_epilogue(const float* x, const float* gamma, const float* beta, i
   if (!x || !out) return CMC_ERR_NULL;
   if (!aligned16(x) || !aligned16(out) || (gamma && !aligned16(gamma)) || (beta && !aligned16(beta)))
     return CMC_ERR_ALIGN;
-  const size_t smem = static_cast<size_t>(D) * sizeof(float);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int D4 = D / 4;
+  if (D4 <= kBridgeRegMaxV * kBridgeThreads) {
+    long long grid = rows;
+    const long long cap = static_cast<long long>(sm_count()) * kBridgeRegCtasPerSm;
+    if (grid > cap) grid = cap;
+    const dim3 gd(static_cast<unsigned>(grid)), bd(kBridgeThreads);
+    const long long R = static_cast<long long>(rows);
+    switch ((D4 + kBridgeThreads - 1) / kBridgeThreads) {
+      case 1: return launch_pdl(bridge_epilogue_reg_kernel<1>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      case 2: return launch_pdl(bridge_epilogue_reg_kernel<2>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      case 3: return launch_pdl(bridge_epilogue_reg_kernel<3>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      default: return launch_pdl(bridge_epilogue_reg_kernel<4>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+    }
+  }
+  const size_t smem = static_cast<size_t>(kBridgeBufs) * D * sizeof(float);
   static bool attr_set[64] = {false};
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
@@ -126,16 +265,18 @@ int cmc_bridge_epilogue(const float* x, const float* gamma, const float* beta, i
   if (dev >= 0 && dev < 64 && !attr_set[dev]) {
     st = record_cuda_error(cudaFuncSetAttribute(bridge_epilogue_kernel,
                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                static_cast<int>(kBridgeMaxD * sizeof(float))));
+                                                static_cast<int>(kBridgeBufs * kBridgeMaxD * sizeof(float))));
     if (st != CMC_OK) return st;
     attr_set[dev] = true;
   }
+  // Persistent CTAs, kBridgeCtasPerSm per SM (one when the row buffers leave
+  // room for only one): each walks about rows / grid rows.
+  const int per_sm = D * 4 * kBridgeBufs * kBridgeCtasPerSm <= 200 * 1024 ? kBridgeCtasPerSm : 1;
   long long grid = rows;
-  const long long cap = static_cast<long long>(sm_count()) * (2048 / kBridgeThreads);
+  const long long cap = static_cast<long long>(sm_count()) * per_sm;
   if (grid > cap) grid = cap;
   return launch_pdl(bridge_epilogue_kernel, dim3(static_cast<unsigned>(grid)), dim3(kBridgeThreads),
-                    smem, static_cast<cudaStream_t>(stream), x, gamma, beta,
-                    static_cast<long long>(rows), D, eps, nu, out);
+                    smem, s, x, gamma, beta, static_cast<long long>(rows), D, eps, nu, out);
 }
 
 }  // extern "C"

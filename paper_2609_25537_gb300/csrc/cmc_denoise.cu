@@ -4,19 +4,31 @@
 // threshold forces one kept token into every run of `keep_every` positions.
 //
 // Two kernels:
-//  1. denoise_pass_kernel -- one warp per token: the token's row and the rows
-//     of its g followers are read with 16-byte loads through L1 (each row is
-//     read from HBM once; the CTA's warps take consecutive tokens, so its
-//     re-reads as a follower mostly hit L1 or L2),
-//     the norms and dot products reduced in a fixed order, and the pass flag
-//     (max cosine >= tau, decided in fp32) written as one byte.
+//  1. denoise_pass_kernel -- a CTA takes a tile of 32 consecutive tokens of
+//     one context.  Their rows and the rows of the g tokens that follow the
+//     tile (together one contiguous span of the [n, H] matrix) are streamed
+//     through shared memory in chunks of 128 features (512 bytes per row),
+//     four stages of 16-byte cp.async copies; rows past the context's tokens
+//     are zero-filled, never read.  Each warp owns four tokens: per chunk a
+//     lane takes one float4 of each of the warp's rows and accumulates the
+//     squared norms and the dot products of every token with its g
+//     followers; lanes are reduced once per tile (fixed order), and lane 0
+//     writes the four pass flags (max cosine >= tau, decided in fp32).  Every
+//     row crosses from HBM once (the g halo rows are the next tile's first
+//     rows, read by the neighbouring CTA at about the same time).  The
+//     tile's 32 pass bits also go to a word of the workspace, and the tile's
+//     positions of kept_idx are set to -1 (the compaction overwrites the
+//     kept ones).
 //  2. denoise_compact_kernel -- one CTA per context.  Walking left to right,
 //     the keep-minimum forces token i exactly when it fails the test and its
 //     distance to the last token that passed (or to position -1) is a
-//     multiple of keep_every, so the walk is data-parallel: a block-wide
-//     prefix maximum gives every thread's chunk the last passing position
-//     before it, and a block-wide prefix sum places the kept positions, which
-//     are written in ascending order.
+//     multiple of keep_every, so the walk is data-parallel.  A thread takes
+//     four 32-token pass words (one 16-byte load) per segment of 131,072
+//     tokens (the next segment's words are loaded ahead); a block-wide prefix
+//     maximum gives it the last passing position before its words, from
+//     which the forced positions of each gap follow with one division; a
+//     block-wide prefix sum places its kept positions; both carry from one
+//     segment to the next.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -27,149 +39,314 @@ namespace cmc {
 
 constexpr int kDenoiseMaxG = 8;
 constexpr int kPassThreads = 256;
+constexpr int kPassTokPerWarp = 4;
+constexpr int kPassTile = kPassTokPerWarp * (kPassThreads / 32);  // 32 tokens per tile
+constexpr int kPassChunk = 128;                                   // features per stage
+constexpr int kPassStageRows = kPassTile + kDenoiseMaxG;          // 40
+constexpr int kPassStageBytes = kPassStageRows * kPassChunk * 4;  // 20 KB
+constexpr int kPassStages = 4;
+constexpr int kPassSmem = kPassStages * kPassStageBytes;          // 80 KB
 constexpr int kCompactThreads = 1024;
+constexpr int kCompactWords = 4;  // pass words (32 tokens each) per compaction thread
 
-__global__ void __launch_bounds__(kPassThreads)
-denoise_pass_kernel(const float* __restrict__ emb, const int32_t* __restrict__ n_tokens, int B,
-                    int n_max, int H, int g, float tau, uint8_t* __restrict__ pass) {
+__device__ __forceinline__ void dn_cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void dn_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void dn_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ float dot4(const float4& a, const float4& b) {
+  return (a.x * b.x + a.y * b.y) + (a.z * b.z + a.w * b.w);
+}
+
+template <int G>
+__global__ void __launch_bounds__(kPassThreads, 2)
+denoise_pass_kernel(const float* __restrict__ emb, const int32_t* __restrict__ n_tokens, int n_max,
+                    int H, float tau, uint8_t* __restrict__ pass, uint32_t* __restrict__ masks,
+                    int32_t* __restrict__ kept_idx, long long tiles, int tiles_per_ctx,
+                    int words_stride) {
+  constexpr int TPW = kPassTokPerWarp;
+  constexpr int SROWS = kPassTile + G;                                // rows staged per chunk
+  constexpr int NCP = (SROWS * 32 + kPassThreads - 1) / kPassThreads;  // copies per thread
+  constexpr int kLast = kPassThreads / 32 - 1;                        // warp that owns the halo norms
+  extern __shared__ __align__(16) float4 dn_stage[];
+  __shared__ float nrm_s[kPassTile + kDenoiseMaxG];  // squared norms of the staged rows
+  __shared__ uint32_t nib[kPassThreads / 32];         // each warp's four pass bits
   pdl_wait();
   pdl_trigger();
-  const int lane = threadIdx.x & 31;
-  const long long warp0 = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const long long nwarps = (static_cast<long long>(gridDim.x) * blockDim.x) >> 5;
-  const long long total = static_cast<long long>(B) * n_max;
-  const int H4 = H >> 2;
-  for (long long t = warp0; t < total; t += nwarps) {
-    const int b = static_cast<int>(t / n_max);
-    const int i = static_cast<int>(t - static_cast<long long>(b) * n_max);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nchunks = (H + kPassChunk - 1) / kPassChunk;
+  const uint32_t sbase = static_cast<uint32_t>(__cvta_generic_to_shared(dn_stage));
+  const int r0 = warp * TPW;  // this warp's first token row in the tile
+  for (long long tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+    const int b = static_cast<int>(tile / tiles_per_ctx);
+    const int i0 = static_cast<int>(tile - static_cast<long long>(b) * tiles_per_ctx) * kPassTile;
     int n = n_tokens ? n_tokens[b] : n_max;
     n = n < 0 ? 0 : (n > n_max ? n_max : n);
-    if (i >= n) {
-      if (lane == 0) pass[t] = 0;
+    uint8_t* pb = pass + static_cast<long long>(b) * n_max;
+    // the compaction overwrites the kept positions; everything else stays -1
+    if (tid < kPassTile && i0 + tid < n_max) kept_idx[static_cast<long long>(b) * n_max + i0 + tid] = -1;
+    if (i0 >= n) {  // a tile past the context's tokens: flags 0
+      if (tid < kPassTile && i0 + tid < n_max) pb[i0 + tid] = 0;
+      if (tid == 0) masks[static_cast<long long>(b) * words_stride + i0 / kPassTile] = 0u;
       continue;
     }
-    const int gg = min(g, n - 1 - i);  // followers that exist
-    const float4* ei = reinterpret_cast<const float4*>(emb + t * H);
-    float ni = 0.f, dot[kDenoiseMaxG], nj[kDenoiseMaxG];
+    const int rows = min(SROWS, n - i0);  // staged rows that hold tokens
+    const float* src0 = emb + (static_cast<long long>(b) * n_max + i0) * H;
+    // this thread's copies: 16-byte piece x = tid + m * kPassThreads of a
+    // chunk, row x / 32, column 4 (x % 32) of the chunk
+    const float* src[NCP];
+    bool live[NCP];
 #pragma unroll
-    for (int s = 0; s < kDenoiseMaxG; ++s) dot[s] = nj[s] = 0.f;
-    // The CTA's warps take consecutive tokens, so a row read here (through
-    // L1) is mostly the follower row of the warps just before: each row
-    // crosses from L2 about once.
-#pragma unroll 2
-    for (int c = lane; c < H4; c += 32) {
-      const float4 a = __ldg(ei + c);
-      ni += (a.x * a.x + a.y * a.y) + (a.z * a.z + a.w * a.w);
+    for (int m = 0; m < NCP; ++m) {
+      const int x = tid + m * kPassThreads;
+      live[m] = x < SROWS * 32 && (x >> 5) < rows;
+      src[m] = src0 + static_cast<long long>(x >> 5) * H + 4 * (x & 31);
+    }
+    auto issue = [&](int c) {
+      const uint32_t dst0 = sbase + (c % kPassStages) * kPassStageBytes;
+      const int col0 = c * kPassChunk;
 #pragma unroll
-      for (int s = 0; s < kDenoiseMaxG; ++s) {
-        if (s < gg) {
-          const float4 v = __ldg(ei + static_cast<long long>(s + 1) * H4 + c);
-          dot[s] += (a.x * v.x + a.y * v.y) + (a.z * v.z + a.w * v.w);
-          nj[s] += (v.x * v.x + v.y * v.y) + (v.z * v.z + v.w * v.w);
+      for (int m = 0; m < NCP; ++m) {
+        const int x = tid + m * kPassThreads;
+        if (x < SROWS * 32) {
+          const bool ok = live[m] && col0 + 4 * (x & 31) < H;
+          dn_cp_async16(dst0 + x * 16, ok ? src[m] + col0 : src0, ok ? 16u : 0u);
         }
       }
+    };
+#pragma unroll
+    for (int c = 0; c < kPassStages - 1; ++c) {
+      if (c < nchunks) issue(c);
+      dn_commit();
     }
+    float nrm[TPW + G], dt[TPW][G];
+#pragma unroll
+    for (int j = 0; j < TPW + G; ++j) nrm[j] = 0.f;
+#pragma unroll
+    for (int t = 0; t < TPW; ++t)
+#pragma unroll
+      for (int s = 0; s < G; ++s) dt[t][s] = 0.f;
+    for (int c = 0; c < nchunks; ++c) {
+      dn_wait<kPassStages - 2>();  // chunk c has landed (this thread's copies)
+      __syncthreads();             // ... everyone's; and chunk c-1's stage is free
+      if (c + kPassStages - 1 < nchunks) issue(c + kPassStages - 1);
+      dn_commit();
+      const float4* st = dn_stage + (c % kPassStages) * (kPassStageBytes / 16) + r0 * 32 + lane;
+      float4 x[TPW + G];
+#pragma unroll
+      for (int j = 0; j < TPW + G; ++j) x[j] = st[j * 32];
+#pragma unroll
+      for (int j = 0; j < TPW; ++j) nrm[j] += dot4(x[j], x[j]);
+      if (warp == kLast) {  // the g rows after the tile
+#pragma unroll
+        for (int j = TPW; j < TPW + G; ++j) nrm[j] += dot4(x[j], x[j]);
+      }
+#pragma unroll
+      for (int t = 0; t < TPW; ++t)
+#pragma unroll
+        for (int s = 0; s < G; ++s) dt[t][s] += dot4(x[t], x[t + 1 + s]);
+    }
+    dn_wait<0>();
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) {
-      ni += __shfl_xor_sync(0xffffffffu, ni, off);
 #pragma unroll
-      for (int s = 0; s < kDenoiseMaxG; ++s) {
-        dot[s] += __shfl_xor_sync(0xffffffffu, dot[s], off);
-        nj[s] += __shfl_xor_sync(0xffffffffu, nj[s], off);
-      }
+      for (int j = 0; j < TPW + G; ++j)
+        if (j < TPW || warp == kLast) nrm[j] += __shfl_xor_sync(0xffffffffu, nrm[j], off);
+#pragma unroll
+      for (int t = 0; t < TPW; ++t)
+#pragma unroll
+        for (int s = 0; s < G; ++s) dt[t][s] += __shfl_xor_sync(0xffffffffu, dt[t][s], off);
     }
     if (lane == 0) {
-      bool ok = false;
 #pragma unroll
-      for (int s = 0; s < kDenoiseMaxG; ++s) {
-        if (s < gg) {
-          const float c = (ni > 0.f && nj[s] > 0.f) ? dot[s] / (sqrtf(ni) * sqrtf(nj[s])) : 0.f;
-          ok = ok || c >= tau;
+      for (int j = 0; j < TPW + G; ++j)
+        if (j < TPW || warp == kLast) nrm_s[r0 + j] = nrm[j];
+    }
+    __syncthreads();  // the norms are shared; the stages are refilled by the next tile
+    if (lane == 0) {
+      uint32_t bits = 0;
+#pragma unroll
+      for (int t = 0; t < TPW; ++t) {
+        const int i = i0 + r0 + t;
+        if (i >= n_max) break;
+        bool ok = false;
+        if (i < n) {
+          const int gg = min(G, n - 1 - i);  // followers that exist
+#pragma unroll
+          for (int s = 0; s < G; ++s) {
+            if (s < gg) {
+              const float ni = nrm[t], nj = nrm_s[r0 + t + 1 + s];
+              const float c = (ni > 0.f && nj > 0.f) ? dt[t][s] / (sqrtf(ni) * sqrtf(nj)) : 0.f;
+              ok = ok || c >= tau;
+            }
+          }
         }
+        pb[i] = ok ? 1 : 0;
+        bits |= ok ? (1u << t) : 0u;
       }
-      pass[t] = ok ? 1 : 0;
+      nib[warp] = bits;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t word = 0;
+#pragma unroll
+      for (int w = 0; w < kPassThreads / 32; ++w) word |= nib[w] << (w * TPW);
+      masks[static_cast<long long>(b) * words_stride + i0 / kPassTile] = word;
     }
   }
 }
 
+// Block-wide exclusive scans over kCompactThreads = 32 warps (identity -1
+// for the maximum, 0 for the sum): a warp scan, then every warp scans the 32
+// warp totals.  `red` holds one int per warp.  Every thread gets the value
+// over the threads before it and the block total.
+static_assert(kCompactThreads == 1024, "the scans take one warp total per lane");
+__device__ __forceinline__ int block_excl_max(int v, int* red, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, v, off);
+    if (lane >= off) v = max(v, u);
+  }
+  int ex = __shfl_up_sync(0xffffffffu, v, 1);
+  if (lane == 0) ex = -1;
+  if (lane == 31) red[warp] = v;
+  __syncthreads();
+  int wv = red[lane];
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, wv, off);
+    if (lane >= off) wv = max(wv, u);
+  }
+  const int before = __shfl_sync(0xffffffffu, wv, (warp + 31) & 31);
+  *total = __shfl_sync(0xffffffffu, wv, 31);
+  __syncthreads();
+  return warp > 0 ? max(before, ex) : ex;
+}
+__device__ __forceinline__ int block_excl_sum(int v, int* red, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int mine = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, v, off);
+    if (lane >= off) v += u;
+  }
+  if (lane == 31) red[warp] = v;
+  __syncthreads();
+  int wv = red[lane];
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, wv, off);
+    if (lane >= off) wv += u;
+  }
+  const int before = __shfl_sync(0xffffffffu, wv, (warp + 31) & 31);
+  *total = __shfl_sync(0xffffffffu, wv, 31);
+  __syncthreads();
+  return (warp > 0 ? before : 0) + v - mine;
+}
+
+// Kept tokens among the 32 tokens i0 .. i0+31 whose pass bits are `m`, given
+// lp, the last passing position before i0 (-1: none): the passing tokens,
+// and in every gap between a passing token (or lp) and the next one, the
+// positions at multiples of K after it.  One division per gap.
+__device__ __forceinline__ uint32_t keep_mask(uint32_t m, int lp, int i0, int K) {
+  uint32_t kept = m;
+  if (K <= 0) return kept;
+  int prev = lp, pos = i0;
+  uint32_t rest = m;
+  while (true) {
+    const int nxt = rest ? i0 + __ffs(rest) - 1 : i0 + 32;  // next passing token, or the end
+    for (int f = prev + K * ((pos - prev + K - 1) / K); f < nxt; f += K) kept |= 1u << (f - i0);
+    if (!rest) break;
+    prev = nxt;
+    pos = nxt + 1;
+    rest &= rest - 1;
+  }
+  return kept;
+}
+
 __global__ void __launch_bounds__(kCompactThreads)
-denoise_compact_kernel(const uint8_t* __restrict__ pass, const int32_t* __restrict__ n_tokens,
-                       int n_max, int keep_every, int32_t* __restrict__ kept_idx,
-                       int32_t* __restrict__ kept_count) {
-  __shared__ int wred[kCompactThreads / 32];
-  __shared__ int wtot;
+denoise_compact_kernel(const uint32_t* __restrict__ masks, const int32_t* __restrict__ n_tokens,
+                       int n_max, int words_stride, int keep_every,
+                       int32_t* __restrict__ kept_idx, int32_t* __restrict__ kept_count) {
+  constexpr int WPT = kCompactWords;  // pass words per thread and segment
+  __shared__ int red[kCompactThreads / 32];
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.x;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x;
   int n = n_tokens ? n_tokens[b] : n_max;
   n = n < 0 ? 0 : (n > n_max ? n_max : n);
-  const uint8_t* pb = pass + static_cast<long long>(b) * n_max;
+  const uint4* mb = reinterpret_cast<const uint4*>(masks + static_cast<long long>(b) * words_stride);
   int32_t* out = kept_idx + static_cast<long long>(b) * n_max;
-  const int C = (n + kCompactThreads - 1) / kCompactThreads;  // tokens per thread
-  const int t0 = tid * C;
-  const int t1 = min(t0 + C, n);
-
-  // last passing position in this thread's chunk, then the prefix maximum
-  // over the threads before it (-1: none)
-  int last = -1;
-  for (int i = t0; i < t1; ++i)
-    if (pb[i]) last = i;
-  int incl = last;
+  const int nq = (n + 32 * WPT - 1) / (32 * WPT);  // uint4s of words that hold tokens
+  int carry_last = -1;                              // last passing position before the segment
+  int carry_cnt = 0;                                // tokens kept before the segment
+  uint4 next = tid < nq ? mb[tid] : make_uint4(0u, 0u, 0u, 0u);
+  for (int q0 = 0; q0 < nq; q0 += kCompactThreads) {
+    const int qi = q0 + tid;
+    const uint4 raw = next;
+    if (qi + kCompactThreads < nq) next = mb[qi + kCompactThreads];  // the next segment's words
+    const uint32_t wr[WPT] = {raw.x, raw.y, raw.z, raw.w};
+    const int t0 = 32 * WPT * qi;  // first token of this thread's words
+    uint32_t m[WPT];
+    int last = -1;
 #pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const int v = __shfl_up_sync(0xffffffffu, incl, off);
-    if (lane >= off) incl = max(incl, v);
-  }
-  if (lane == 31) wred[warp] = incl;
-  __syncthreads();
-  int carry = -1;  // last passing position before this thread's chunk
-  for (int w = 0; w < warp; ++w) carry = max(carry, wred[w]);
-  const int prev_lane = __shfl_up_sync(0xffffffffu, incl, 1);
-  if (lane > 0) carry = max(carry, prev_lane);
-  __syncthreads();  // wred is reused below
-
-  // kept tokens of the chunk: passed, or forced by the keep-minimum
-  auto kept = [&](int i, int lastp) {
-    return pb[i] != 0 || (keep_every > 0 && (i - lastp) % keep_every == 0);
-  };
-  int cnt = 0;
-  int lp = carry;
-  for (int i = t0; i < t1; ++i) {
-    if (kept(i, lp)) ++cnt;
-    if (pb[i]) lp = i;
-  }
-  // exclusive prefix sum of the counts
-  int inc = cnt;
+    for (int j = 0; j < WPT; ++j) {
+      const int nv = min(max(n - (t0 + 32 * j), 0), 32);  // tokens of word j that exist
+      m[j] = wr[j] & (nv >= 32 ? ~0u : ((1u << nv) - 1u));
+      if (m[j]) last = t0 + 32 * j + 31 - __clz(m[j]);
+    }
+    int seg_last, seg_cnt;
+    int lp = max(block_excl_max(last, red, &seg_last), carry_last);
+    uint32_t kept[WPT];
+    int cnt = 0;
 #pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const int v = __shfl_up_sync(0xffffffffu, inc, off);
-    if (lane >= off) inc += v;
+    for (int j = 0; j < WPT; ++j) {
+      const int i0 = t0 + 32 * j;
+      const int nv = min(max(n - i0, 0), 32);
+      kept[j] = nv > 0 ? keep_mask(m[j], lp, i0, keep_every) & (nv >= 32 ? ~0u : ((1u << nv) - 1u)) : 0u;
+      cnt += __popc(kept[j]);
+      if (m[j]) lp = i0 + 31 - __clz(m[j]);
+    }
+    int slot = carry_cnt + block_excl_sum(cnt, red, &seg_cnt);
+#pragma unroll
+    for (int j = 0; j < WPT; ++j) {
+      uint32_t k = kept[j];
+      while (k) {
+        out[slot++] = t0 + 32 * j + __ffs(k) - 1;
+        k &= k - 1;
+      }
+    }
+    carry_last = max(carry_last, seg_last);
+    carry_cnt += seg_cnt;
   }
-  if (lane == 31) wred[warp] = inc;
-  __syncthreads();
-  int before = 0;
-  for (int w = 0; w < warp; ++w) before += wred[w];
-  if (tid == kCompactThreads - 1) wtot = before + inc;
-  int slot = before + inc - cnt;
-  lp = carry;
-  for (int i = t0; i < t1; ++i) {
-    if (kept(i, lp)) out[slot++] = i;
-    if (pb[i]) lp = i;
-  }
-  __syncthreads();
-  const int total = wtot;
-  for (int i = total + tid; i < n_max; i += kCompactThreads) out[i] = -1;
-  if (tid == 0) kept_count[b] = total;
+  if (tid == 0) kept_count[b] = carry_cnt;
 }
 
 }  // namespace cmc
 
 extern "C" {
 
+// [0, B * n_max): one pass byte per token; then, 256-byte aligned, one
+// 32-bit pass word per tile of 32 tokens, [B, words_stride] with the row
+// stride rounded up to whole 16-byte groups.
+static size_t dn_words_offset(int B, int n_max) {
+  return cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(n_max), 256);
+}
+static int dn_words_stride(int n_max) {
+  const int words = (n_max + 31) / 32;
+  return (words + cmc::kCompactWords - 1) / cmc::kCompactWords * cmc::kCompactWords;
+}
+
 size_t cmc_denoise_workspace_size(int B, int n_max) {
   if (B < 1 || n_max < 1) return 0;
-  return cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(n_max), 256);
+  const size_t words = static_cast<size_t>(B) * static_cast<size_t>(dn_words_stride(n_max));
+  return cmc::align_up(dn_words_offset(B, n_max) + 4 * words, 256);
 }
 
 int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int H, int g,
@@ -188,16 +365,44 @@ int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int
   if (static_cast<long long>(B) * n_max * H >= (1LL << 40)) return CMC_ERR_SHAPE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* pass = static_cast<uint8_t*>(workspace);
-  const long long warps = static_cast<long long>(B) * n_max;
-  long long blocks = (warps * 32 + kPassThreads - 1) / kPassThreads;
-  const long long cap = static_cast<long long>(sm_count()) * (2048 / kPassThreads) * 4;
+  uint32_t* masks = reinterpret_cast<uint32_t*>(pass + dn_words_offset(B, n_max));
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  int st = record_cuda_error(cudaGetDevice(&dev));
+  if (st != CMC_OK) return st;
+  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+    const void* kerns[8] = {
+        reinterpret_cast<const void*>(denoise_pass_kernel<1>), reinterpret_cast<const void*>(denoise_pass_kernel<2>),
+        reinterpret_cast<const void*>(denoise_pass_kernel<3>), reinterpret_cast<const void*>(denoise_pass_kernel<4>),
+        reinterpret_cast<const void*>(denoise_pass_kernel<5>), reinterpret_cast<const void*>(denoise_pass_kernel<6>),
+        reinterpret_cast<const void*>(denoise_pass_kernel<7>), reinterpret_cast<const void*>(denoise_pass_kernel<8>)};
+    for (const void* k : kerns) {
+      st = record_cuda_error(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kPassSmem));
+      if (st != CMC_OK) return st;
+    }
+    attr_set[dev] = true;
+  }
+  const int tiles_per_ctx = (n_max + kPassTile - 1) / kPassTile;
+  const long long tiles = static_cast<long long>(B) * tiles_per_ctx;
+  long long blocks = tiles;
+  const long long cap = static_cast<long long>(sm_count()) * 2 * 64;  // grid-stride beyond
   if (blocks > cap) blocks = cap;
-  int st = launch_pdl(denoise_pass_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kPassThreads),
-                      0, s, emb, n_tokens, B, n_max, H, g, tau, pass);
+  switch (g) {
+#define CMC_DN_CASE(GG)                                                                             \
+  case GG:                                                                                          \
+    st = launch_pdl(denoise_pass_kernel<GG>, dim3(static_cast<unsigned>(blocks)), dim3(kPassThreads), \
+                    static_cast<size_t>(kPassSmem), s, emb, n_tokens, n_max, H, tau, pass, masks,  \
+                    kept_idx, tiles, tiles_per_ctx, dn_words_stride(n_max));                        \
+    break;
+    CMC_DN_CASE(1) CMC_DN_CASE(2) CMC_DN_CASE(3) CMC_DN_CASE(4)
+    CMC_DN_CASE(5) CMC_DN_CASE(6) CMC_DN_CASE(7) CMC_DN_CASE(8)
+#undef CMC_DN_CASE
+    default: return CMC_ERR_RANGE;
+  }
   if (st != CMC_OK) return st;
   return launch_pdl(denoise_compact_kernel, dim3(B), dim3(kCompactThreads), 0, s,
-                    static_cast<const uint8_t*>(pass), n_tokens, n_max, keep_every, kept_idx,
-                    kept_count);
+                    static_cast<const uint32_t*>(masks), n_tokens, n_max, dn_words_stride(n_max), keep_every,
+                    kept_idx, kept_count);
 }
 
 }  // extern "C"

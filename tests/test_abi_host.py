@@ -254,7 +254,8 @@ def test_bridge_epilogue_argument_checks(L):
 
 
 def test_denoise_workspace_size(L):
-    assert L.cmc_denoise_workspace_size(2, 1000) == 2048
+    # 2,000 pass bytes (to 2,048), then 2 x 32 pass words of 4 bytes
+    assert L.cmc_denoise_workspace_size(2, 1000) == 2048 + 256
     assert L.cmc_denoise_workspace_size(0, 10) == 0
 
 
