@@ -121,16 +121,20 @@ def kernel_source_hash() -> str:
     return h.hexdigest()
 
 
-def profiled_traffic():
+def profiled_traffic(workload: str, tier1: str):
     """DRAM bytes per launch of the fused decode kernel from the committed ncu
-    summary, if it was taken on the current kernel source; else None."""
+    summary, if it was taken on the current kernel source, for this workload
+    and Tier-1 form; else None."""
     try:
         txt = open(PROFILE_FILE).read()
     except OSError:
         return None
     m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", txt)
     h = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", txt)
-    if not m or not h or h.group(1) != kernel_source_hash():
+    c = re.search(r"profiled_config:\s*(\S+)\s+(\S+)", txt)
+    if not m or not h or not c or h.group(1) != kernel_source_hash():
+        return None
+    if (c.group(1), c.group(2)) != (workload, tier1):
         return None
     return int(m.group(1))
 
@@ -565,6 +569,8 @@ def run_gpu(args, w, world, rank, local):
         # graph-based denoising of one context of |C| = N * r tokens (H = 1280,
         # GPT2-Large's width; g = 3, tau = 0.05, keep-minimum 16)
         ratio = 8 if w.N >= 16384 else 4
+        if args.denoise_tokens:
+            ratio = max(1, args.denoise_tokens // w.N)
         ci = context_inputs(w.with_(B=1), H=1280, ratio=ratio)
         emb = torch.from_numpy(ci.emb).to(dev)
         ws_d = torch.empty(cmc.lib().cmc_denoise_workspace_size(1, emb.shape[1]),
@@ -613,7 +619,7 @@ def run_gpu(args, w, world, rank, local):
                      "kernel": (f"fused decode step: two_tier_attn_kernel<{w.d},{w.Hq // w.Hkv},fused,3>"
                                 + (" (one CTA per unit, no combine launch)" if step_launches == 1
                                    else " + two_tier_combine_kernel")),
-                     "bytes_per_launch": nbytes, "traffic": profiled_traffic(),
+                     "bytes_per_launch": nbytes, "traffic": profiled_traffic(w.name, mode),
                      "flops_per_launch": decode_step_flops(w.B, w.L, w.Hq, w.d, w.k, w.W)},
         "select_roofline": {"bound": "hbm", "bytes": select_bytes(w.B, w.N, w.D, w.k),
                             "achieved": select_bytes(w.B, w.N, w.D, w.k) / (select_us * 1e-6)
@@ -750,6 +756,8 @@ def main(argv=None):
     ap.add_argument("--variant-replays", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--ref-step-seconds", type=float, default=2.0)
+    ap.add_argument("--denoise-tokens", type=int, default=0,
+                    help="tokens of the denoised context (default N x 4, N x 8 for N >= 16384)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         raise SystemExit("--warmup must be >= 3")
