@@ -38,6 +38,13 @@
 // through an "empty" mbarrier.  Every mbarrier wait has an iteration limit.
 // Warps are merged in shared memory at the end of a unit.
 //
+// K/V rows are read once per launch, so their loads carry an L2 evict-first
+// policy.  Before its grid dependency wait (programmatic dependent launch)
+// each CTA prefetches its first four box tiles into L2: CTAs that become
+// resident in free slots or in the slots of the previous launch's exiting
+// CTAs thus pull their first tiles from HBM while that launch drains, and the
+// evict-first stream of the running launch does not push them out again.
+//
 // The fused decode step also appends the new token: the producer copies the
 // new token's K/V rows next to the tile that holds its ring slot, a consumer
 // warp patches them over the stale ring row in shared memory and stores them
@@ -185,13 +192,20 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // --- TMA loads into shared memory, completing on an mbarrier.
-__device__ __forceinline__ void tma_box(uint32_t dst, const CUtensorMap* map, int col, int row,
-                                        uint64_t* bar) {
+// A 2-D TMA box load into shared memory, completing on an mbarrier, with an
+// L2 cache policy (createpolicy) attached.
+__device__ __forceinline__ void tma_box_hint(uint32_t dst, const CUtensorMap* map, int col, int row,
+                                             uint64_t* bar, uint64_t policy) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
-      "l"(map), "r"(col), "r"(row), "r"(smem_addr(bar))
+      "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;\n" ::"r"(dst),
+      "l"(map), "r"(col), "r"(row), "r"(smem_addr(bar)), "l"(policy)
       : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;\n" : "=l"(pol));
+  return pol;
 }
 __device__ __forceinline__ void bulk_copy(uint32_t dst, const void* src, uint32_t bytes,
                                           uint64_t* bar) {
@@ -319,6 +333,11 @@ struct MetaSlot {
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes));
 }
+__device__ __forceinline__ void cp_async16_hint(uint32_t dst, const void* src, uint32_t src_bytes,
+                                                uint64_t policy) {
+  asm volatile("cp.async.cg.shared.global.L2::cache_hint [%0], [%1], 16, %2, %3;\n" ::"r"(dst), "l"(src),
+               "r"(src_bytes), "l"(policy));
+}
 // Adds one pending arrival to `bar` now and completes it once every cp.async
 // this thread issued so far has landed.
 __device__ __forceinline__ void mbar_arrive_cp_async(uint64_t* bar) {
@@ -442,10 +461,13 @@ __device__ __forceinline__ void issue_box_loads(const AttnParams& p, const AttnM
   const uint32_t sK = smem_addr(stage + S::kK);
   const uint32_t sV = smem_addr(stage + S::kV);
   mbar_expect_tx(full, 2 * H * kHalfBytes + G * D * 2);
+  // K/V rows are read once per step: evict-first keeps them from displacing
+  // what is worth keeping in L2 (the prefetched first tiles of the next launch)
+  const uint64_t pol = policy_evict_first();
 #pragma unroll
   for (int h = 0; h < H; ++h) {
-    tma_box(sK + h * kHalfBytes, mk, h * 64, row, full);
-    tma_box(sV + h * kHalfBytes, mv, h * 64, row, full);
+    tma_box_hint(sK + h * kHalfBytes, mk, h * 64, row, full, pol);
+    tma_box_hint(sV + h * kHalfBytes, mv, h * 64, row, full, pol);
   }
   const uint16_t* qsrc =
       p.q + ((static_cast<long long>(c.b) * p.L + c.l) * p.Hq + static_cast<long long>(c.g) * G) * D;
@@ -517,6 +539,7 @@ __device__ __forceinline__ void finish_tile(const AttnParams& p, uint8_t* stage,
     const int chunk = lane % LPR;
     const int rsub = lane / LPR;
     const long long ubase = static_cast<long long>(c.u) * p.N * D + chunk * 8;
+    const uint64_t pol = policy_evict_first();
 #pragma unroll 8
     for (int jj = 0; jj < kTileKeys / RPP; ++jj) {
       const int r = jj * RPP + rsub;
@@ -524,8 +547,8 @@ __device__ __forceinline__ void finish_tile(const AttnParams& p, uint8_t* stage,
       const bool ok = r < n_rows && static_cast<unsigned>(row) < static_cast<unsigned>(p.N);
       const long long e = ubase + static_cast<long long>(ok ? row : 0) * D;
       const uint32_t off = swz(r, chunk);
-      cp_async16(sK + off, p.t1k + e, ok ? 16u : 0u);
-      cp_async16(sV + off, p.t1v + e, ok ? 16u : 0u);
+      cp_async16_hint(sK + off, p.t1k + e, ok ? 16u : 0u, pol);
+      cp_async16_hint(sV + off, p.t1v + e, ok ? 16u : 0u, pol);
     }
     mbar_arrive_cp_async(full);
     bad_lo = __ballot_sync(0xffffffffu, lane < n_rows && static_cast<unsigned>(meta.idx_lo) >= static_cast<unsigned>(p.N));
@@ -1153,10 +1176,12 @@ static bool encode_rows(CUtensorMap* map, const void* base, long long rows, int 
 // Pipeline depth: stages of 64 keys per CTA.  Three stages keep a CTA at
 // ~110 KB of shared memory at d = 128, G <= 4, so two CTAs share an SM.
 constexpr int kStages = 3;
-// Box tiles per CTA prefetched into L2 before the grid dependency wait.  One
-// tile hides most of the HBM latency at the start of a launch; deeper
-// prefetch competes with the running kernel's stream and measured slower.
-constexpr int kL2PrefetchTiles = 1;
+// Box tiles per CTA prefetched into L2 before the grid dependency wait.  With
+// the streamed K/V loads marked evict-first, four tiles (128 KB per CTA, half
+// of them in free slots while the previous launch runs, the rest in its tail)
+// measured best at the model shapes; without the evict-first policy one tile
+// was best and deeper prefetch slower.
+constexpr int kL2PrefetchTiles = 4;
 
 // Launch plan of one attention call on the current device.
 struct AttnPlan {
