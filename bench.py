@@ -483,9 +483,17 @@ def run_gpu(args, w, world, rank, local):
 
     launches_dec = K * R * T
     # kernels per fused decode call (attention, plus combine if units are split)
-    step_launches = cmc.decode_attn_plan(
+    step_ctas, step_launches = cmc.decode_attn_plan(
         cmc.dims_of(reqs[0].out, reqs[0].t1k_dense if mode == "dense" else reqs[0].t1k,
-                    None if mode == "dense" else reqs[0].idx, reqs[0].ring_k), fused=True)[1]
+                    None if mode == "dense" else reqs[0].idx, reqs[0].ring_k), fused=True)
+    n_units = w.B * w.L * w.Hkv
+    if step_launches > 1:
+        plan_txt = " + two_tier_combine_kernel (units split between CTAs)"
+    elif step_ctas > n_units:
+        plan_txt = (f" (clusters of {step_ctas // n_units} CTAs per unit, merged in distributed "
+                    "shared memory; one launch)")
+    else:
+        plan_txt = " (one CTA per unit; one launch)"
     launch_us = 1000.0 * sum(dec_ms) / launches_dec
     nbytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W, gather=mode == "gather")
     achieved = nbytes / (launch_us * 1e-6) / 1e9
@@ -617,8 +625,7 @@ def run_gpu(args, w, world, rank, local):
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
                      "kernel": (f"fused decode step: two_tier_attn_kernel<{w.d},{w.Hq // w.Hkv},fused,3>"
-                                + (" (one CTA per unit, no combine launch)" if step_launches == 1
-                                   else " + two_tier_combine_kernel")),
+                                + plan_txt),
                      "bytes_per_launch": nbytes, "traffic": profiled_traffic(w.name, mode),
                      "flops_per_launch": decode_step_flops(w.B, w.L, w.Hq, w.d, w.k, w.W)},
         "select_roofline": {"bound": "hbm", "bytes": select_bytes(w.B, w.N, w.D, w.k),

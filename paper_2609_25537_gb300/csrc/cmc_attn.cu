@@ -4,16 +4,18 @@
 //
 // Work decomposition.  A unit is one (sequence b, layer l, KV head g).  Its
 // keys are cut into tiles of 64: ceil(k / 64) Tier-1 tiles, then ceil(W / 64)
-// tiles of ring slots; no tile mixes the two tiers.  The flattened list of
-// (unit, tile) pairs is split into equal contiguous ranges, one per CTA.  When
-// the units fit in one wave of resident CTAs the grid is a whole number of
-// CTAs per unit -- one per unit at the model shapes, so no unit is split and
-// every CTA streams the same bytes; otherwise it is one wave of resident CTAs
-// (stream-K).  A CTA accumulates across the tiles of a unit and writes the
-// bf16 output of every unit it covers whole; for a unit cut between CTAs each
-// CTA writes an fp32 (max, sum, output) partial record, and a small combine
-// kernel that follows on the stream merges the records with a log-sum-exp
-// rescale.  No CTA ever waits on another.
+// tiles of ring slots; no tile mixes the two tiers.  With m = resident CTAs
+// per unit (at most one per tile): m = 1 (the Llama- and Mistral-shaped
+// steps) gives one CTA per unit, nothing split; 2 <= m <= 8 (long units, few
+// of them) gives thread-block clusters of m CTAs per unit, each CTA taking a
+// contiguous share of the unit's tiles: at the end every CTA leaves its fp32
+// (max, sum, output) record in its own shared memory, and after a cluster
+// barrier each CTA merges a slice of the output columns from all m records
+// (distributed shared memory, log-sum-exp rescale); m > 8, or more units
+// than resident CTAs, splits the flattened (unit, tile) list into equal
+// contiguous ranges (stream-K), partial records go to global memory, and a
+// small combine kernel that follows on the stream merges them.  No CTA ever
+// waits on another outside its cluster's two barriers.
 //
 // Inside a CTA one producer warp streams the tiles through a ring of shared-
 // memory stages.  Ring tiles, and Tier-1 tiles when the Tier-1 rows are the
@@ -102,6 +104,8 @@ struct AttnParams {
   int rot;                // in-unit processing order: tile (j + rot) % tpu at position j
   long long base;         // tiles per CTA (CTAs below `rem` take one more)
   long long rem;
+  int cm;                 // > 0: clusters of cm CTAs share each unit (CTA j of the cluster
+                          // takes positions [j tpu / cm, (j+1) tpu / cm)); 0: flat split
   float scale_log2;       // softmax scale * log2(e)
   long long rope_offset;  // rotary embedding (GQA-layer step): position of ring token 0
   int l2_prefetch;        // box tiles per CTA prefetched into L2 before the grid dependency wait
@@ -232,6 +236,36 @@ __device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes
 // Named barrier over the consumer warps only (the producer warp never joins).
 __device__ __forceinline__ void consumer_sync() {
   asm volatile("bar.sync 1, %0;\n" ::"n"(kWarps * 32) : "memory");
+}
+
+// --- thread-block cluster: barrier (every thread of every CTA of the
+// cluster arrives, then waits) and loads from a peer CTA's shared memory.
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release;\n" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire;\n" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t peer_smem(uint32_t local_addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(local_addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_peer_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];\n" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ float4 ld_peer_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];\n"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
 }
 
 // ---------------------------------------------------------------------------
@@ -619,8 +653,16 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
   const int warp = tid >> 5;
 
   const long long cta = blockIdx.x;
-  const long long t_begin = cta_first_tile(cta, p.base, p.rem);
-  const long long t_end = t_begin + p.base + (cta < p.rem ? 1 : 0);
+  long long t_begin, t_end;
+  if (p.cm > 0) {  // clusters of cm CTAs per unit
+    const long long u = cta / p.cm;
+    const int j = static_cast<int>(cta - u * p.cm);
+    t_begin = u * p.tpu + (static_cast<long long>(j) * p.tpu) / p.cm;
+    t_end = u * p.tpu + (static_cast<long long>(j + 1) * p.tpu) / p.cm;
+  } else {
+    t_begin = cta_first_tile(cta, p.base, p.rem);
+    t_end = t_begin + p.base + (cta < p.rem ? 1 : 0);
+  }
   const int n_tiles = static_cast<int>(t_end - t_begin);
 
   if (tid == 0) {
@@ -727,6 +769,13 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     cp_async_wait<0>();
     // Let this CTA's loads land before the warp exits (bounded).
     if (issued > 0) mbar_wait(&full_bar[(issued - 1) % NST], static_cast<uint32_t>(((issued - 1) / NST) & 1));
+    // A cluster plan: the consumers of every CTA of the cluster pass two
+    // cluster barriers at the end of their (one) unit; this warp passes the
+    // same two, so every thread of the cluster arrives at each.
+    if (p.cm > 0) {
+      cluster_sync_all();
+      cluster_sync_all();
+    }
     return;
   }
 
@@ -949,7 +998,15 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
       const bool whole = ut0 >= t_begin && ut0 + p.tpu <= t_end;
       const long long out_base =
           ((static_cast<long long>(cc.b) * p.L + cc.l) * p.Hq + static_cast<long long>(cc.g) * G) * D;
-      for (int x = tid; x < G * D / 4; x += kThreads) {
+      constexpr int NGR = G * D / 4;                      // 4-column groups of the unit's output
+      constexpr int XPT = (NGR + kThreads - 1) / kThreads;  // groups per thread
+      const bool clus = !whole && p.cm > 0;
+      float4 cacc[XPT];
+      float cls[XPT];
+#pragma unroll
+      for (int xi = 0; xi < XPT; ++xi) {
+        const int x = tid + xi * kThreads;
+        if (x >= NGR) break;
         const int hh = (4 * x) / D;
         const int c = (4 * x) % D;
         float4 acc = *reinterpret_cast<const float4*>(merge_o + hh * D + c);
@@ -964,6 +1021,9 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
           const float inv = Ls > 0.f ? __frcp_rn(Ls) : 0.f;
           *reinterpret_cast<uint2*>(p.out + out_base + hh * D + c) =
               make_uint2(pack_bf16_rn(acc.x * inv, acc.y * inv), pack_bf16_rn(acc.z * inv, acc.w * inv));
+        } else if (clus) {  // merged across the cluster below
+          cacc[xi] = acc;
+          cls[xi] = Ls;
         } else {  // merged by two_tier_combine_kernel
           constexpr int PW = rec_floats(G, D);
           float* rec = p.partials + (ut0 + (ut0 > t_begin ? 0 : t_begin - ut0)) * PW;
@@ -976,6 +1036,61 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
           }
           *reinterpret_cast<float4*>(rec + rec_out_offset(G) + hh * D + c) = acc;
         }
+      }
+      if (clus) {
+        // Each CTA of the cluster holds one share of the unit.  Its (max, sum,
+        // output) record goes to its own shared memory (over the merge
+        // buffer, now read); after a cluster barrier every CTA merges a slice
+        // of the output columns from all the records (log-sum-exp rescale, in
+        // rank order) and writes them; a second barrier keeps each record
+        // alive until every peer has read it.
+        float* rec = merge_o;
+        consumer_sync();
+#pragma unroll
+        for (int xi = 0; xi < XPT; ++xi) {
+          const int x = tid + xi * kThreads;
+          if (x >= NGR) break;
+          const int hh = (4 * x) / D;
+          const int c = (4 * x) % D;
+          if (c == 0) {
+            float M = merge_m[hh];
+#pragma unroll
+            for (int w = 1; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + hh]);
+            rec[hh] = M;
+            rec[G + hh] = cls[xi];
+          }
+          *reinterpret_cast<float4*>(rec + rec_out_offset(G) + hh * D + c) = cacc[xi];
+        }
+        cluster_sync_all();
+        const int cm = p.cm;
+        const int rank = static_cast<int>(cluster_ctarank());
+        const int x0 = (rank * NGR) / cm, x1 = ((rank + 1) * NGR) / cm;
+        const uint32_t rec_local = smem_addr(rec);
+        for (int x = x0 + tid; x < x1; x += kThreads) {
+          const int hh = (4 * x) / D;
+          const int c = (4 * x) % D;
+          float M = -INFINITY;
+          for (int r = 0; r < cm; ++r)
+            M = fmaxf(M, ld_peer_f32(peer_smem(rec_local + hh * 4, r)));
+          float Ls = 0.f;
+          float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (M != -INFINITY) {
+            for (int r = 0; r < cm; ++r) {
+              const uint32_t base = peer_smem(rec_local, r);
+              const float f = ex2(ld_peer_f32(base + hh * 4) - M);
+              const float4 o4 = ld_peer_f4(base + (rec_out_offset(G) + hh * D + c) * 4);
+              Ls = fmaf(f, ld_peer_f32(base + (G + hh) * 4), Ls);
+              O.x = fmaf(f, o4.x, O.x);
+              O.y = fmaf(f, o4.y, O.y);
+              O.z = fmaf(f, o4.z, O.z);
+              O.w = fmaf(f, o4.w, O.w);
+            }
+          }
+          const float inv = Ls > 0.f ? __frcp_rn(Ls) : 0.f;
+          *reinterpret_cast<uint2*>(p.out + out_base + hh * D + c) =
+              make_uint2(pack_bf16_rn(O.x * inv, O.y * inv), pack_bf16_rn(O.z * inv, O.w * inv));
+        }
+        cluster_sync_all();
       }
       if (i + 1 < n_tiles) consumer_sync();  // merge buffers are reused by the next unit
     }
@@ -1185,9 +1300,13 @@ constexpr int kL2PrefetchTiles = 4;
 
 // Launch plan of one attention call on the current device.
 struct AttnPlan {
-  long long ctas, base, rem;  // grid size; tiles per CTA (the first `rem` CTAs take one more)
-  bool split;                 // some unit is cut between CTAs: the combine kernel runs
+  long long ctas, base, rem;  // grid size; flat split: tiles per CTA (the first `rem` take one more)
+  int cm;                     // > 0: clusters of cm CTAs per unit (DSMEM merge, no combine)
+  bool split;                 // flat split cuts some unit: the combine kernel runs
 };
+
+// Largest cluster of CTAs that share one unit (the portable cluster size).
+constexpr int kMaxClusterCtas = 8;
 
 template <int D, int G, bool FUSED, bool ROPE>
 static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
@@ -1207,39 +1326,76 @@ static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
     if (per_sm < 1) per_sm = 1;
     if (dev >= 0 && dev < 64) configured[dev] = per_sm;
   }
-  // Grid: with no more units than resident CTAs, a whole number of CTAs per
-  // unit (one per unit when they fit: no unit is split and no combine kernel
-  // runs); otherwise one wave of resident CTAs, each taking an equal share of
-  // the flattened tiles.
+  // Grid.  With no more units than resident CTAs: m = resident CTAs per unit
+  // (at most one per tile).  m = 1: one CTA per unit, nothing is split.
+  // 2 <= m <= 8: clusters of m CTAs per unit, merged in distributed shared
+  // memory.  m > 8 (few, long units): a flat split of m CTAs per unit merged
+  // by the combine kernel.  More units than resident CTAs: one wave of CTAs,
+  // each taking an equal share of the flattened tiles (combine kernel).
   const long long slots = static_cast<long long>(per_sm) * sm_count();
   const long long units = total_tiles / tpu;
-  long long ctas = units <= slots ? units * (slots / units) : slots;
+  pl->cm = 0;
+  long long ctas;
+  if (units <= slots) {
+    long long m = slots / units;
+    if (m > tpu) m = tpu;
+    if (m >= 2 && m <= kMaxClusterCtas) pl->cm = static_cast<int>(m);
+    ctas = units * m;
+  } else {
+    ctas = slots;
+  }
   if (ctas > total_tiles) ctas = total_tiles;
   if (ctas < 1) ctas = 1;
   pl->ctas = ctas;
   pl->base = total_tiles / ctas;
   pl->rem = total_tiles % ctas;
-  // Is any unit split between CTAs (a CTA boundary inside a unit)?
+  // Flat split: is any unit cut between CTAs (a CTA boundary inside a unit)?
   pl->split = false;
-  for (long long c = 1; c < ctas && !pl->split; ++c) {
+  for (long long c = 1; pl->cm == 0 && c < ctas && !pl->split; ++c) {
     const long long t = c * pl->base + (c < pl->rem ? c : pl->rem);
     pl->split = (t % tpu) != 0;
   }
   return CMC_OK;
 }
 
+// Launches the attention kernel with programmatic stream serialization and,
+// for a cluster plan, the cluster dimension.
+template <int D, int G, bool FUSED, bool ROPE>
+static int launch_attn_kernel(const AttnMaps& maps, const AttnParams& p, const AttnPlan& pl,
+                              cudaStream_t s) {
+  constexpr size_t smem = attn_smem_bytes<D, G, kStages, ROPE>();
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  int na = 1;
+  if (pl.cm > 0) {
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = static_cast<unsigned>(pl.cm);
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    na = 2;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(pl.ctas));
+  cfg.blockDim = dim3(kThreads + 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = na;
+  return record_cuda_error(cudaLaunchKernelEx(&cfg, two_tier_attn_kernel<D, G, FUSED, kStages, ROPE>, maps, p));
+}
+
 template <int D, int G, bool FUSED, bool ROPE>
 static int launch_attn(const AttnMaps& maps, const AttnParams& p0, long long total_tiles,
                        cudaStream_t s) {
-  constexpr size_t smem = attn_smem_bytes<D, G, kStages, ROPE>();
   AttnPlan pl;
   int st = plan_attn<D, G, FUSED, ROPE>(total_tiles, p0.tpu, &pl);
   if (st != CMC_OK) return st;
   AttnParams p = p0;
   p.base = pl.base;
   p.rem = pl.rem;
-  st = launch_pdl(two_tier_attn_kernel<D, G, FUSED, kStages, ROPE>, dim3(static_cast<unsigned>(pl.ctas)),
-                  dim3(kThreads + 32), smem, s, maps, p);
+  p.cm = pl.cm;
+  st = launch_attn_kernel<D, G, FUSED, ROPE>(maps, p, pl, s);
   if (st != CMC_OK || !pl.split) return st;
   return launch_pdl(two_tier_combine_kernel<D, G>, dim3(static_cast<unsigned>(total_tiles / p.tpu)),
                     dim3(kThreads), 0, s, p);
@@ -1343,6 +1499,7 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   p.rot = p.t1_tiles % tpu;  // the first ring tile
   p.base = 0;
   p.rem = 0;
+  p.cm = 0;
   const float sc = scale > 0.f ? scale : 1.0f / sqrtf(static_cast<float>(m.d));
   p.scale_log2 = sc * 1.4426950408889634f;
   p.rope_offset = rope ? rope_offset : 0;

@@ -391,7 +391,48 @@ def test_decode_attn_plan(cuda_device):
     ctas, launches = cmc.decode_attn_plan(dims, fused=False)
     assert launches in (1, 2) and ctas >= 64
     if 2 * sms >= 256:
-        assert (ctas, launches) == (256, 2)
+        # 64 units of 64 tiles, four CTAs per unit: clusters merged in
+        # distributed shared memory, no combine launch
+        assert (ctas, launches) == (256, 1)
+
+
+def _cluster_case(B, L, Hkv, k, W, N=None, T=3):
+    Hq = 4 * Hkv
+    return WORKLOADS["tiny"].with_(B=B, L=L, Hq=Hq, Hkv=Hkv, d=128, N=N or max(k, 1) + 17, k=k,
+                                   W=W, T=T, kv_std=1.0 / np.sqrt(128), q_std=1.0 / np.sqrt(128),
+                                   W0=tuple((W * (i + 1)) // B for i in range(B)))
+
+
+# (B, L, Hkv, k, W): units B*L*Hkv, tiles per unit ceil(k/64) + ceil(W/64);
+# on 152 SMs with two CTAs each these give clusters of 2, 3, 5 and 8 CTAs per
+# unit, and a flat split (20 CTAs per unit) merged by the combine kernel
+CLUSTER_CASES = [(19, 1, 8, 64, 64), (1, 1, 2, 32, 128), (15, 1, 4, 128, 192),
+                 (19, 2, 1, 256, 256), (1, 1, 2, 640, 640)]
+
+
+@pytest.mark.parametrize("mode", MODES)
+@pytest.mark.parametrize("case", CLUSTER_CASES, ids=lambda c: "x".join(map(str, c)))
+def test_split_units(cuda_device, case, mode):
+    """Units shared by several CTAs: each plan's launches, and parity with
+    the oracle over ragged fills (some CTAs of a unit hold no key)."""
+    B, L, Hkv, k, W = case
+    w = _cluster_case(B, L, Hkv, k, W)
+    tpu = -(-k // 64) + -(-W // 64)
+    units = B * L * Hkv
+    sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
+    dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.N, w.k, w.W)
+    ctas, launches = cmc.decode_attn_plan(dims)
+    m = min((2 * sms) // units, tpu)
+    # two resident CTAs per SM (the plan of more units than that fills them)
+    two_per_sm = cmc.decode_attn_plan(cmc.CmcDims(2 * sms + 1, 1, 4, 1, 128, 64, 64, 64))[0] == 2 * sms
+    if two_per_sm and 2 * sms >= units:
+        assert ctas == units * m
+        assert launches == (2 if m > 8 else 1)
+    P = Problem(w, cuda_device, mode=mode)
+    for t in range(w.T):
+        out, ref = P.step(step_inputs(w, t))
+        assert_attn_close(to_f64(out), ref, f"split units {case} step {t}")
+    P.check_state()
 
 
 # ----------------------------------------------------------------------------
