@@ -27,7 +27,11 @@ namespace cmc {
 
 constexpr int kScoreThreads = 256;
 constexpr int kScoreUnroll = 4;
-constexpr int kSelectThreads = 512;
+// Threads of the selection CTA: 512 for banks of up to kSelectWideN CMEs, 1024
+// above (measured: the wider block halves the top-k time at 16,384 CMEs and
+// costs a little at 1,024).
+constexpr int kSelectThreadsMax = 1024;
+constexpr int kSelectWideN = 8192;
 
 __global__ void __launch_bounds__(kScoreThreads)
 cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ bank, int N, int D,
@@ -131,12 +135,13 @@ question_pool_kernel(const float* __restrict__ tokens, const int32_t* __restrict
   reinterpret_cast<float4*>(q_vec + static_cast<long long>(b) * D)[c4] = acc;
 }
 
-// Exclusive prefix sum of one value per thread over the block (kSelectThreads
-// threads, warps in order); `wsum` is a kSelectThreads/32-entry shared array
+// Exclusive prefix sum of one value per thread over the block (NT threads,
+// warps in order); `wsum` is an NT/32-entry shared array
 // used by this call only.  Returns this thread's exclusive prefix; *total gets
 // the block total.
+template <int NT>
 __device__ __forceinline__ uint32_t block_exclusive_sum(uint32_t v, uint32_t* wsum, uint32_t* total) {
-  constexpr int kW = kSelectThreads / 32;
+  constexpr int kW = NT / 32;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t inc = v;
 #pragma unroll
@@ -158,8 +163,13 @@ __device__ __forceinline__ uint32_t block_exclusive_sum(uint32_t v, uint32_t* ws
 }
 
 // Sequences of at most this many CMEs keep their keys in shared memory for
-// the radix passes and the compaction; longer ones re-read the scores.
-constexpr int kSelectSmemKeys = 16384;
+// the radix passes and the compaction; longer ones re-read the scores.  Key
+// j sits at word j + j / 32, so that the compaction's threads, each reading
+// its own run of consecutive keys, hit different banks.
+constexpr int kSelectSmemKeys = 49152;
+__host__ __device__ constexpr size_t select_smem_words(int n) {
+  return static_cast<size_t>(n) + static_cast<size_t>(n) / 32 + 1;
+}
 
 // CME-guided localisation for the Tier-2 window (optional part of the
 // selection CTA): alpha = offset of the chunk behind the CME of largest norm
@@ -175,8 +185,8 @@ struct LocateArgs {
 };
 
 __device__ __forceinline__ void locate_window(const LocateArgs& la, int b, int N) {
-  __shared__ float wbest[kSelectThreads / 32];
-  __shared__ int wbidx[kSelectThreads / 32];
+  __shared__ float wbest[kSelectThreadsMax / 32];
+  __shared__ int wbidx[kSelectThreadsMax / 32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const float* sq = la.sqnorm + static_cast<long long>(b) * N;
   float best = -1.f;
@@ -206,12 +216,13 @@ __device__ __forceinline__ void locate_window(const LocateArgs& la, int b, int N
   }
 }
 
-__global__ void __launch_bounds__(kSelectThreads)
+template <int NT>
+__global__ void __launch_bounds__(NT)
 topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __restrict__ idx_out,
                    const LocateArgs la) {
   extern __shared__ uint32_t skeys[];
   __shared__ uint32_t hist[256];
-  __shared__ uint32_t wsum[3][kSelectThreads / 32];
+  __shared__ uint32_t wsum[3][NT / 32];
   __shared__ uint32_t sh_prefix, sh_krem;
   const int b = blockIdx.x;
   const int tid = threadIdx.x;
@@ -229,9 +240,9 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
   const bool in_smem = N <= kSelectSmemKeys;
   for (int j = tid; j < 256; j += blockDim.x) hist[j] = 0u;
   if (in_smem)
-    for (int j = tid; j < N; j += blockDim.x) skeys[j] = orderable(s[j]);
+    for (int j = tid; j < N; j += blockDim.x) skeys[j + (j >> 5)] = orderable(s[j]);
   __syncthreads();
-  auto key_at = [&](int j) -> uint32_t { return in_smem ? skeys[j] : orderable(s[j]); };
+  auto key_at = [&](int j) -> uint32_t { return in_smem ? skeys[j + (j >> 5)] : orderable(s[j]); };
 
   // Radix select, 8 bits a pass from the top: after the passes `prefix` is the
   // key T of the k-th largest score and krem of the keys equal to T are kept.
@@ -296,7 +307,7 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
       if (j < N && key_at(j) == T) ++n_eq;
     }
     uint32_t eq_total, sel_total;
-    const uint32_t eq0 = run_eq + block_exclusive_sum(n_eq, wsum[1], &eq_total);
+    const uint32_t eq0 = run_eq + block_exclusive_sum<NT>(n_eq, wsum[1], &eq_total);
     uint32_t n_sel = 0u, r = eq0;
     for (int e = 0; e < C; ++e) {
       const int j = j0 + e;
@@ -306,7 +317,7 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
         else if (key == T) n_sel += (r++ < krem) ? 1u : 0u;
       }
     }
-    uint32_t slot = run_sel + block_exclusive_sum(n_sel, wsum[2], &sel_total);
+    uint32_t slot = run_sel + block_exclusive_sum<NT>(n_sel, wsum[2], &sel_total);
     r = eq0;
     for (int e = 0; e < C; ++e) {
       const int j = j0 + e;
@@ -342,15 +353,21 @@ static int launch_score_select(const float* question_emb, const float* cme_bank,
   if (st != CMC_OK) return st;
   if (dev >= 0 && dev < 64) {
     std::call_once(attr_once[dev], [&] {
-      st = record_cuda_error(cudaFuncSetAttribute(topk_select_kernel,
-                                                  cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                  static_cast<int>(kSelectSmemKeys * sizeof(uint32_t))));
+      const int bytes = static_cast<int>(select_smem_words(kSelectSmemKeys) * sizeof(uint32_t));
+      st = record_cuda_error(cudaFuncSetAttribute(topk_select_kernel<512>,
+                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+      if (st == CMC_OK)
+        st = record_cuda_error(cudaFuncSetAttribute(topk_select_kernel<kSelectThreadsMax>,
+                                                    cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
     });
     if (st != CMC_OK) return st;
   }
   const size_t smem =
-      (N <= kSelectSmemKeys && k > 0 && k < N) ? static_cast<size_t>(N) * sizeof(uint32_t) : 0;
-  return launch_pdl(topk_select_kernel, dim3(B), dim3(kSelectThreads), smem, s,
+      (N <= kSelectSmemKeys && k > 0 && k < N) ? select_smem_words(N) * sizeof(uint32_t) : 0;
+  if (N > kSelectWideN)
+    return launch_pdl(topk_select_kernel<kSelectThreadsMax>, dim3(B), dim3(kSelectThreadsMax), smem, s,
+                      static_cast<const float*>(sc), N, k, idx_out, la);
+  return launch_pdl(topk_select_kernel<512>, dim3(B), dim3(512), smem, s,
                     static_cast<const float*>(sc), N, k, idx_out, la);
 }
 
