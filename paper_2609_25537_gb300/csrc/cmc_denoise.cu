@@ -19,16 +19,15 @@
 //     tile's 32 pass bits also go to a word of the workspace, and the tile's
 //     positions of kept_idx are set to -1 (the compaction overwrites the
 //     kept ones).
-//  2. denoise_compact_kernel -- one CTA per context.  Walking left to right,
-//     the keep-minimum forces token i exactly when it fails the test and its
+//  2. denoise_compact_kernel -- one cluster of 8 CTAs per context.  Walking
+//     left to right, the keep-minimum forces token i exactly when it fails the test and its
 //     distance to the last token that passed (or to position -1) is a
 //     multiple of keep_every, so the walk is data-parallel.  A thread takes
-//     four 32-token pass words (one 16-byte load) per segment of 131,072
-//     tokens (the next segment's words are loaded ahead); a block-wide prefix
-//     maximum gives it the last passing position before its words, from
-//     which the forced positions of each gap follow with one division; a
-//     block-wide prefix sum places its kept positions; both carry from one
-//     segment to the next.
+//     one 32-token pass word per segment of 262,144 tokens (the next
+//     segment's word is loaded ahead); a cluster-wide prefix maximum gives it
+//     the last passing position before its word, from which the forced
+//     positions of each gap follow with one division; a cluster-wide prefix
+//     sum places its kept positions; both carry from one segment to the next.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -47,7 +46,8 @@ constexpr int kPassStageBytes = kPassStageRows * kPassChunk * 4;  // 20 KB
 constexpr int kPassStages = 4;
 constexpr int kPassSmem = kPassStages * kPassStageBytes;          // 80 KB
 constexpr int kCompactThreads = 1024;
-constexpr int kCompactWords = 4;  // pass words (32 tokens each) per compaction thread
+constexpr int kCompactWords = 4;  // pass words per 16-byte group of the word array's rows
+constexpr int kCompactCtas = 8;   // CTAs (one thread-block cluster) per context
 
 __device__ __forceinline__ void dn_cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes)
@@ -269,63 +269,99 @@ __device__ __forceinline__ uint32_t keep_mask(uint32_t m, int lp, int i0, int K)
   return kept;
 }
 
+__device__ __forceinline__ void dn_cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\n" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire;\n" ::: "memory");
+}
+__device__ __forceinline__ uint32_t dn_cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+  return r;
+}
+// Value of an int in the shared memory of CTA `rank` of the cluster, at the
+// same offset as `local` in this CTA.
+__device__ __forceinline__ int dn_ld_peer(const int* local, uint32_t rank) {
+  uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(local)), r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(rank));
+  int v;
+  asm volatile("ld.shared::cluster.s32 %0, [%1];\n" : "=r"(v) : "r"(r) : "memory");
+  return v;
+}
+
+// One cluster of kCompactCtas CTAs per context.  A segment is
+// kCompactCtas * kCompactThreads pass words (32 tokens each), one per
+// thread, CTA r taking the r-th run of kCompactThreads words.  Both scans
+// (the last passing position, then the kept counts) go block-wide first;
+// each CTA then publishes its block total in shared memory, and after a
+// cluster barrier every thread adds the totals of the CTAs before its own
+// (distributed shared memory).  The published totals are double-buffered by
+// segment parity, so two cluster barriers per segment suffice; a last one
+// keeps them readable until every CTA is done.  Every thread of the cluster
+// passes the same barriers (all CTAs of a cluster walk the same context).
 __global__ void __launch_bounds__(kCompactThreads)
 denoise_compact_kernel(const uint32_t* __restrict__ masks, const int32_t* __restrict__ n_tokens,
                        int n_max, int words_stride, int keep_every,
                        int32_t* __restrict__ kept_idx, int32_t* __restrict__ kept_count) {
-  constexpr int WPT = kCompactWords;  // pass words per thread and segment
+  constexpr int CS = kCompactCtas;
+  constexpr int SEGW = CS * kCompactThreads;  // words per segment
   __shared__ int red[kCompactThreads / 32];
+  __shared__ int pub[2][2];  // [segment parity][last passing position, kept count]
   pdl_wait();
   pdl_trigger();
-  const int b = blockIdx.x;
+  const int b = blockIdx.x / CS;
+  const int rank = static_cast<int>(dn_cluster_rank());
   const int tid = threadIdx.x;
   int n = n_tokens ? n_tokens[b] : n_max;
   n = n < 0 ? 0 : (n > n_max ? n_max : n);
-  const uint4* mb = reinterpret_cast<const uint4*>(masks + static_cast<long long>(b) * words_stride);
+  const uint32_t* mb = masks + static_cast<long long>(b) * words_stride;
   int32_t* out = kept_idx + static_cast<long long>(b) * n_max;
-  const int nq = (n + 32 * WPT - 1) / (32 * WPT);  // uint4s of words that hold tokens
-  int carry_last = -1;                              // last passing position before the segment
-  int carry_cnt = 0;                                // tokens kept before the segment
-  uint4 next = tid < nq ? mb[tid] : make_uint4(0u, 0u, 0u, 0u);
-  for (int q0 = 0; q0 < nq; q0 += kCompactThreads) {
-    const int qi = q0 + tid;
-    const uint4 raw = next;
-    if (qi + kCompactThreads < nq) next = mb[qi + kCompactThreads];  // the next segment's words
-    const uint32_t wr[WPT] = {raw.x, raw.y, raw.z, raw.w};
-    const int t0 = 32 * WPT * qi;  // first token of this thread's words
-    uint32_t m[WPT];
-    int last = -1;
-#pragma unroll
-    for (int j = 0; j < WPT; ++j) {
-      const int nv = min(max(n - (t0 + 32 * j), 0), 32);  // tokens of word j that exist
-      m[j] = wr[j] & (nv >= 32 ? ~0u : ((1u << nv) - 1u));
-      if (m[j]) last = t0 + 32 * j + 31 - __clz(m[j]);
+  const int nw = (n + 31) / 32;  // words that hold tokens
+  int carry_last = -1;           // last passing position before the segment
+  int carry_cnt = 0;             // tokens kept before the segment
+  const int mine = rank * kCompactThreads + tid;  // this thread's word within a segment
+  uint32_t next = mine < nw ? mb[mine] : 0u;
+  int par = 0;
+  for (int w0 = 0; w0 < nw; w0 += SEGW, par ^= 1) {
+    const int wi = w0 + mine;
+    const uint32_t raw = next;
+    if (wi + SEGW < nw) next = mb[wi + SEGW];  // the next segment's word
+    const int i0 = 32 * wi;
+    const int nv = min(max(n - i0, 0), 32);  // tokens of this word that exist
+    const uint32_t valid = nv >= 32 ? ~0u : ((1u << nv) - 1u);
+    const uint32_t m = raw & valid;
+    const int last = m ? i0 + 31 - __clz(m) : -1;
+    int cta_last;
+    int lp = block_excl_max(last, red, &cta_last);
+    if (tid == 0) pub[par][0] = cta_last;
+    dn_cluster_sync();
+    int seg_last = carry_last;
+    for (int r = 0; r < CS; ++r) {
+      const int v = dn_ld_peer(&pub[par][0], static_cast<uint32_t>(r));
+      if (r < rank) lp = max(lp, v);
+      seg_last = max(seg_last, v);
     }
-    int seg_last, seg_cnt;
-    int lp = max(block_excl_max(last, red, &seg_last), carry_last);
-    uint32_t kept[WPT];
-    int cnt = 0;
-#pragma unroll
-    for (int j = 0; j < WPT; ++j) {
-      const int i0 = t0 + 32 * j;
-      const int nv = min(max(n - i0, 0), 32);
-      kept[j] = nv > 0 ? keep_mask(m[j], lp, i0, keep_every) & (nv >= 32 ? ~0u : ((1u << nv) - 1u)) : 0u;
-      cnt += __popc(kept[j]);
-      if (m[j]) lp = i0 + 31 - __clz(m[j]);
+    lp = max(lp, carry_last);
+    uint32_t kept = nv > 0 ? keep_mask(m, lp, i0, keep_every) & valid : 0u;
+    int cta_cnt;
+    int slot = block_excl_sum(__popc(kept), red, &cta_cnt);
+    if (tid == 0) pub[par][1] = cta_cnt;
+    dn_cluster_sync();
+    int seg_cnt = 0;
+    for (int r = 0; r < CS; ++r) {
+      const int v = dn_ld_peer(&pub[par][1], static_cast<uint32_t>(r));
+      if (r < rank) slot += v;
+      seg_cnt += v;
     }
-    int slot = carry_cnt + block_excl_sum(cnt, red, &seg_cnt);
-#pragma unroll
-    for (int j = 0; j < WPT; ++j) {
-      uint32_t k = kept[j];
-      while (k) {
-        out[slot++] = t0 + 32 * j + __ffs(k) - 1;
-        k &= k - 1;
-      }
+    slot += carry_cnt;
+    while (kept) {
+      out[slot++] = i0 + __ffs(kept) - 1;
+      kept &= kept - 1;
     }
-    carry_last = max(carry_last, seg_last);
+    carry_last = seg_last;
     carry_cnt += seg_cnt;
   }
-  if (tid == 0) kept_count[b] = carry_cnt;
+  dn_cluster_sync();  // the peers' published totals stay readable until here
+  if (rank == 0 && tid == 0) kept_count[b] = carry_cnt;
 }
 
 }  // namespace cmc
@@ -400,9 +436,22 @@ int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int
     default: return CMC_ERR_RANGE;
   }
   if (st != CMC_OK) return st;
-  return launch_pdl(denoise_compact_kernel, dim3(B), dim3(kCompactThreads), 0, s,
-                    static_cast<const uint32_t*>(masks), n_tokens, n_max, dn_words_stride(n_max), keep_every,
-                    kept_idx, kept_count);
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = kCompactCtas;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(B) * kCompactCtas);
+  cfg.blockDim = dim3(kCompactThreads);
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return record_cuda_error(cudaLaunchKernelEx(&cfg, denoise_compact_kernel,
+                                              static_cast<const uint32_t*>(masks), n_tokens, n_max,
+                                              dn_words_stride(n_max), keep_every, kept_idx, kept_count));
 }
 
 }  // extern "C"

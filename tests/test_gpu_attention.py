@@ -396,10 +396,9 @@ def test_decode_attn_plan(cuda_device):
         assert (ctas, launches) == (256, 1)
 
 
-def _cluster_case(B, L, Hkv, k, W, N=None, T=3):
-    Hq = 4 * Hkv
-    return WORKLOADS["tiny"].with_(B=B, L=L, Hq=Hq, Hkv=Hkv, d=128, N=N or max(k, 1) + 17, k=k,
-                                   W=W, T=T, kv_std=1.0 / np.sqrt(128), q_std=1.0 / np.sqrt(128),
+def _cluster_case(B, L, Hkv, k, W, N=None, T=3, G=4, d=128):
+    return WORKLOADS["tiny"].with_(B=B, L=L, Hq=G * Hkv, Hkv=Hkv, d=d, N=N or max(k, 1) + 17, k=k,
+                                   W=W, T=T, kv_std=1.0 / np.sqrt(d), q_std=1.0 / np.sqrt(d),
                                    W0=tuple((W * (i + 1)) // B for i in range(B)))
 
 
@@ -433,6 +432,19 @@ def test_split_units(cuda_device, case, mode):
         out, ref = P.step(step_inputs(w, t))
         assert_attn_close(to_f64(out), ref, f"split units {case} step {t}")
     P.check_state()
+
+
+@pytest.mark.parametrize("G,d", [(8, 128), (1, 64), (2, 64), (8, 64)])
+def test_split_units_head_shapes(cuda_device, G, d):
+    """Clusters of 3 and 5 CTAs per unit with other query-group sizes and head
+    dimensions (the merge's share of output columns per CTA differs)."""
+    for case in ((1, 1, 2, 32, 128), (15, 1, 4, 128, 192)):
+        w = _cluster_case(*case, G=G, d=d)
+        P = Problem(w, cuda_device, mode="dense")
+        for t in range(w.T):
+            out, ref = P.step(step_inputs(w, t))
+            assert_attn_close(to_f64(out), ref, f"split units {case} G={G} d={d} step {t}")
+        P.check_state()
 
 
 # ----------------------------------------------------------------------------
