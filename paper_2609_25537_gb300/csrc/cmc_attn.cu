@@ -59,6 +59,7 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <cstring>
 #include <mutex>
 
@@ -1312,11 +1313,11 @@ template <int D, int G, bool FUSED, bool ROPE>
 static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
   constexpr size_t smem = attn_smem_bytes<D, G, kStages, ROPE>();
   auto kern = two_tier_attn_kernel<D, G, FUSED, kStages, ROPE>;
-  static int configured[64] = {0};  // per device: attribute set and occupancy known
+  static std::atomic<int> configured[64];  // per device: attribute set and occupancy known (idempotent)
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
   if (st != CMC_OK) return st;
-  int per_sm = (dev >= 0 && dev < 64) ? configured[dev] : 0;
+  int per_sm = (dev >= 0 && dev < 64) ? configured[dev].load(std::memory_order_acquire) : 0;
   if (per_sm <= 0) {
     st = record_cuda_error(
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
@@ -1324,7 +1325,7 @@ static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
     st = record_cuda_error(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads + 32, smem));
     if (st != CMC_OK) return st;
     if (per_sm < 1) per_sm = 1;
-    if (dev >= 0 && dev < 64) configured[dev] = per_sm;
+    if (dev >= 0 && dev < 64) configured[dev].store(per_sm, std::memory_order_release);
   }
   // Grid.  With no more units than resident CTAs: m = resident CTAs per unit
   // (at most one per tile).  m = 1: one CTA per unit, nothing is split.

@@ -24,6 +24,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "cmc_internal.cuh"
 
 namespace cmc {
@@ -258,16 +260,16 @@ int cmc_bridge_epilogue(const float* x, const float* gamma, const float* beta, i
     }
   }
   const size_t smem = static_cast<size_t>(kBridgeBufs) * D * sizeof(float);
-  static bool attr_set[64] = {false};
+  static std::atomic<bool> attr_set[64];  // per device: the attribute is set (idempotent)
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
   if (st != CMC_OK) return st;
-  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+  if (dev >= 0 && dev < 64 && !attr_set[dev].load(std::memory_order_acquire)) {
     st = record_cuda_error(cudaFuncSetAttribute(bridge_epilogue_kernel,
                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                 static_cast<int>(kBridgeBufs * kBridgeMaxD * sizeof(float))));
     if (st != CMC_OK) return st;
-    attr_set[dev] = true;
+    attr_set[dev].store(true, std::memory_order_release);
   }
   // Persistent CTAs, kBridgeCtasPerSm per SM (one when the row buffers leave
   // room for only one): each walks about rows / grid rows.

@@ -32,6 +32,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "cmc_internal.cuh"
 
 namespace cmc {
@@ -402,11 +404,11 @@ int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* pass = static_cast<uint8_t*>(workspace);
   uint32_t* masks = reinterpret_cast<uint32_t*>(pass + dn_words_offset(B, n_max));
-  static bool attr_set[64] = {false};
+  static std::atomic<bool> attr_set[64];  // per device: the attribute is set (idempotent)
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
   if (st != CMC_OK) return st;
-  if (dev >= 0 && dev < 64 && !attr_set[dev]) {
+  if (dev >= 0 && dev < 64 && !attr_set[dev].load(std::memory_order_acquire)) {
     const void* kerns[8] = {
         reinterpret_cast<const void*>(denoise_pass_kernel<1>), reinterpret_cast<const void*>(denoise_pass_kernel<2>),
         reinterpret_cast<const void*>(denoise_pass_kernel<3>), reinterpret_cast<const void*>(denoise_pass_kernel<4>),
@@ -416,7 +418,7 @@ int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int
       st = record_cuda_error(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kPassSmem));
       if (st != CMC_OK) return st;
     }
-    attr_set[dev] = true;
+    attr_set[dev].store(true, std::memory_order_release);
   }
   const int tiles_per_ctx = (n_max + kPassTile - 1) / kPassTile;
   const long long tiles = static_cast<long long>(B) * tiles_per_ctx;
