@@ -32,7 +32,8 @@ Reported (one JSON line on rank 0):
   variant        the decode step with the other Tier-1 form, us per launch;
   e2e            the same metric through the Python API with host buffers
                  (question vector, CME bank and every step's q / new K,V
-                 copied in from pinned memory, every step's output copied out);
+                 copied in from pinned memory, every step's output copied out,
+                 one copy each way per round of R decode steps);
   cpu_baseline   the fp64 oracle on the host, on a bounded sample.
 
 `--impl reference` times the fp64 oracle alone on the host cores (the
@@ -364,7 +365,7 @@ class Request:
         cmc.tier1_gather(self.t1k, self.t1v, self.idx, out_k=self.t1k_dense,
                          out_v=self.t1v_dense, workspace=self.ws_dense)
 
-    def decode(self, p, q=None, k_new=None, v_new=None, mode="dense", rope=False):
+    def decode(self, p, q=None, k_new=None, v_new=None, mode="dense", rope=False, out=None):
         """One fused decode step; with `rope` the GQA-layer step that rotates
         q and k_new (theta 5e5, the Llama-3 base; positions after the k
         Tier-1 rows)."""
@@ -372,13 +373,14 @@ class Request:
         q = self.q[p] if q is None else q
         k_new = self.k_new[p] if k_new is None else k_new
         v_new = self.v_new[p] if v_new is None else v_new
+        out = self.out if out is None else out
         kw = dict(rope_theta=500000.0, rope_offset=self.idx.shape[1]) if rope else {}
         if mode == "dense":
             cmc.decode_step(q, self.t1k_dense, self.t1v_dense, None, self.ring_k, self.ring_v,
-                            self.pos, k_new, v_new, out=self.out, workspace=self.ws_dense, **kw)
+                            self.pos, k_new, v_new, out=out, workspace=self.ws_dense, **kw)
         else:
             cmc.decode_step(q, self.t1k, self.t1v, self.idx, self.ring_k, self.ring_v,
-                            self.pos, k_new, v_new, out=self.out, workspace=self.ws, **kw)
+                            self.pos, k_new, v_new, out=out, workspace=self.ws, **kw)
 
     def host_state(self):
         def bits(t):
@@ -643,62 +645,67 @@ def run_gpu(args, w, world, rank, local):
 def run_e2e(args, w, reqs, dev, stream, world):
     """Same metric through the public Python API with host buffers: the
     question vector and CME bank of each request and, every decode step, q and
-    the new token's K,V (one packed pinned buffer per step) are copied in and
-    the output copied back to pinned host memory.  The per-step sequence is
-    captured in a CUDA graph of P rounds, as a serving loop would: copies in
-    run on one side stream and copies out on another, so they overlap the
-    decode kernels of the other requests; each request's decode waits for its
-    own inputs and for the previous read-back of its output buffer.
+    the new token's K,V are copied in from pinned host memory and the output
+    copied back to pinned host memory.  As a serving loop would, each
+    scheduling round (one decode step of each of the R requests) moves its
+    inputs in one host-to-device copy and its outputs in one device-to-host
+    copy, on two side streams, double-buffered by round parity: the copy in
+    of round p+1 overlaps the decode kernels of round p, and only the first
+    decode of a round waits on a copy (the others follow their predecessor by
+    programmatic dependent launch).  P rounds are captured in one CUDA graph.
     Selection and compaction run eagerly."""
     import paper_2609_25537_gb300 as cmc
     R, T, P = args.requests, args.decode_steps, args.pool
     steps = max(1, min(args.steps, args.e2e_steps))
     nq, nk = reqs[0].q[0].numel(), reqs[0].k_new[0].numel()
-    host = []
-    for r in reqs:
-        packed = torch.cat([r.q.reshape(P, -1), r.k_new.reshape(P, -1), r.v_new.reshape(P, -1)],
-                           dim=1)
-        inp_d = torch.empty(packed.shape[1], dtype=torch.bfloat16, device=dev)
-        h = {
-            "qemb": r.qemb.cpu().pin_memory(), "bank": r.bank.cpu().pin_memory(),
-            "inp": packed.cpu().pin_memory(), "inp_d": inp_d,
-            "q_d": inp_d[:nq].view(r.q[0].shape),
-            "k_d": inp_d[nq:nq + nk].view(r.k_new[0].shape),
-            "v_d": inp_d[nq + nk:].view(r.v_new[0].shape),
-            "out": torch.empty((P,) + tuple(r.out.shape), dtype=torch.bfloat16).pin_memory(),
-        }
-        host.append(h)
+    per_req = nq + 2 * nk
+    # host: round p holds the R requests' packed (q, k_new, v_new) of step p
+    host_in = torch.cat([torch.cat([r.q.reshape(P, -1), r.k_new.reshape(P, -1),
+                                    r.v_new.reshape(P, -1)], dim=1) for r in reqs],
+                        dim=1).cpu().pin_memory()                      # [P, R * per_req]
+    out_shape = tuple(reqs[0].out.shape)
+    host_out = torch.empty((P, R) + out_shape, dtype=torch.bfloat16).pin_memory()
+    host_sel = [(r.qemb.cpu().pin_memory(), r.bank.cpu().pin_memory()) for r in reqs]
+    in_d = [torch.empty(R * per_req, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    out_d = [torch.empty((R,) + out_shape, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+
+    def views(par, i):
+        base = in_d[par][i * per_req:(i + 1) * per_req]
+        return (base[:nq].view(reqs[i].q[0].shape), base[nq:nq + nk].view(reqs[i].k_new[0].shape),
+                base[nq + nk:].view(reqs[i].v_new[0].shape))
+
     s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
 
     def rounds():
-        """P rounds of R decode steps with their copies; returns after joining
-        the side streams back into `stream`."""
+        """P rounds with their copies; returns after joining the side streams
+        back into `stream`."""
         fork = torch.cuda.Event()
         fork.record(stream)
         s_in.wait_event(fork)
         s_out.wait_event(fork)
-        done = [None] * R   # decode finished (its inputs and output are final)
-        freed = [None] * R  # read-back of the output finished
+        decoded = [None, None]  # last round's decodes per buffer parity (inputs free)
+        copied = [None, None]   # last read-back per parity (output buffers free)
         for p in range(P):
-            for i, (r, h) in enumerate(zip(reqs, host)):
-                with torch.cuda.stream(s_in):
-                    if done[i] is not None:
-                        s_in.wait_event(done[i])
-                    h["inp_d"].copy_(h["inp"][p], non_blocking=True)
-                    ready = torch.cuda.Event()
-                    ready.record(s_in)
-                stream.wait_event(ready)
-                if freed[i] is not None:
-                    stream.wait_event(freed[i])
-                with torch.cuda.stream(stream):
-                    r.decode(p, q=h["q_d"], k_new=h["k_d"], v_new=h["v_d"], mode=args.tier1)
-                done[i] = torch.cuda.Event()
-                done[i].record(stream)
-                with torch.cuda.stream(s_out):
-                    s_out.wait_event(done[i])
-                    h["out"][p].copy_(r.out, non_blocking=True)
-                    freed[i] = torch.cuda.Event()
-                    freed[i].record(s_out)
+            par = p & 1
+            with torch.cuda.stream(s_in):
+                for ev in (decoded[par], copied[par]):
+                    if ev is not None:
+                        s_in.wait_event(ev)
+                in_d[par].copy_(host_in[p], non_blocking=True)
+                ready = torch.cuda.Event()
+                ready.record(s_in)
+            stream.wait_event(ready)
+            with torch.cuda.stream(stream):
+                for i, r in enumerate(reqs):
+                    q, k, v = views(par, i)
+                    r.decode(p, q=q, k_new=k, v_new=v, mode=args.tier1, out=out_d[par][i])
+            decoded[par] = torch.cuda.Event()
+            decoded[par].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(decoded[par])
+                host_out[p].copy_(out_d[par], non_blocking=True)
+                copied[par] = torch.cuda.Event()
+                copied[par].record(s_out)
         for side in (s_in, s_out):
             j = torch.cuda.Event()
             j.record(side)
@@ -716,9 +723,9 @@ def run_e2e(args, w, reqs, dev, stream, world):
 
     def step():
         with torch.cuda.stream(stream):
-            for r, h in zip(reqs, host):
-                r.qemb.copy_(h["qemb"], non_blocking=True)
-                r.bank.copy_(h["bank"], non_blocking=True)
+            for r, (hq, hb) in zip(reqs, host_sel):
+                r.qemb.copy_(hq, non_blocking=True)
+                r.bank.copy_(hb, non_blocking=True)
                 cmc.score_select(r.qemb, r.bank, w.k, idx_out=r.idx, workspace=r.sel_ws)
                 if args.tier1 == "dense":
                     r.gather()
@@ -736,12 +743,12 @@ def run_e2e(args, w, reqs, dev, stream, world):
         step()
     el = time.perf_counter() - t0
     el = max_over_ranks(el, world, dev)
-    h2d = R * (reqs[0].qemb.numel() * 4 + reqs[0].bank.numel() * 4
-               + T * 2 * host[0]["inp_d"].numel())
+    h2d = R * (reqs[0].qemb.numel() * 4 + reqs[0].bank.numel() * 4) + T * R * per_req * 2
     d2h = R * T * reqs[0].out.numel() * 2
     return {"value": world * steps * R * w.B * T / el, "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
-            "per_step_graph": graph is not None}
+            "per_step_graph": graph is not None,
+            "copies": "one host-to-device and one device-to-host copy per round of R decode steps"}
 
 
 def main(argv=None):
