@@ -751,6 +751,90 @@ def run_e2e(args, w, reqs, dev, stream, world):
             "copies": "one host-to-device and one device-to-host copy per round of R decode steps"}
 
 
+def run_ablation(args, dev):
+    """The ablation sweep on the Llama-3-8B head shape (one layer, bank of
+    1,024 CMEs): for every (k, W, B) of the grid, the fused decode step over a
+    dense Tier-1 cache of k rows (idx passed instead when k = 0: Tier-1 empty)
+    and a full ring of W slots, timed as CUDA graphs of 8 rounds of R requests
+    round-robin, R chosen so that R steps read at least 2 x 129 MB (at most
+    8; smaller points are L2-resident and latency-bound, and say so).  Inputs
+    are seeded Gaussian bf16 drawn on the device.  One JSON line."""
+    import paper_2609_25537_gb300 as cmc
+    from workloads.configs import ABLATION_B, ABLATION_K, ABLATION_W, ablation_workload
+    torch.cuda.set_device(dev)
+    cmc.lib()
+    stream = torch.cuda.Stream(device=dev)
+    peak, peak_kind = measured_peaks()
+    P, reps = 8, 20
+    rows = []
+    for k in ABLATION_K:
+        for W in ABLATION_W:
+            for B in ABLATION_B:
+                w = ablation_workload(k, W, B)
+                nbytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W,
+                                           gather=w.k == 0)
+                R = max(1, min(8, -(-2 * 129_000_000 // nbytes)))
+                g = torch.Generator(device=dev).manual_seed(4)
+
+                def randn(shape, std):
+                    return (torch.randn(shape, generator=g, device=dev) * std).to(torch.bfloat16)
+                reqs = []
+                for _ in range(R):
+                    kk = max(w.k, 1)
+                    st = {
+                        "t1k": randn((B, 1, w.Hkv, kk, w.d), w.kv_std),
+                        "t1v": randn((B, 1, w.Hkv, kk, w.d), w.kv_std),
+                        "idx": (torch.empty((B, 0), dtype=torch.int32, device=dev) if w.k == 0
+                                else None),
+                        "ring_k": randn((B, 1, w.Hkv, W, w.d), w.kv_std),
+                        "ring_v": randn((B, 1, w.Hkv, W, w.d), w.kv_std),
+                        "pos": torch.full((B,), W, dtype=torch.int64, device=dev),
+                        "q": randn((P, B, 1, w.Hq, w.d), w.q_std),
+                        "kn": randn((P, B, 1, w.Hkv, w.d), w.kv_std),
+                        "vn": randn((P, B, 1, w.Hkv, w.d), w.kv_std),
+                        "out": torch.empty((B, 1, w.Hq, w.d), dtype=torch.bfloat16, device=dev),
+                    }
+                    st["ws"] = cmc.DecodeWorkspace(
+                        cmc.dims_of(st["out"], st["t1k"], st["idx"], st["ring_k"]), dev)
+                    reqs.append(st)
+
+                def call(st, p):
+                    cmc.decode_step(st["q"][p], st["t1k"], st["t1v"], st["idx"], st["ring_k"],
+                                    st["ring_v"], st["pos"], st["kn"][p], st["vn"][p],
+                                    out=st["out"], workspace=st["ws"])
+                with torch.cuda.stream(stream):
+                    for st in reqs:
+                        call(st, 0)
+                stream.synchronize()
+                gr = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(gr, stream=stream):
+                    for p in range(P):
+                        for st in reqs:
+                            call(st, p)
+                with torch.cuda.stream(stream):
+                    for _ in range(3):
+                        gr.replay()
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                    for _ in range(reps):
+                        gr.replay()
+                    e1.record(stream)
+                stream.synchronize()
+                us = 1000.0 * e0.elapsed_time(e1) / (reps * P * R)
+                ctas, launches = cmc.decode_attn_plan(
+                    cmc.dims_of(reqs[0]["out"], reqs[0]["t1k"], reqs[0]["idx"], reqs[0]["ring_k"]))
+                gbs = nbytes / (us * 1e-6) / 1e9
+                rows.append({"k": k, "W": W, "B": B, "bytes_per_step": nbytes, "requests": R,
+                             "l2": "resident" if R * nbytes < 129_000_000 else "larger than L2",
+                             "us_per_step": round(us, 3), "achieved_gbs": round(gbs, 1),
+                             "frac": round(gbs / peak, 4), "ctas": ctas, "launches": launches})
+                del reqs, gr
+    print(json.dumps({"ablation": rows, "peak_gbs": peak, "peak_kind": peak_kind,
+                      "shape": "Llama-3-8B heads (32 q / 8 KV, d = 128), one layer, bank of 1,024 CMEs",
+                      "tier1": "dense (k = 0: none)"}), flush=True)
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -770,6 +854,8 @@ def main(argv=None):
     ap.add_argument("--variant-replays", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--ref-step-seconds", type=float, default=2.0)
+    ap.add_argument("--ablation", action="store_true",
+                    help="time the fused decode step over the k x W x B ablation grid instead")
     ap.add_argument("--denoise-tokens", type=int, default=0,
                     help="tokens of the denoised context (default N x 4, N x 8 for N >= 16384)")
     args = ap.parse_args(argv)
@@ -782,6 +868,8 @@ def main(argv=None):
         int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")), 0)
     if world != args.gpus and rank == 0:
         print(f"warning: --gpus {args.gpus} but WORLD_SIZE {world}", file=sys.stderr)
+    if args.ablation and args.impl == "cmc":
+        return run_ablation(args, torch.device("cuda", local))
     if args.impl == "reference":
         return run_reference(args, w, world, rank)
     return run_gpu(args, w, world, rank, local)

@@ -5,14 +5,14 @@
 // Work decomposition.  A unit is one (sequence b, layer l, KV head g).  Its
 // keys are cut into tiles of 64: ceil(k / 64) Tier-1 tiles, then ceil(W / 64)
 // tiles of ring slots; no tile mixes the two tiers.  With m = resident CTAs
-// per unit (at most one per tile): m = 1 (the Llama- and Mistral-shaped
-// steps) gives one CTA per unit, nothing split; 2 <= m <= 8 (long units, few
-// of them) gives thread-block clusters of m CTAs per unit, each CTA taking a
-// contiguous share of the unit's tiles: at the end every CTA leaves its fp32
-// (max, sum, output) record in its own shared memory, and after a cluster
-// barrier each CTA merges a slice of the output columns from all m records
-// (distributed shared memory, log-sum-exp rescale); m > 8, or more units
-// than resident CTAs, splits the flattened (unit, tile) list into equal
+// per unit (at most one per tile, at most 8): m = 1 (the Llama- and
+// Mistral-shaped steps) gives one CTA per unit, nothing split; m >= 2 (long
+// units, few of them) gives thread-block clusters of m CTAs per unit, each
+// CTA taking a contiguous share of the unit's tiles: at the end every CTA
+// leaves its fp32 (max, sum, output) record in its own shared memory, and
+// after a cluster barrier each CTA merges a slice of the output columns from
+// all m records (distributed shared memory, log-sum-exp rescale).  More units
+// than resident CTAs splits the flattened (unit, tile) list into equal
 // contiguous ranges (stream-K), partial records go to global memory, and a
 // small combine kernel that follows on the stream merges them.  No CTA ever
 // waits on another outside its cluster's two barriers.
@@ -1327,12 +1327,15 @@ static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
     if (per_sm < 1) per_sm = 1;
     if (dev >= 0 && dev < 64) configured[dev].store(per_sm, std::memory_order_release);
   }
-  // Grid.  With no more units than resident CTAs: m = resident CTAs per unit
-  // (at most one per tile).  m = 1: one CTA per unit, nothing is split.
-  // 2 <= m <= 8: clusters of m CTAs per unit, merged in distributed shared
-  // memory.  m > 8 (few, long units): a flat split of m CTAs per unit merged
-  // by the combine kernel.  More units than resident CTAs: one wave of CTAs,
-  // each taking an equal share of the flattened tiles (combine kernel).
+  // Grid.  With no more units than resident CTAs: m = resident CTAs per unit,
+  // at most one per tile and at most 8 (the portable cluster size).  m = 1:
+  // one CTA per unit, nothing is split.  m >= 2: clusters of m CTAs per unit,
+  // merged in distributed shared memory.  More units than resident CTAs: one
+  // wave of CTAs, each taking an equal share of the flattened tiles (stream-K;
+  // the combine kernel merges the units cut between CTAs).  (A flat split
+  // for few, long units -- m up to 38 at one sequence of one layer -- left
+  // about one tile per CTA and a combine over 38 records: 33.4 us against
+  // 9.4 us for clusters of 8 at k = 1024, W = 2048.)
   const long long slots = static_cast<long long>(per_sm) * sm_count();
   const long long units = total_tiles / tpu;
   pl->cm = 0;
@@ -1340,7 +1343,8 @@ static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
   if (units <= slots) {
     long long m = slots / units;
     if (m > tpu) m = tpu;
-    if (m >= 2 && m <= kMaxClusterCtas) pl->cm = static_cast<int>(m);
+    if (m > kMaxClusterCtas) m = kMaxClusterCtas;
+    if (m >= 2) pl->cm = static_cast<int>(m);
     ctas = units * m;
   } else {
     ctas = slots;
