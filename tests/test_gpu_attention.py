@@ -409,18 +409,24 @@ CLUSTER_CASES = [(19, 1, 8, 64, 64), (1, 1, 2, 32, 128), (15, 1, 4, 128, 192),
                  (19, 2, 1, 256, 256), (1, 1, 2, 640, 640)]
 
 
-def test_stream_k_plan(cuda_device):
-    """More units than resident CTAs: one wave, tiles split evenly (units cut
-    between CTAs), the combine kernel merges them; parity over ragged fills."""
+@pytest.mark.parametrize("extra,launches", [(17, 2), (None, 1)])
+def test_more_units_than_ctas(cuda_device, extra, launches):
+    """More units than resident CTAs.  A few units over a multiple of the CTA
+    count: tiles split evenly (units cut between CTAs) and the combine kernel
+    merges them.  Half again as many: whole units per CTA, one launch.  Parity
+    over ragged fills either way."""
     sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
-    w = _cluster_case(2 * sms + 17, 1, 2, 64, 128, T=2)
+    B = 2 * sms + extra if extra is not None else 3 * sms // 2
+    w = _cluster_case(B, 1, 2, 64, 128, T=2)
     dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.N, w.k, w.W)
-    ctas, launches = cmc.decode_attn_plan(dims)
-    assert launches == 2 and ctas <= w.B * w.Hkv
+    ctas, got = cmc.decode_attn_plan(dims)
+    two_per_sm = cmc.decode_attn_plan(cmc.CmcDims(2 * sms + 1, 1, 4, 1, 128, 64, 64, 64))[0] == 2 * sms
+    if two_per_sm:
+        assert (ctas, got) == (2 * sms, launches)
     P = Problem(w, cuda_device, mode="dense")
     for t in range(w.T):
         out, ref = P.step(step_inputs(w, t))
-        assert_attn_close(to_f64(out), ref, f"stream-K step {t}")
+        assert_attn_close(to_f64(out), ref, f"{w.B * w.Hkv} units step {t}")
     P.check_state()
 
 
