@@ -312,12 +312,14 @@ CMC_API int cmc_tier1_gather(const void* bank_k, const void* bank_v, const int32
  * (fused == 1) or cmc_decode_step_rope (fused == 2) for `dims` on the
  * current device: *ctas receives the grid size
  * of the attention kernel and *launches the number of kernels one call
- * enqueues: 1 when every (sequence, layer, KV head) unit is handled by one
- * CTA or by a thread-block cluster of 2 to 8 CTAs that merge their partial
- * results in distributed shared memory; 2 when units are split further (or
- * there are more units than resident CTAs) and a combine kernel merges the
- * partial results.  No work is enqueued.  Useful for sizing CUDA graphs and
- * for counting launches.
+ * enqueues: 1 when every (sequence, layer, KV head) unit is handled whole by
+ * one CTA (several units per CTA when there are more units than resident
+ * CTAs and they share out evenly enough) or by a thread-block cluster of 2 to
+ * 8 CTAs that merge their partial results in distributed shared memory; 2
+ * when, with more units than resident CTAs, the tiles are split evenly
+ * instead (units cut between CTAs) and a combine kernel merges the partial
+ * results.  No work is enqueued.  Useful for sizing CUDA graphs and for
+ * counting launches.
  */
 CMC_API int cmc_decode_attn_plan(const cmc_dims* dims, int fused, int* ctas, int* launches);
 
