@@ -484,7 +484,7 @@ def run_gpu(args, w, world, rank, local):
     value = job_tokens_per_s(world, K, R, w.B, T, max_ms)
 
     launches_dec = K * R * T
-    # kernels per fused decode call (attention, plus combine if units are split)
+    # kernels per fused decode call (attention, plus combine after a stream-K split)
     step_ctas, step_launches = cmc.decode_attn_plan(
         cmc.dims_of(reqs[0].out, reqs[0].t1k_dense if mode == "dense" else reqs[0].t1k,
                     None if mode == "dense" else reqs[0].idx, reqs[0].ring_k), fused=True)
@@ -494,6 +494,10 @@ def run_gpu(args, w, world, rank, local):
     elif step_ctas > n_units:
         plan_txt = (f" (clusters of {step_ctas // n_units} CTAs per unit, merged in distributed "
                     "shared memory; one launch)")
+    elif step_ctas < n_units:
+        plan_txt = " (whole units per CTA; one launch)"
+    elif step_ctas < n_units:
+        plan_txt = " (whole units per CTA; one launch)"
     else:
         plan_txt = " (one CTA per unit; one launch)"
     launch_us = 1000.0 * sum(dec_ms) / launches_dec

@@ -1334,8 +1334,9 @@ static int plan_attn(long long total_tiles, int tpu, AttnPlan* pl) {
   // at most one per tile and at most 8 (the portable cluster size).  m = 1:
   // one CTA per unit, nothing is split.  m >= 2: clusters of m CTAs per unit,
   // merged in distributed shared memory.  More units than resident CTAs: one
-  // wave of CTAs, each taking an equal share of the flattened tiles (stream-K;
-  // the combine kernel merges the units cut between CTAs).  (A flat split
+  // wave of CTAs, each taking a run of whole units or, when that would leave
+  // too few CTAs for the last round, an equal share of the flattened tiles
+  // (stream-K; the combine kernel merges the units cut between CTAs).  (A flat split
   // for few, long units -- m up to 38 at one sequence of one layer -- left
   // about one tile per CTA and a combine over 38 records: 33.4 us against
   // 9.4 us for clusters of 8 at k = 1024, W = 2048.)

@@ -378,8 +378,8 @@ def test_tier1_gather_bad_index_zero_row_and_flag(cuda_device):
 
 def test_decode_attn_plan(cuda_device):
     """One CTA per (layer, KV head) unit and a single launch per step at the
-    Llama-3-8B shape when 256 CTAs fit in one wave; split units (long-context
-    shape) add the combine launch."""
+    Llama-3-8B shape when 256 CTAs fit in one wave; the long-context shape's
+    long units are split over clusters, still one launch."""
     sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
     w = WORKLOADS["llama3_8b"]
     dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.k, w.W)
