@@ -496,8 +496,6 @@ def run_gpu(args, w, world, rank, local):
                     "shared memory; one launch)")
     elif step_ctas < n_units:
         plan_txt = " (whole units per CTA; one launch)"
-    elif step_ctas < n_units:
-        plan_txt = " (whole units per CTA; one launch)"
     else:
         plan_txt = " (one CTA per unit; one launch)"
     launch_us = 1000.0 * sum(dec_ms) / launches_dec
