@@ -112,7 +112,8 @@ struct AttnParams {
   float scale_log2;       // softmax scale * log2(e)
   long long rope_offset;  // rotary embedding (GQA-layer step): position of ring token 0
   int l2_prefetch;        // box tiles per CTA prefetched into L2 before the grid dependency wait
-  double rope_inv_freq[64];  // theta^(-2i/d) for the d/2 pairs, computed on the host
+  unsigned long long rope_turns[64];  // theta^(-2i/d) / (2 pi) of the d/2 pairs as 0.64 fixed
+                                      // point (turns per position), computed on the host
 };
 
 // ---------------------------------------------------------------------------
@@ -456,25 +457,31 @@ __device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
 // Rotary embedding of a GQA-layer step: (cos, sin) of the angle
 // p * theta^(-2i/d) of pairs i = lane and lane + 32 (i < d/2) at the new
 // token's position p = rope_offset + pos.  Angles reach 10^5 rad and more, so
-// the product and its reduction to [-pi, pi] (2 pi split into a high and a
-// low part) are done in double; sine and cosine of the reduced angle in float.
+// they are reduced in turns with integer arithmetic: with F_i =
+// theta^(-2i/d) / (2 pi) held as a 64-bit binary fraction (rounded on the
+// host), p * F_i mod 2^64 is the fractional turn of the angle, off by at most
+// p * 2^-65 turns; its top 32 bits, read as a signed fraction of a half turn,
+// give the angle in [-pi, pi) for sincospif.  Below p = 2^32 the (cos, sin)
+// pairs are within 1e-7 of exact (checked against 200-bit arithmetic); a
+// double-precision product p * theta^(-2i/d) would be off by p * 2^-53 rad.
+// `turns` holds F_lane and F_(lane+32) (0 past d/2), loaded from the kernel
+// parameters before the grid dependency wait.
 template <int D>
-__device__ __forceinline__ void rope_pairs(const AttnParams& p, long long pos, int lane,
+__device__ __forceinline__ void rope_pairs(const AttnParams& p, long long pos,
+                                           const unsigned long long (&turns)[2], int lane,
                                            float2 (&cs)[2]) {
-  constexpr double kTwoPiHi = 6.283185307179586;      // 2 pi rounded to double
-  constexpr double kTwoPiLo = 2.4492935982947064e-16;  // 2 pi - kTwoPiHi
-  constexpr double kInvTwoPi = 0.15915494309189535;
-  const double pp = static_cast<double>(p.rope_offset + pos);
+  const unsigned long long pp = static_cast<unsigned long long>(p.rope_offset + pos);
 #pragma unroll
   for (int e = 0; e < 2; ++e) {
     const int i = lane + 32 * e;
     cs[e] = make_float2(1.f, 0.f);
     if (i < D / 2) {
-      const double a = pp * p.rope_inv_freq[i];
-      const double n = rint(a * kInvTwoPi);
-      const double r = fma(-n, kTwoPiLo, fma(-n, kTwoPiHi, a));
+      const unsigned long long frac = pp * turns[e];  // mod 2^64: the fractional turn
+      const int hi = static_cast<int>(static_cast<long long>(frac) >> 32);  // [-2^31, 2^31)
+      // angle / pi = 2 * turn in [-1, 1)
+      const float x = static_cast<float>(hi) * 4.656612873077393e-10f;  // 2^-31
       float sn, cn;
-      sincosf(static_cast<float>(r), &sn, &cn);
+      sincospif(x, &sn, &cn);
       cs[e] = make_float2(cn, sn);
     }
   }
@@ -732,6 +739,11 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     SeqState sq;
     sq.pos = 0; sq.count = 0; sq.new_slot = -1; sq.bad = true;
     float2 rope[2] = {make_float2(1.f, 0.f), make_float2(1.f, 0.f)};
+    unsigned long long turns[2] = {0ull, 0ull};  // this lane's rotary frequencies (ROPE)
+    if (ROPE) {
+      turns[0] = p.rope_turns[lane];
+      if (lane + 32 < D / 2) turns[1] = p.rope_turns[lane + 32];
+    }
     for (int i = 0; i < n_tiles; ++i) {
       const int s = i % NST;
       if (i >= NST) {
@@ -757,7 +769,7 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
         run_b = ci.b;
         run_tiles = 0;
         sq = seq_state<FUSED>(p, meta.pos);
-        if (ROPE && !sq.bad) rope_pairs<D>(p, meta.pos, lane, rope);
+        if (ROPE && !sq.bad) rope_pairs<D>(p, meta.pos, turns, lane, rope);
       }
       ++run_tiles;
       finish_tile<D, G, FUSED, ROPE>(p, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, meta, sq,
@@ -1462,6 +1474,14 @@ static int dispatch_attn(const AttnMaps& maps, const AttnParams& p, int d, int G
   }
 }
 
+// theta^(-2i/d) / (2 pi) -- the pair's turns per position, below 1/6 -- as a
+// 64-bit binary fraction, rounded to nearest, computed in long double.
+static unsigned long long rope_turns_fixed(double theta, int i, int d) {
+  const long double two_pi = 6.283185307179586476925286766559L;
+  const long double t = powl(static_cast<long double>(theta), -2.0L * i / d) / two_pi;
+  return static_cast<unsigned long long>(t * 18446744073709551616.0L + 0.5L);  // t * 2^64
+}
+
 static int run_attention(const void* q, const void* tier1_k, const void* tier1_v,
                          const int32_t* idx, void* ring_k, void* ring_v, int64_t* pos,
                          const void* k_new, const void* v_new, const cmc_dims* dims, float scale,
@@ -1530,7 +1550,7 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   p.rope_offset = rope ? rope_offset : 0;
   p.l2_prefetch = kL2PrefetchTiles;
   for (int i = 0; i < 64; ++i)
-    p.rope_inv_freq[i] = (rope && i < m.d / 2) ? pow(rope_theta, -2.0 * i / m.d) : 0.0;
+    p.rope_turns[i] = (rope && i < m.d / 2) ? rope_turns_fixed(rope_theta, i, m.d) : 0ull;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int G = m.Hq / m.Hkv;
   if (rope) return dispatch_attn<true, true>(maps, p, m.d, G, tiles, s);
