@@ -1,0 +1,40 @@
+"""The algorithmic bytes and flops bench.py divides by, checked against the
+cost model written out by hand for the Llama-3-8B-shaped step (32 layers,
+32 query / 8 KV heads, head_dim 128, k = 128 selected rows, W = 512 window)
+and the paper's MACs per generated token (appendix, Attention MACs
+Analysis: MACs_t = 2 n_h d_h n_l L_t, two flops per MAC)."""
+
+import bench
+
+
+def test_decode_step_bytes_llama_shape():
+    B, L, Hq, Hkv, d, k, W = 1, 32, 32, 8, 128, 128, 512
+    row = d * 2  # one bf16 K or V row
+    units = B * L * Hkv
+    kv_read = units * 2 * row * (k + W - 1)   # k Tier-1 rows and W - 1 old ring rows, K and V
+    new_tok = units * 2 * row * 2             # the new token's K,V read once and written once
+    q_out = B * L * Hq * d * 2 * 2            # q read, out written
+    assert bench.decode_step_bytes(B, L, Hq, Hkv, d, k, W) == kv_read + new_tok + q_out
+    assert bench.decode_step_bytes(B, L, Hq, Hkv, d, k, W) == 84_541_440
+    # idx read as well when the step gathers the Tier-1 rows itself
+    assert bench.decode_step_bytes(B, L, Hq, Hkv, d, k, W, gather=True) == 84_541_440 + 4 * k
+
+
+def test_decode_step_flops_are_twice_the_papers_macs():
+    B, L, Hq, d, k, W = 1, 32, 32, 128, 128, 512
+    macs_per_token = 2 * Hq * d * L * (k + W)  # MACs_t with L_t = k + W cached keys
+    assert bench.decode_step_flops(B, L, Hq, d, k, W) == 2 * macs_per_token == 335_544_320
+
+
+def test_select_and_gather_bytes():
+    # one bank of 1,024 CMEs of dimension 4,096 (fp32) read once, q_vec read,
+    # k indices written
+    assert bench.select_bytes(1, 1024, 4096, 128) == 4 * 1024 * 4096 + 4 * 4096 + 4 * 128
+    # the selected K and V rows of every (layer, KV head) read and written,
+    # idx read
+    assert bench.tier1_gather_bytes(1, 32, 8, 128, 128) == 2 * 2 * 32 * 8 * 128 * 128 * 2 + 4 * 128
+
+
+def test_job_value_counts_every_rank():
+    # tokens/s of the whole job: N ranks x steps x requests x batch x decode steps / time
+    assert bench.job_tokens_per_s(2, 10, 4, 1, 3000, 1000.0) == 2 * 10 * 4 * 1 * 3000 / 1.0
