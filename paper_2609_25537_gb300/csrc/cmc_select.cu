@@ -8,7 +8,8 @@
 //     partial sums meet in a fixed tree (warp shuffles, then the eight warps
 //     in order), so equal rows produce bit-identical scores.  HBM-bound:
 //     4*D bytes per row, with a whole row per CTA in flight.
-//  2. topk_select_kernel -- one CTA per sequence.  Scores are mapped to
+//  2. topk_select_kernel -- one CTA per sequence (above 8,192 CMEs,
+//     topk_select_cluster_kernel: a cluster of 8, see there).  Scores are mapped to
 //     order-preserving uint32 keys; a 4-pass MSB radix select (8 bits a pass)
 //     finds the key T of the k-th largest score and how many of the keys equal
 //     to T are needed; an ordered compaction then writes the selected indices
@@ -333,6 +334,174 @@ topk_select_kernel(const float* __restrict__ scores, int N, int k, int32_t* __re
   }
 }
 
+// --- thread-block cluster helpers (barrier over every thread of the
+// cluster; loads from a peer CTA's shared memory).
+__device__ __forceinline__ void sel_cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\n" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire;\n" ::: "memory");
+}
+__device__ __forceinline__ uint32_t sel_cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t sel_ld_peer(const uint32_t* local, uint32_t rank) {
+  uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(local)), r, v;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(a), "r"(rank));
+  asm volatile("ld.shared::cluster.u32 %0, [%1];\n" : "=r"(v) : "r"(r) : "memory");
+  return v;
+}
+
+// Banks of more than kSelectWideN CMEs: one cluster of kSelectClusterCtas
+// CTAs per sequence, CTA r holding the keys of indices [r N / 8, (r+1) N / 8)
+// in its shared memory.  Each radix pass builds the CTA's histogram, and after
+// a cluster barrier every CTA adds the eight histograms (distributed shared
+// memory, rank order) and takes the same decision; the histograms are
+// double-buffered by pass parity.  The compaction counts each CTA's keys above
+// and equal to T, combines the counts across the cluster (exclusive sums over
+// the ranks) to place the keys equal to T in global index order and each
+// CTA's outputs, then writes.  Every thread of the cluster passes the same
+// seven cluster barriers.
+constexpr int kSelectClusterCtas = 8;
+
+__global__ void __launch_bounds__(kSelectThreadsMax)
+topk_select_cluster_kernel(const float* __restrict__ scores, int N, int k,
+                           int32_t* __restrict__ idx_out, const LocateArgs la) {
+  constexpr int NT = kSelectThreadsMax;
+  constexpr int CS = kSelectClusterCtas;
+  extern __shared__ uint32_t skeys[];
+  __shared__ uint32_t hist[2][256];
+  __shared__ uint32_t wsum[3][NT / 32];
+  __shared__ uint32_t pub[2];  // this CTA's keys equal to T, and its selected keys
+  __shared__ uint32_t sh_prefix, sh_krem;
+  const int b = blockIdx.x / CS;
+  const uint32_t rank = sel_cluster_rank();
+  const int tid = threadIdx.x;
+  const int lane = tid & 31, warp = tid >> 5;
+  pdl_wait();  // the scores of the kernel before
+  pdl_trigger();
+  if (la.sqnorm && rank == 0) locate_window(la, b, N);
+  const float* s = scores + static_cast<long long>(b) * N;
+  int32_t* out = idx_out + static_cast<long long>(b) * k;
+  if (k <= 0) return;  // the same for every CTA of the cluster
+  if (k >= N) {
+    if (rank == 0)
+      for (int j = tid; j < N; j += NT) out[j] = j;
+    return;
+  }
+  const int jb = static_cast<int>((static_cast<long long>(rank) * N) / CS);  // this CTA's first key
+  const int n = static_cast<int>((static_cast<long long>(rank + 1) * N) / CS) - jb;
+  for (int j = tid; j < 2 * 256; j += NT) hist[j >> 8][j & 255] = 0u;
+  for (int j = tid; j < n; j += NT) skeys[j + (j >> 5)] = orderable(s[jb + j]);
+  __syncthreads();
+  auto key_at = [&](int j) -> uint32_t { return skeys[j + (j >> 5)]; };
+
+  uint32_t prefix = 0u, mask = 0u, krem = static_cast<uint32_t>(k);
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    uint32_t* h = hist[pass & 1];
+    for (int base = 0; base < n; base += NT) {
+      const int j = base + tid;
+      const uint32_t key = j < n ? key_at(j) : 0u;
+      const bool part = j < n && (key & mask) == prefix;
+      const uint32_t bin = part ? ((key >> shift) & 255u) : 0xFFFFFFFFu;
+      const uint32_t peers = __match_any_sync(0xffffffffu, bin);
+      if (part && lane == __ffs(peers) - 1) atomicAdd(&h[bin], __popc(peers));
+    }
+    sel_cluster_sync();  // every CTA's histogram of this pass is complete
+    uint32_t c = 0u, inc = 0u;
+    if (tid < 256) {
+      for (int r = 0; r < CS; ++r) c += sel_ld_peer(&h[255 - tid], static_cast<uint32_t>(r));
+      inc = c;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xffffffffu, inc, off);
+        if (lane >= off) inc += t;
+      }
+      if (lane == 31) wsum[0][warp] = inc;
+      // the other buffer was read by every peer before this pass's barrier
+      hist[(pass + 1) & 1][tid] = 0u;
+    }
+    __syncthreads();
+    if (tid < 256) {
+      for (int w = 0; w < warp; ++w) inc += wsum[0][w];
+      const uint32_t excl = inc - c;
+      if (excl < krem && inc >= krem) {
+        sh_prefix = prefix | (static_cast<uint32_t>(255 - tid) << shift);
+        sh_krem = krem - excl;
+      }
+    }
+    __syncthreads();
+    prefix = sh_prefix;
+    krem = sh_krem;
+    mask |= 0xFFu << shift;
+  }
+
+  // This CTA's keys above T and equal to T; then, across the cluster, the
+  // keys equal to T before this CTA (they rank first among the equal keys)
+  // and the selected keys before this CTA (its first output slot).
+  const uint32_t T = prefix;
+  uint32_t n_gt = 0u, n_eq = 0u;
+  for (int j = tid; j < n; j += NT) {
+    const uint32_t key = key_at(j);
+    n_gt += key > T ? 1u : 0u;
+    n_eq += key == T ? 1u : 0u;
+  }
+  uint32_t gt_total, eq_total;
+  block_exclusive_sum<NT>(n_gt, wsum[1], &gt_total);
+  block_exclusive_sum<NT>(n_eq, wsum[2], &eq_total);
+  if (tid == 0) pub[0] = eq_total;
+  sel_cluster_sync();
+  uint32_t eq_before = 0u;
+  for (int r = 0; r < static_cast<int>(rank); ++r) eq_before += sel_ld_peer(&pub[0], static_cast<uint32_t>(r));
+  const uint32_t eq_take = krem > eq_before ? min(krem - eq_before, eq_total) : 0u;
+  if (tid == 0) pub[1] = gt_total + eq_take;
+  sel_cluster_sync();
+  uint32_t sel_before = 0u;
+  for (int r = 0; r < static_cast<int>(rank); ++r) sel_before += sel_ld_peer(&pub[1], static_cast<uint32_t>(r));
+  __syncthreads();  // wsum is reused below
+
+  // Ordered compaction of this CTA's keys, as in topk_select_kernel, with
+  // the running counts starting from the cluster-wide offsets.
+  const int per = (n + NT - 1) / NT;
+  const int C = per < 32 ? per : 32;
+  const int chunk = C * NT;
+  uint32_t run_eq = eq_before, run_sel = sel_before;
+  for (int base = 0; base < n; base += chunk) {
+    const int j0 = base + tid * C;
+    uint32_t m_eq = 0u;
+    for (int e = 0; e < C; ++e) {
+      const int j = j0 + e;
+      if (j < n && key_at(j) == T) ++m_eq;
+    }
+    uint32_t eqc, selc;
+    const uint32_t eq0 = run_eq + block_exclusive_sum<NT>(m_eq, wsum[1], &eqc);
+    uint32_t m_sel = 0u, r = eq0;
+    for (int e = 0; e < C; ++e) {
+      const int j = j0 + e;
+      if (j < n) {
+        const uint32_t key = key_at(j);
+        if (key > T) ++m_sel;
+        else if (key == T) m_sel += (r++ < krem) ? 1u : 0u;
+      }
+    }
+    uint32_t slot = run_sel + block_exclusive_sum<NT>(m_sel, wsum[2], &selc);
+    r = eq0;
+    for (int e = 0; e < C; ++e) {
+      const int j = j0 + e;
+      if (j < n) {
+        const uint32_t key = key_at(j);
+        const bool sel = key > T || (key == T && r++ < krem);
+        if (sel && slot < static_cast<uint32_t>(k)) out[slot++] = jb + j;
+      }
+    }
+    run_eq += eqc;
+    run_sel += selc;
+    __syncthreads();
+  }
+  sel_cluster_sync();  // the published counts stay readable until every CTA is done
+}
+
 // The two selection kernels, scores written to `sc` (device, B * N floats);
 // with la.sqnorm set, the squared norms too and the localisation runs in the
 // selection kernel.
@@ -359,11 +528,33 @@ static int launch_score_select(const float* question_emb, const float* cme_bank,
       if (st == CMC_OK)
         st = record_cuda_error(cudaFuncSetAttribute(topk_select_kernel<kSelectThreadsMax>,
                                                     cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+      if (st == CMC_OK)
+        st = record_cuda_error(cudaFuncSetAttribute(topk_select_cluster_kernel,
+                                                    cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
     });
     if (st != CMC_OK) return st;
   }
   const size_t smem =
       (N <= kSelectSmemKeys && k > 0 && k < N) ? select_smem_words(N) * sizeof(uint32_t) : 0;
+  const int per_cta = (N + kSelectClusterCtas - 1) / kSelectClusterCtas;
+  if (N > kSelectWideN && k > 0 && k < N && per_cta <= kSelectSmemKeys) {
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = kSelectClusterCtas;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(B) * kSelectClusterCtas);
+    cfg.blockDim = dim3(kSelectThreadsMax);
+    cfg.dynamicSmemBytes = select_smem_words(per_cta) * sizeof(uint32_t);
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return record_cuda_error(cudaLaunchKernelEx(&cfg, topk_select_cluster_kernel,
+                                                static_cast<const float*>(sc), N, k, idx_out, la));
+  }
   if (N > kSelectWideN)
     return launch_pdl(topk_select_kernel<kSelectThreadsMax>, dim3(B), dim3(kSelectThreadsMax), smem, s,
                       static_cast<const float*>(sc), N, k, idx_out, la);

@@ -78,11 +78,12 @@ def test_select_ties_go_to_lower_index(cuda_device):
     np.testing.assert_array_equal(idx, ref_idx)
 
 
-# the last two: the 1,024-thread selection CTA with keys in shared memory
-# (N > 8,192), and keys re-read from the scores in global memory (N > 49,152)
+# the last three: a cluster of 8 selection CTAs per sequence (N > 8,192),
+# keys split across their shared memories (also unevenly: 50,001 = 8 x 6,250
+# + 1), and one CTA re-reading the keys from global memory (N / 8 > 49,152)
 @pytest.mark.parametrize("N,D,k", [(1, 4, 1), (1, 4, 0), (5, 8, 5), (1000, 36, 999),
                                    (1025, 512, 17), (3000, 4, 1500), (4096, 128, 4095),
-                                   (9000, 8, 1234), (50001, 4, 777)])
+                                   (9000, 8, 1234), (50001, 4, 777), (400003, 4, 1000)])
 def test_select_edge_shapes(cuda_device, N, D, k):
     rng = np.random.default_rng(N + D + k)
     B = 3
