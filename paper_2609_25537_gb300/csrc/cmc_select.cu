@@ -108,32 +108,49 @@ cosine_scores_kernel(const float* __restrict__ qv, const float* __restrict__ ban
 }
 
 // q_vec[b] = mean of the first q_len[b] question-token embeddings (Section
-// 2.5, Tier-1): one thread per 4 columns sums the tokens in order and divides
-// by the count; an empty question gives the zero vector.
+// 2.5, Tier-1); an empty question gives the zero vector.  A CTA covers 32
+// four-column groups: lane c of warp s sums the tokens s, s + 8, s + 16, ...
+// of its group (so every warp reads whole 512-byte row segments, and all of a
+// question's rows are in flight at once), then the eight partial sums of a
+// group are added in warp order and divided by the count.
 constexpr int kPoolThreads = 256;
+constexpr int kPoolSlices = kPoolThreads / 32;  // token slices (warps) per CTA
 
 __global__ void __launch_bounds__(kPoolThreads)
 question_pool_kernel(const float* __restrict__ tokens, const int32_t* __restrict__ q_len, int Lq,
                      int D, float* __restrict__ q_vec) {
+  __shared__ float4 part[kPoolSlices][32];
   pdl_wait();
   pdl_trigger();
   const int b = blockIdx.y;
-  const int c4 = blockIdx.x * kPoolThreads + threadIdx.x;
+  const int lane = threadIdx.x & 31, sl = threadIdx.x >> 5;
+  const int c4 = blockIdx.x * 32 + lane;
   const int D4 = D >> 2;
-  if (c4 >= D4) return;
   int n = q_len ? q_len[b] : Lq;
   n = n < 0 ? 0 : (n > Lq ? Lq : n);
-  const float4* t = reinterpret_cast<const float4*>(tokens + static_cast<long long>(b) * Lq * D) + c4;
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int i = 0; i < n; ++i) {
-    const float4 v = __ldg(t + static_cast<long long>(i) * D4);
-    acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+  if (c4 < D4) {
+    const float4* t = reinterpret_cast<const float4*>(tokens + static_cast<long long>(b) * Lq * D) + c4;
+    for (int i = sl; i < n; i += kPoolSlices) {
+      const float4 v = __ldg(t + static_cast<long long>(i) * D4);
+      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    }
   }
-  if (n > 0) {
-    const float fn = static_cast<float>(n);
-    acc.x /= fn; acc.y /= fn; acc.z /= fn; acc.w /= fn;
+  part[sl][lane] = acc;
+  __syncthreads();
+  if (sl == 0 && c4 < D4) {
+    float4 tot = part[0][lane];
+#pragma unroll
+    for (int w = 1; w < kPoolSlices; ++w) {
+      const float4 v = part[w][lane];
+      tot.x += v.x; tot.y += v.y; tot.z += v.z; tot.w += v.w;
+    }
+    if (n > 0) {
+      const float fn = static_cast<float>(n);
+      tot.x /= fn; tot.y /= fn; tot.z /= fn; tot.w /= fn;
+    }
+    reinterpret_cast<float4*>(q_vec + static_cast<long long>(b) * D)[c4] = tot;
   }
-  reinterpret_cast<float4*>(q_vec + static_cast<long long>(b) * D)[c4] = acc;
 }
 
 // Exclusive prefix sum of one value per thread over the block (NT threads,
@@ -628,7 +645,7 @@ int cmc_question_select(const float* question_tokens, const int32_t* q_len, int 
   float* sq = sc + align_up(static_cast<size_t>(B) * N * sizeof(float), 256) / sizeof(float);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int D4 = D / 4;
-  int st = launch_pdl(question_pool_kernel, dim3((D4 + kPoolThreads - 1) / kPoolThreads, B),
+  int st = launch_pdl(question_pool_kernel, dim3((D4 + 31) / 32, B),
                       dim3(kPoolThreads), 0, s, question_tokens, q_len, Lq, D, q_vec_out);
   if (st != CMC_OK) return st;
   LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out};
