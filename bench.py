@@ -47,13 +47,13 @@ import hashlib
 import json
 import math
 import os
-import re
 import statistics
 import subprocess
 import sys
 import time
 
-# The CPU oracle legs run single-threaded and say so.
+# The CPU oracle legs use one BLAS thread per process (the multi-core legs run
+# one process per core) and say so.
 for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
     os.environ.setdefault(_v, "1")
 
@@ -69,7 +69,8 @@ from workloads import (WORKLOADS, context_inputs, kv_inputs, question_inputs,  #
 METRIC = ("two-tier decode-attn tokens/s and % of 8 TB/s HBM; CME top-k select µs")
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
-PROFILE_FILE = os.path.join(ROOT, "profiles", "decode_step_llama3_8b.md")
+# machine-readable companion of profiles/decode_step_llama3_8b.md
+PROFILE_FILE = os.path.join(ROOT, "profiles", "decode_step_llama3_8b.json")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2609_25537_gb300", "csrc", f)
                   for f in ("cmc_attn.cu", "cmc_internal.cuh")]
 
@@ -124,20 +125,18 @@ def kernel_source_hash() -> str:
 
 def profiled_traffic(workload: str, tier1: str):
     """DRAM bytes per launch of the fused decode kernel from the committed ncu
-    summary, if it was taken on the current kernel source, for this workload
+    record, if it was taken on the current kernel source, for this workload
     and Tier-1 form; else None."""
     try:
-        txt = open(PROFILE_FILE).read()
-    except OSError:
+        with open(PROFILE_FILE) as f:
+            rec = json.load(f)
+        if rec["kernel_source_sha256"] != kernel_source_hash():
+            return None
+        if (rec["workload"], rec["tier1"]) != (workload, tier1):
+            return None
+        return int(rec["dram_bytes_per_launch"])
+    except (OSError, ValueError, KeyError, TypeError):
         return None
-    m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", txt)
-    h = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", txt)
-    c = re.search(r"profiled_config:\s*(\S+)\s+(\S+)", txt)
-    if not m or not h or not c or h.group(1) != kernel_source_hash():
-        return None
-    if (c.group(1), c.group(2)) != (workload, tier1):
-        return None
-    return int(m.group(1))
 
 
 # ----------------------------------------------------------------------------
@@ -263,6 +262,42 @@ def oracle_sample(w, host_state, seconds: float, min_steps: int = 1):
     return steps * w.B / el, steps, el
 
 
+def step_pool(w, n: int = 8):
+    """The first n decode steps' inputs, cycled by the multi-core oracle leg
+    (the GPU arm cycles a pool of the same size)."""
+    sts = [step_inputs(w, t) for t in range(n)]
+    return [s.q for s in sts], [s.k_new for s in sts], [s.v_new for s in sts]
+
+
+def oracle_sample_parallel(w, host_state, seconds: float, step_seconds: float, pool=None):
+    """Times the unchanged oracle on all host cores: one Tier-1 selection
+    (one process), then decode steps run as disjoint slices of the problem
+    (layers, or sequences) in a pool of spawned processes side by side, sized
+    to take about `seconds` given the single-thread step time.  Returns
+    (decode tokens/s, steps, elapsed, worker processes, slices)."""
+    import oracle
+    from oracle.host_pool import HostPool, host_cores
+    qemb, bank, t1k, t1v, ring_k, ring_v, pos = host_state
+    cores = host_cores()
+    n_units = w.B if (w.B >= cores or w.L == 1) else w.L
+    workers = max(1, min(cores, n_units))
+    own = pool is None
+    if own:
+        pool = HostPool(workers)
+    try:
+        qs, ks, vs = step_pool(w)
+        n_steps = max(2, int(seconds * workers / max(step_seconds, 1e-6)))
+        t0 = time.perf_counter()
+        idx, _ = oracle.score_select(qemb, bank, w.k)
+        t_sel = time.perf_counter() - t0
+        el, n_slices = pool.decode_steps(t1k, t1v, idx, ring_k, ring_v, pos, qs, ks, vs, n_steps)
+    finally:
+        if own:
+            pool.close()
+    total = t_sel + el
+    return n_steps * w.B / total, n_steps, total, pool.workers, n_slices
+
+
 def host_state_for(w):
     si = selection_inputs(w)
     kv = kv_inputs(w)
@@ -271,30 +306,44 @@ def host_state_for(w):
 
 
 def run_reference(args, w, world, rank):
-    """The reference arm: the fp64 oracle on the host cores, rank 0 only."""
+    """The reference arm: the fp64 oracle on all host cores, rank 0 only.
+    Each step is one Tier-1 selection plus ~ref_step_seconds of decode steps,
+    the problem's layers (or sequences) split over a pool of spawned worker
+    processes; a step's time is the selection's plus the slowest worker's."""
     if rank != 0:
         return 0
+    from oracle.host_pool import HostPool, host_cores
     state = host_state_for(w)
     per_step = args.ref_step_seconds
-    for _ in range(args.warmup):
-        oracle_sample(w, state, 0.0, min_steps=1)
-    t0 = time.perf_counter()
-    tokens = 0
-    for _ in range(args.steps):
-        tps, steps, el = oracle_sample(w, state, per_step, min_steps=1)
-        tokens += steps * w.B
-    elapsed = time.perf_counter() - t0
+    # single-thread step time, to size each step's sample
+    _, n1, el1 = oracle_sample(w, state, 0.0, min_steps=2)
+    step_s = el1 / n1
+    cores = host_cores()
+    n_units = w.B if (w.B >= cores or w.L == 1) else w.L
+    pool = HostPool(max(1, min(cores, n_units)))
+    try:
+        for _ in range(args.warmup):
+            oracle_sample_parallel(w, state, 0.0, step_s, pool=pool)
+        tokens, elapsed = 0, 0.0
+        for _ in range(args.steps):
+            _, steps, el, workers, n_slices = oracle_sample_parallel(w, state, per_step, step_s,
+                                                                     pool=pool)
+            tokens += steps * w.B
+            elapsed += el
+    finally:
+        pool.close()
     value = tokens / elapsed
     sample = (f"per step: one Tier-1 selection + ~{per_step:g}s of fused decode steps "
-              f"(all {w.L} layers) of {w.name}; fp64 numpy, 1 thread")
+              f"(all {w.L} layers) of {w.name}, split into {n_slices} slices over {workers} "
+              f"worker processes; fp64 numpy, 1 BLAS thread each; host has {cores} cores")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1000.0 * elapsed / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(w, args.requests),
-        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": workers,
+                         "host_cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -598,10 +647,19 @@ def run_gpu(args, w, world, rank, local):
     # CPU oracle baseline (rank 0, N = 1)
     cpu = None
     if want_cpu:
-        tps, steps, el = oracle_sample(w, cpu_state, args.cpu_seconds)
-        cpu = {"value": tps, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+        from oracle.host_pool import host_cores
+        tps1, steps1, el1 = oracle_sample(w, cpu_state, args.cpu_seconds)
+        tps, steps, el, workers, n_slices = oracle_sample_parallel(
+            w, cpu_state, args.cpu_seconds, el1 / steps1)
+        cpu = {"value": tps, "unit": "tokens/s", "cores": workers, "host_cores": host_cores(),
+               "kind": "oracle",
                "sample": (f"one Tier-1 selection + {steps} fused decode steps (all {w.L} "
-                          f"layers) of {w.name} in {el:.1f}s; fp64 numpy, 1 thread")}
+                          f"layers) of {w.name} in {el:.1f}s, the step split into {n_slices} "
+                          f"slices run side by side in {workers} spawned worker processes "
+                          "(fp64 numpy, 1 BLAS thread each)"),
+               "single_thread": {"value": tps1, "unit": "tokens/s", "cores": 1,
+                                 "sample": (f"one Tier-1 selection + {steps1} fused decode "
+                                            f"steps in {el1:.1f}s, one process")}}
 
     if rank != 0:
         return 0

@@ -60,8 +60,9 @@ typedef enum cmc_status {
  * cmc_read_status).  Kernels skip the offending element and carry on. */
 #define CMC_DEVFLAG_BAD_INDEX 1u /* an idx entry outside [0, N): that row was skipped   */
 #define CMC_DEVFLAG_BAD_POS 2u   /* a negative pos: that sequence was skipped            */
-#define CMC_DEVFLAG_TIMEOUT 4u   /* a pipeline wait hit its iteration limit: the call's
-                                    outputs are invalid (never expected in operation)     */
+#define CMC_DEVFLAG_TIMEOUT 4u   /* a pipeline wait gave up after its time limit (1 s of
+                                    %globaltimer): the call's outputs and ring update are
+                                    invalid (never expected in operation)                 */
 
 /* Shapes of one decode problem. */
 typedef struct cmc_dims {
@@ -337,11 +338,21 @@ CMC_API int cmc_decode_attn_plan(const cmc_dims* dims, int fused, int* ctas, int
  * the prefill input [M* | C_local | q]).  The kernel rotates every query head
  * and the new key at p, appends the rotated key (bf16, round to nearest even)
  * and the value to the ring, and attends with the rotated query over
- * [Tier-1 | Tier-2] exactly as cmc_decode_step.  Angles are formed in double
- * precision.  Other arguments are those of cmc_decode_step.
+ * [Tier-1 | Tier-2] exactly as cmc_decode_step.  Other arguments are those of
+ * cmc_decode_step.
+ *
+ * Angles.  The host turns each pair's frequency rope_theta^(-2i/d) / (2 pi)
+ * into a 64-bit binary fraction F_i (turns per position, rounded to
+ * nearest).  The kernel forms p * F_i mod 2^64 in integer arithmetic -- the
+ * angle's fractional turn, exact but for the rounding of F_i, so off by at
+ * most p * 2^-65 turns -- and passes its top 32 bits, as a signed fraction of
+ * a half turn, to sincospif.  The angle error is thus below
+ * 2 pi (p * 2^-65 + 2^-32) rad plus sincospif's, and (cos, sin) are within
+ * about 1e-7 of exact for p up to 2^33; from there the first term grows as
+ * p * 1.7e-19 rad.
  *
  * Errors: as cmc_decode_step; rope_theta must be positive and finite and
- * 0 <= rope_offset <= 2^53 (else CMC_ERR_RANGE).
+ * 0 <= rope_offset <= 2^32 (else CMC_ERR_RANGE).
  */
 CMC_API int cmc_decode_step_rope(const void* q, const void* tier1_k, const void* tier1_v,
                                  const int32_t* idx, void* ring_k, void* ring_v, int64_t* pos,

@@ -22,7 +22,6 @@ made once per question by :func:`tier1_gather` is passed.
 from __future__ import annotations
 
 import ctypes
-import math
 from typing import Dict, Optional, Tuple
 
 import torch
@@ -408,7 +407,3 @@ def window_append(ring_k: torch.Tensor, ring_v: torch.Tensor, pos: torch.Tensor,
     st = lib().cmc_window_append(_p(ring_k), _p(ring_v), _p(pos), _p(k_new), _p(v_new),
                                  ctypes.byref(dims), _stream(dev))
     check(st, "cmc_window_append")
-
-
-def default_scale(d: int) -> float:
-    return 1.0 / math.sqrt(d)

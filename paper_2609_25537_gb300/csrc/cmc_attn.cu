@@ -38,7 +38,7 @@
 // an online softmax in the log2 domain (running max / sum per head), and
 //   O += P V    with mma.sync, P taken straight from the S accumulators,
 // reading K with ldmatrix and V with ldmatrix.trans, then hand the stage back
-// through an "empty" mbarrier.  Every mbarrier wait has an iteration limit.
+// through an "empty" mbarrier.  Every mbarrier wait has a wall-time limit.
 // Warps are merged in shared memory at the end of a unit.
 //
 // K/V rows are read once per launch, so their loads carry an L2 evict-first
@@ -162,10 +162,25 @@ __device__ __forceinline__ uint32_t pack_bf16_rn(float lo, float hi) {
   return r;
 }
 
-// --- mbarrier (shared::cta).  Every wait is bounded: after kMaxWaitSpins
-// failed polls the waiter reports CMC_DEVFLAG_TIMEOUT and gives up, so a
-// broken pipeline cannot hang the GPU.
-constexpr uint32_t kMaxWaitSpins = 1u << 22;
+// --- mbarrier (shared::cta).  Every wait is bounded in wall time: a waiter
+// that has not seen its phase complete kWaitNs after it started polling
+// (%globaltimer, nanoseconds) raises the CTA's abort flag, reports
+// CMC_DEVFLAG_TIMEOUT and gives up; once the flag is up every other wait of
+// the CTA gives up at its next poll.  A poll-count cap backs the deadline up
+// in case the timer ever stood still.  Named-barrier and cluster-barrier
+// participation never depends on whether a wait succeeded (see the kernel),
+// so a CTA whose waits gave up still reaches its end.
+constexpr uint32_t kWaitNs = 1000000000u;  // 1 s: the kernel runs for microseconds
+constexpr uint32_t kDrainNs = 2000000u;    // after a timeout: wait for issued loads
+constexpr uint32_t kMaxWaitPolls = 1u << 28;
+
+// Low 32 bits of %globaltimer (nanoseconds).  Differences of readings less
+// than 2^32 ns (4.29 s) apart are exact in unsigned 32-bit arithmetic.
+__device__ __forceinline__ uint32_t global_ns32() {
+  uint32_t t;
+  asm volatile("mov.u32 %0, %%globaltimer_lo;\n" : "=r"(t));
+  return t;
+}
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(smem_addr(bar)), "r"(count));
@@ -192,11 +207,25 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Waits for the phase of `bar` with the given parity to complete; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  for (uint32_t it = 0; it < kMaxWaitSpins; ++it)
+// The CTA's abort flag: raised by the first wait that times out.
+__shared__ int attn_abort;
+
+__device__ __forceinline__ bool attn_aborted() { return *static_cast<volatile int*>(&attn_abort) != 0; }
+
+// Waits for the phase of `bar` with the given parity to complete.  False when
+// the CTA's abort flag is (or goes) up, or on timeout, which raises it.
+__device__ __forceinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity) {
+  const uint32_t t0 = global_ns32();
+  for (uint32_t it = 0; it < kMaxWaitPolls; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
+    if (attn_aborted()) return false;
+    if (global_ns32() - t0 > kWaitNs) break;
+  }
+  *static_cast<volatile int*>(&attn_abort) = 1;
   return false;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity);
 }
 
 // --- TMA loads into shared memory, completing on an mbarrier.
@@ -680,6 +709,7 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
       mbar_init(&full_bar[s], 1);        // the producer's arrive (plus tracked cp.async arrivals)
       mbar_init(&empty_bar[s], kWarps);  // one arrive per consumer warp
     }
+    attn_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
   }
   __syncthreads();
@@ -747,10 +777,14 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     for (int i = 0; i < n_tiles; ++i) {
       const int s = i % NST;
       if (i >= NST) {
-        if (!mbar_wait(&empty_bar[s], static_cast<uint32_t>((i / NST - 1) & 1))) {
-          if (lane == 0) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
-          break;
-        }
+        // Lane 0 waits for the consumers to release the stage; the warp barrier
+        // orders the other lanes' copies into it after that, and the broadcast
+        // makes the whole warp leave together if the wait gave up.
+        int ok = 0;
+        if (lane == 0) ok = mbar_wait(&empty_bar[s], static_cast<uint32_t>((i / NST - 1) & 1)) ? 1 : 0;
+        __syncwarp();
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
         if (lane == 0 && !gathered_tile(p, ci))
           issue_box_loads<D, G>(p, maps, smem + s * S::kBytes, aux0 + s * S::kAuxBytes, ci, &full_bar[s]);
       }
@@ -781,9 +815,21 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
       cm.next(p);
     }
     if (FUSED && run_b >= 0 && issued == n_tiles && lane == 0) seq_run_done(p, run_b, run_tiles, sq);
-    cp_async_wait<0>();
-    // Let this CTA's loads land before the warp exits (bounded).
-    if (issued > 0) mbar_wait(&full_bar[(issued - 1) % NST], static_cast<uint32_t>(((issued - 1) / NST) & 1));
+    cp_async_wait<0>();  // this lane's cp.async copies (metadata, gathered rows) have landed
+    // No CTA exits while bulk loads it issued may still be writing into its
+    // shared memory.  Normally the consumers have waited for every stage but
+    // the last few, and this wait for the last issued stage covers the rest
+    // (a stage's bytes complete its barrier phase).  If waits gave up (abort
+    // flag), barrier phases are no evidence, so the warp stays kDrainNs longer
+    // -- every bulk load was issued before that, and loads of valid addresses
+    // land within microseconds -- with a sleep-count cap behind the timer.
+    if (lane == 0 && issued > 0 &&
+        !mbar_wait(&full_bar[(issued - 1) % NST], static_cast<uint32_t>(((issued - 1) / NST) & 1))) {
+      const uint32_t t0 = global_ns32();
+      for (uint32_t it = 0; it < (1u << 16) && global_ns32() - t0 < kDrainNs; ++it) __nanosleep(1000);
+    }
+    if (lane == 0 && attn_aborted()) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
+    __syncwarp();
     // A cluster plan: the consumers of every CTA of the cluster pass two
     // cluster barriers at the end of their (one) unit; this warp passes the
     // same two, so every thread of the cluster arrives at each.
@@ -800,7 +846,6 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
   TileCursor cc;
   cc.init(t_begin, p);
   int cur_u = -1;
-  bool dead = false;
   uint32_t qa[KS][2];
   float m_run = -INFINITY, l_run = 0.f;
   float o[NT][4];
@@ -813,10 +858,10 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     const int s = i % NST;
     uint8_t* stage = smem + s * S::kBytes;
     const uint8_t* aux = aux0 + s * S::kAuxBytes;
-    if (!dead && !mbar_wait(&full_bar[s], static_cast<uint32_t>((i / NST) & 1))) {
-      dead = true;
-      if (lane == 0) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
-    }
+    // A stage whose wait gave up (this warp's or another's: the CTA's abort
+    // flag) is skipped: no key, no patch.  Barrier participation below does
+    // not depend on it.
+    const bool dead = attn_aborted() || !mbar_wait(&full_bar[s], static_cast<uint32_t>((i / NST) & 1));
     const int* hw = reinterpret_cast<const int*>(aux + S::kHdr);
     const int u = cc.u;
     const int n_rows = dead ? 0 : hw[H_NROWS];
@@ -828,10 +873,11 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
           static_cast<uint32_t>(hw[H_BADLO]));
     bool wrote_stage = false;  // generic-proxy writes into the stage by this warp
 
-    if (FUSED && new_row >= 0) {
+    if (FUSED && new_row >= 0 && (new_row >> 4) == warp) {
       // Patch the new token over its stale ring row (swizzled) and append it
-      // to the ring in global memory.  Warp 0 writes, all consumers wait.
-      if (warp == 0 && lane < 2 * (D / 8)) {
+      // to the ring in global memory.  Each consumer warp reads only its own
+      // 16 rows of K and V, so the warp that owns the row does it alone.
+      if (lane < 2 * (D / 8)) {
         const int which = lane / (D / 8);  // 0: K, 1: V
         const int c = lane - which * (D / 8);
         uint4 v = *reinterpret_cast<const uint4*>(aux + S::kNew + which * D * 2 + c * 16);
@@ -858,8 +904,8 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
         uint16_t* ring = which ? p.ring_v : p.ring_k;
         *reinterpret_cast<uint4*>(ring + (static_cast<long long>(u) * p.W + hw[H_NEWSLOT]) * D + c * 8) = v;
       }
-      consumer_sync();
-      wrote_stage = (warp == 0);
+      __syncwarp();
+      wrote_stage = true;
     }
 
     if (u != cur_u) {  // first tile of a unit in this CTA
@@ -1111,6 +1157,7 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     }
     cc.next(p);
   }
+  if (tid == 0 && attn_aborted()) atomicOr(p.status, CMC_DEVFLAG_TIMEOUT);
 }
 
 // Finishes the units that two_tier_attn_kernel split between CTAs: merges
@@ -1494,7 +1541,7 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   if (!q || !tier1_k || !tier1_v || !ring_k || !ring_v || !pos || !out) return CMC_ERR_NULL;
   if (fused && (!k_new || !v_new)) return CMC_ERR_NULL;
   if (rope && !(rope_theta > 0.0 && rope_theta < 1e300)) return CMC_ERR_RANGE;
-  if (rope && (rope_offset < 0 || rope_offset > (1LL << 53))) return CMC_ERR_RANGE;
+  if (rope && (rope_offset < 0 || rope_offset > (1LL << 32))) return CMC_ERR_RANGE;
   if (!aligned16(q) || !aligned16(tier1_k) || !aligned16(tier1_v) || !aligned16(ring_k) ||
       !aligned16(ring_v) || !aligned16(out))
     return CMC_ERR_ALIGN;

@@ -518,7 +518,8 @@ def test_rope_llama_shape(cuda_device, mode):
 
 
 def test_rope_large_positions_and_peaked_queries(cuda_device):
-    """Positions past 10^5 (long contexts): the angles need double precision."""
+    """Positions past 10^5 (long contexts): angles of 10^5 rad and more, which
+    the kernel reduces to turns with 64-bit integer arithmetic."""
     w = WORKLOADS["tiny"].with_(B=2, T=4, kv_std=0.3)
     _rope_run(w, cuda_device, "dense", theta=10000.0, offset=123457, q_std=3.0 / 0.3)
 
@@ -551,3 +552,127 @@ def test_rope_plan_matches_the_fused_step(cuda_device):
     w = WORKLOADS["llama3_8b"]
     dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.k, w.W)
     assert cmc.decode_attn_plan(dims, rope=True) == cmc.decode_attn_plan(dims)
+
+
+def _rope_append_host(P, st, theta, offset):
+    """The oracle side of a step whose output is not compared: the new key
+    rotated at its position and rounded to bf16, then appended with the value
+    (the first half of oracle.decode_step_rope)."""
+    k_rot = np.empty(st.k_new.shape, dtype=np.uint16)
+    for b in range(P.w.B):
+        p = offset + int(P.o_pos[b])
+        k_rot[b] = oracle.f64_to_bf16_bits(oracle.rope_rotate(st.k_new[b], p, theta))
+    oracle.window_append(P.o_ring_k, P.o_ring_v, P.o_pos, k_rot, st.v_new)
+
+
+def _rope_sampled_run(w, dev, mode, theta, offset, sample_steps):
+    """Every step runs the rotary decode step on the GPU; the outputs of the
+    sampled steps are compared with oracle.decode_step_rope, and the ring and
+    pos after the last step with the oracle's replay of every append."""
+    P = Problem(w, dev, mode=mode)
+    sample_steps = set(sample_steps)
+    q_fill = dev_bf16(step_inputs(w, 0, parts="q").q, dev)
+    for t in range(w.T):
+        if t in sample_steps:
+            st = step_inputs(w, t)
+            q_dev = dev_bf16(st.q, dev)
+        else:
+            st = step_inputs(w, t, parts="kv")
+            q_dev = q_fill
+        out = cmc.decode_step(q_dev, P.t1k, P.t1v, P.idx, P.ring_k, P.ring_v, P.pos,
+                              dev_bf16(st.k_new, dev), dev_bf16(st.v_new, dev), workspace=P.ws,
+                              rope_theta=theta, rope_offset=offset)
+        if t in sample_steps:
+            ref = oracle.decode_step_rope(st.q, P.kv.tier1_k, P.kv.tier1_v, P.idx_host,
+                                          P.o_ring_k, P.o_ring_v, P.o_pos, st.k_new, st.v_new,
+                                          theta=theta, rope_offset=offset)
+            assert_attn_close(to_f64(out), ref, f"{w.name} rope step {t}")
+        else:
+            _rope_append_host(P, st, theta, offset)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(P.pos.cpu().numpy(), P.o_pos)
+    np.testing.assert_array_equal(host_bits(P.ring_v), P.o_ring_v)
+    _ring_close_bf16(host_bits(P.ring_k), P.o_ring_k, f"{w.name} rotated keys")
+    assert P.ws.status() == 0
+
+
+def _two_ctas_per_sm(sms):
+    return cmc.decode_attn_plan(cmc.CmcDims(2 * sms + 1, 1, 4, 1, 128, 64, 64, 64),
+                                rope=True)[0] == 2 * sms
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_rope_llama_full_shape_one_cta_per_unit(cuda_device, mode):
+    """The rotary step at the benchmarked shape: 32 layers, 256 units, one CTA
+    per unit (the plan the bench times), Llama-3's theta = 5e5, through the
+    ring's wrap: W + 2 steps, outputs compared at 0, 1, 2, W-1, W, W+1."""
+    w = WORKLOADS["llama3_8b"]
+    w = w.with_(T=w.W + 2)
+    sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
+    dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.k, w.W)
+    if _two_ctas_per_sm(sms) and 2 * sms >= 256:
+        assert cmc.decode_attn_plan(dims, rope=True) == (256, 1)
+    _rope_sampled_run(w, cuda_device, mode, theta=500000.0, offset=w.k,
+                      sample_steps=[0, 1, 2, w.W - 1, w.W, w.W + 1])
+
+
+def test_rope_whole_units_per_cta_several_sequences(cuda_device):
+    """More units than resident CTAs, whole units per CTA: with one KV head per
+    sequence, a CTA that takes two units takes two sequences, so the producer
+    forms the rotary table of a second position inside one CTA's run."""
+    sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
+    B = 3 * sms
+    w = _cluster_case(B, 1, 1, 64, 128, T=3)
+    w = w.with_(W0=tuple((17 * b) % (w.W + 1) for b in range(B)))
+    dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.N, w.k, w.W)
+    ctas, launches = cmc.decode_attn_plan(dims, rope=True)
+    if _two_ctas_per_sm(sms):
+        # 3 sms units on 2 sms CTAs: half of the CTAs take two whole units
+        assert (ctas, launches) == (2 * sms, 1)
+    P = Problem(w, cuda_device, mode="dense")
+    for t in range(w.T):
+        st = step_inputs(w, t)
+        out = cmc.decode_step(dev_bf16(st.q, cuda_device), P.t1k, P.t1v, P.idx, P.ring_k,
+                              P.ring_v, P.pos, dev_bf16(st.k_new, cuda_device),
+                              dev_bf16(st.v_new, cuda_device), workspace=P.ws,
+                              rope_theta=500000.0, rope_offset=w.k)
+        ref = oracle.decode_step_rope(st.q, P.kv.tier1_k, P.kv.tier1_v, P.idx_host, P.o_ring_k,
+                                      P.o_ring_v, P.o_pos, st.k_new, st.v_new, theta=500000.0,
+                                      rope_offset=w.k)
+        assert_attn_close(to_f64(out), ref, f"whole units rope step {t}")
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(P.pos.cpu().numpy(), P.o_pos)
+    np.testing.assert_array_equal(host_bits(P.ring_v), P.o_ring_v)
+    _ring_close_bf16(host_bits(P.ring_k), P.o_ring_k, "whole units rotated keys")
+    assert P.ws.status() == 0
+
+
+@pytest.mark.parametrize("mode", MODES)
+def test_rope_stream_k_and_combine(cuda_device, mode):
+    """A few units over a multiple of the CTA count: the tiles are split evenly
+    (units cut between CTAs, runs of several sequences per CTA) and the combine
+    kernel merges the cut units -- the rotary step on that plan."""
+    sms = torch.cuda.get_device_properties(cuda_device).multi_processor_count
+    B = 2 * sms + 17
+    w = _cluster_case(B, 1, 2, 64, 128, T=3)
+    dims = cmc.CmcDims(w.B, w.L, w.Hq, w.Hkv, w.d, w.N, w.k, w.W)
+    ctas, launches = cmc.decode_attn_plan(dims, rope=True)
+    if _two_ctas_per_sm(sms):
+        assert (ctas, launches) == (2 * sms, 2)
+    P = Problem(w, cuda_device, mode=mode)
+    theta, offset = 500000.0, 3 * w.k + 5
+    for t in range(w.T):
+        st = step_inputs(w, t)
+        out = cmc.decode_step(dev_bf16(st.q, cuda_device), P.t1k, P.t1v, P.idx, P.ring_k,
+                              P.ring_v, P.pos, dev_bf16(st.k_new, cuda_device),
+                              dev_bf16(st.v_new, cuda_device), workspace=P.ws,
+                              rope_theta=theta, rope_offset=offset)
+        ref = oracle.decode_step_rope(st.q, P.kv.tier1_k, P.kv.tier1_v, P.idx_host, P.o_ring_k,
+                                      P.o_ring_v, P.o_pos, st.k_new, st.v_new, theta=theta,
+                                      rope_offset=offset)
+        assert_attn_close(to_f64(out), ref, f"stream-K rope step {t}")
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(P.pos.cpu().numpy(), P.o_pos)
+    np.testing.assert_array_equal(host_bits(P.ring_v), P.o_ring_v)
+    _ring_close_bf16(host_bits(P.ring_k), P.o_ring_k, "stream-K rotated keys")
+    assert P.ws.status() == 0
