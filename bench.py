@@ -397,7 +397,8 @@ class Request:
         self.t1k_dense = torch.empty((B, L, Hkv, w.k, d), dtype=torch.bfloat16, device=dev)
         self.t1v_dense = torch.empty((B, L, Hkv, w.k, d), dtype=torch.bfloat16, device=dev)
         self.out = torch.empty((B, L, Hq, d), dtype=torch.bfloat16, device=dev)
-        self.sel_ws = torch.empty(cmc.score_select_workspace_size(B, w.N), dtype=torch.uint8,
+        # zero-filled once: the selection's completion counters start at zero
+        self.sel_ws = torch.zeros(cmc.score_select_workspace_size(B, w.N), dtype=torch.uint8,
                                   device=dev)
         self.ws = cmc.DecodeWorkspace(cmc.dims_of(self.out, self.t1k, self.idx, self.ring_k),
                                       dev)
@@ -617,8 +618,8 @@ def run_gpu(args, w, world, rank, local):
         qlen = torch.from_numpy(qi.q_len).to(dev)
         offs = torch.from_numpy(qi.chunk_offset).to(dev)
         clen = torch.from_numpy(qi.ctx_len).to(dev)
-        ws_q = torch.empty(cmc.score_select_workspace_size(w.B, w.N) * 2, dtype=torch.uint8,
-                           device=dev)
+        ws_q = torch.zeros(cmc.lib().cmc_question_select_workspace_size(w.B, w.N),
+                           dtype=torch.uint8, device=dev)
         r0 = reqs[0]
         prologue_us = cold_us(lambda: cmc.question_select(
             tok, r0.bank, w.k, q_len=qlen, chunk_offset=offs, ctx_len=clen, W=w.W, workspace=ws_q))

@@ -144,7 +144,9 @@ CMC_API int cmc_bridge_epilogue(const float* x, const float* gamma, const float*
  * (Section 2.5, the score_j equation and the top-K re-ordering after it)    *
  * ------------------------------------------------------------------------ */
 
-/* Bytes of workspace cmc_score_select needs for B sequences of N CMEs. */
+/* Bytes of workspace cmc_score_select needs for B sequences of N CMEs: the
+ * B * N fp32 scores (rounded up to 256 bytes), then B completion counters
+ * (rounded up to 256 bytes). */
 CMC_API size_t cmc_score_select_workspace_size(int B, int N);
 
 /*
@@ -157,7 +159,17 @@ CMC_API size_t cmc_score_select_workspace_size(int B, int N);
  *   cme_bank      fp32 [B, N, D]    the decoder-ready CMEs m_j of each sequence
  *   idx_out       int32 [B, k]      output, ascending within each row
  *   scores_out    fp32 [B, N]       optional output (NULL: not written)
- *   workspace     >= cmc_score_select_workspace_size(B, N) bytes, any content
+ *   workspace     >= cmc_score_select_workspace_size(B, N) bytes, 16-byte
+ *                 aligned, ZERO-FILLED ONCE before its first use: it holds
+ *                 one completion counter per sequence, which every call leaves
+ *                 at zero again (the scores part may hold anything).  It may
+ *                 be NULL when scores_out is given.
+ *
+ * With a workspace, N <= 8192 and D <= 4096 the call is one kernel launch:
+ * the CTA that writes the last score of a sequence (a counter in the
+ * workspace tells it) selects that sequence's top k.  Otherwise (larger
+ * banks, or no workspace) scoring and selection are two launches.  Both give
+ * the same selection.
  *
  * Scores are computed in fp32 with a fixed summation order, so equal rows get
  * bit-identical scores.  Equal scores go to the lower index; -0 equals +0.  A
@@ -197,8 +209,10 @@ CMC_API size_t cmc_question_select_workspace_size(int B, int N);
  *   idx_out          int32 [B, k] ascending (may be NULL when k == 0)
  *   alpha_out, start_out  int32 [B]; either may be NULL; when both are NULL
  *                    chunk_offset, ctx_len and W are not used
- *   workspace        >= cmc_question_select_workspace_size(B, N) bytes, any
- *                    content, 16-byte aligned
+ *   workspace        >= cmc_question_select_workspace_size(B, N) bytes,
+ *                    16-byte aligned, zero-filled once before its first use
+ *                    (as for cmc_score_select: scores, squared norms, then
+ *                    B completion counters that every call leaves at zero)
  *
  * Limits: those of cmc_score_select, Lq >= 1, Lq * D <= 2^31, W >= 1 when
  * localising.

@@ -138,12 +138,27 @@ def score_select_workspace_size(B: int, N: int) -> int:
     return int(lib().cmc_score_select_workspace_size(B, N))
 
 
+_sel_ws_cache: Dict[Tuple, torch.Tensor] = {}
+
+
+def _selection_workspace(kind: str, nbytes: int, device: torch.device) -> torch.Tensor:
+    """A zero-filled selection workspace, one per (kind, device, stream, size):
+    its completion counters start at zero, and every call leaves them so."""
+    key = (kind, device.index, torch.cuda.current_stream(device).cuda_stream, nbytes)
+    ws = _sel_ws_cache.get(key)
+    if ws is None:
+        ws = torch.zeros(nbytes, dtype=torch.uint8, device=device)
+        _sel_ws_cache[key] = ws
+    return ws
+
+
 def score_select(question_emb: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
                  idx_out: Optional[torch.Tensor] = None,
                  scores_out: Optional[torch.Tensor] = None,
                  workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
     """Top-k CMEs by cosine similarity to the question vector, as int32 [B, k]
-    indices in ascending (document) order.  See cmc_score_select."""
+    indices in ascending (document) order.  See cmc_score_select.  A given
+    ``workspace`` must have been zero-filled before its first use."""
     _need(cme_bank, "cme_bank", torch.float32, 3)
     dev = cme_bank.device
     _need(question_emb, "question_emb", torch.float32, 2, dev)
@@ -159,12 +174,9 @@ def score_select(question_emb: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
         _need(scores_out, "scores_out", torch.float32, 2, dev)
         if tuple(scores_out.shape) != (B, N):
             raise ValueError(f"scores_out shape {tuple(scores_out.shape)} != {(B, N)}")
-    ws_bytes = 0
-    if scores_out is None:
-        need = score_select_workspace_size(B, N)
-        if workspace is None:
-            workspace = torch.empty(need, dtype=torch.uint8, device=dev)
-        ws_bytes = workspace.numel() * workspace.element_size()
+    if workspace is None:
+        workspace = _selection_workspace("select", score_select_workspace_size(B, N), dev)
+    ws_bytes = workspace.numel() * workspace.element_size()
     st = lib().cmc_score_select(_p(question_emb), _p(cme_bank), B, N, D, k, _p(idx_out),
                                 _p(scores_out), _p(workspace), ws_bytes, _stream(dev))
     check(st, "cmc_score_select")
@@ -203,7 +215,7 @@ def question_select(question_tokens: torch.Tensor, cme_bank: torch.Tensor, k: in
     start = torch.empty(B, dtype=torch.int32, device=dev) if locate else None
     need = int(lib().cmc_question_select_workspace_size(B, N))
     if workspace is None:
-        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+        workspace = _selection_workspace("question", need, dev)
     st = lib().cmc_question_select(
         _p(question_tokens), _p(q_len), Lq, _p(cme_bank), B, N, D, k, _p(chunk_offset),
         _p(ctx_len), int(W or 0), _p(q_vec), _p(idx), _p(alpha), _p(start), _p(workspace),

@@ -519,13 +519,332 @@ topk_select_cluster_kernel(const float* __restrict__ scores, int N, int k,
   sel_cluster_sync();  // the published counts stay readable until every CTA is done
 }
 
+// ---------------------------------------------------------------------------
+// One launch for scoring and selection (banks of at most kFusedMaxN CMEs of
+// dimension at most kFusedMaxD).
+//
+// CTA c scores the contiguous rows [c R, (c+1) R) of the flattened [B, N]
+// bank (R a multiple of the group size), a group of rows at a time with
+// every load of the group in flight at once (the thread's share of each row
+// is J float4s, its share of q_vec the same J float4s, held in registers).
+// Before the grid dependency wait the CTA asks L2 to prefetch its first rows,
+// so under programmatic dependent launch the bank streams in while the
+// previous kernel drains (a prefetch is a hint and leaves L2 coherent with
+// that kernel's writes).  The sums meet in a fixed tree (xor shuffles, then
+// the warps in order), so equal rows get bit-identical scores.
+//
+// At the end of each run of rows of one sequence the CTA fences its score
+// writes and adds the run's length to the sequence's counter; the CTA whose
+// addition completes N is the last to score that sequence and selects its
+// top k itself: keys are the order-preserving uint32 images of the scores,
+// a bit-by-bit search from the top bit finds the largest T with at least k
+// keys >= T (the k-th largest key), and an ordered compaction writes the keys
+// > T and the lowest-index keys == T in ascending index order.  It then puts
+// the counter back to zero for the next call.  No CTA waits on another.
+// ---------------------------------------------------------------------------
+
+constexpr int kFusedThreads = 512;
+constexpr int kFusedWarps = kFusedThreads / 32;
+constexpr int kFusedMaxN = 8192;                            // CMEs per sequence
+constexpr int kFusedMaxKpt = kFusedMaxN / kFusedThreads;    // keys per thread in the selection
+constexpr int kFusedMaxD = 4096;                            // J <= 2 float4s per thread and row
+constexpr int kFusedRows = 4;                               // rows per group (all loads in flight)
+
+struct FusedArgs {
+  const float* qv;        // [B, D]
+  const float* bank;      // [B, N, D]
+  int N, D, k;
+  long long rows;         // B * N
+  long long rows_per_cta;
+  float* scores;          // [B, N]
+  unsigned int* counters; // [B]: zero before the call, zero after it
+  int32_t* idx_out;       // [B, k]
+  LocateArgs la;          // la.sqnorm: also write squared norms and localise
+};
+
+// Exclusive prefix sums over the block of two per-thread values (warps in
+// order); `ws` holds two kFusedWarps-entry arrays used by this call only.
+__device__ __forceinline__ void fused_scan2(uint32_t a, uint32_t b, uint32_t (*ws)[kFusedWarps],
+                                            uint32_t* a_before, uint32_t* b_before) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t ia = a, ib = b;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t ta = __shfl_up_sync(0xffffffffu, ia, off);
+    const uint32_t tb = __shfl_up_sync(0xffffffffu, ib, off);
+    if (lane >= off) { ia += ta; ib += tb; }
+  }
+  if (lane == 31) { ws[0][warp] = ia; ws[1][warp] = ib; }
+  __syncthreads();
+  uint32_t pa = 0, pb = 0;
+  for (int w = 0; w < warp; ++w) { pa += ws[0][w]; pb += ws[1][w]; }
+  *a_before = pa + ia - a;
+  *b_before = pb + ib - b;
+}
+
+// The selection (and, with la.sqnorm, the localisation) of sequence b by the
+// CTA that completed its scores.  Every thread of the CTA calls it.
+__device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
+  __shared__ uint32_t cnt[2][kFusedWarps];
+  __shared__ uint32_t scan_a[2][kFusedWarps], scan_b[2][kFusedWarps];
+  __shared__ float best_v[kFusedWarps];
+  __shared__ int best_i[kFusedWarps];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int N = a.N, k = a.k;
+  __threadfence();  // the other CTAs' scores (published before their counter additions)
+  __syncthreads();
+  if (a.la.sqnorm) {
+    // CME-guided localisation: argmax of the squared norms, ties to the lower index
+    const float* sq = a.la.sqnorm + static_cast<long long>(b) * N;
+    float best = -1.f;
+    int bi = 0x7fffffff;
+    for (int j = tid; j < N; j += kFusedThreads) {
+      const float v = __ldcg(sq + j);
+      if (v > best) { best = v; bi = j; }
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, best, off);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+      if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
+    }
+    if (lane == 0) { best_v[warp] = best; best_i[warp] = bi; }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 1; w < kFusedWarps; ++w)
+        if (best_v[w] > best || (best_v[w] == best && best_i[w] < bi)) { best = best_v[w]; bi = best_i[w]; }
+      const long long alpha = a.la.chunk_offset[static_cast<long long>(b) * N + bi];
+      long long st = static_cast<long long>(a.la.ctx_len[b]) - a.la.W;
+      const long long centred = alpha - a.la.W / 2;
+      if (centred < st) st = centred;
+      if (st < 0) st = 0;
+      if (a.la.alpha_out) a.la.alpha_out[b] = static_cast<int32_t>(alpha);
+      if (a.la.start_out) a.la.start_out[b] = static_cast<int32_t>(st);
+    }
+  }
+  int32_t* out = a.idx_out + static_cast<long long>(b) * k;
+  if (k >= N) {
+    for (int j = tid; j < N; j += kFusedThreads) out[j] = j;
+  } else if (k > 0) {
+    // thread t holds the keys of indices t*kpt .. t*kpt + kpt - 1 (index order
+    // is thread order, then position); padding keys are 0, below every score's key
+    const int kpt = (N + kFusedThreads - 1) / kFusedThreads;
+    const float* sc = a.scores + static_cast<long long>(b) * N;
+    uint32_t key[kFusedMaxKpt];
+#pragma unroll
+    for (int e = 0; e < kFusedMaxKpt; ++e) {
+      const int j = tid * kpt + e;
+      key[e] = (e < kpt && j < N) ? orderable(__ldcg(sc + j)) : 0u;
+    }
+    int par = 0;
+    auto count_ge = [&](uint32_t c) -> uint32_t {  // keys >= c over the block (c >= 1)
+      uint32_t n = 0;
+#pragma unroll
+      for (int e = 0; e < kFusedMaxKpt; ++e) n += key[e] >= c ? 1u : 0u;
+      n = __reduce_add_sync(0xffffffffu, n);
+      if (lane == 0) cnt[par][warp] = n;
+      __syncthreads();
+      uint32_t tot = 0;
+#pragma unroll
+      for (int w = 0; w < kFusedWarps; ++w) tot += cnt[par][w];
+      par ^= 1;  // the other buffer: its readers passed this call's barrier
+      return tot;
+    };
+    // the k-th largest key: the largest T with at least k keys >= T
+    uint32_t T = 0u;
+    for (int bit = 31; bit >= 0; --bit) {
+      const uint32_t c = T | (1u << bit);
+      if (count_ge(c) >= static_cast<uint32_t>(k)) T = c;
+    }
+    const uint32_t gt = T == 0xFFFFFFFFu ? 0u : count_ge(T + 1u);
+    const uint32_t need = static_cast<uint32_t>(k) - gt;  // keys == T to keep, lowest index first
+    uint32_t n_gt = 0, n_eq = 0;
+#pragma unroll
+    for (int e = 0; e < kFusedMaxKpt; ++e) {
+      n_gt += key[e] > T ? 1u : 0u;
+      n_eq += key[e] == T ? 1u : 0u;
+    }
+    uint32_t eq_before, unused;
+    fused_scan2(n_eq, 0u, scan_a, &eq_before, &unused);
+    const uint32_t take = need > eq_before ? min(need - eq_before, n_eq) : 0u;
+    uint32_t slot, unused2;
+    fused_scan2(n_gt + take, 0u, scan_b, &slot, &unused2);
+    uint32_t r = eq_before;
+#pragma unroll
+    for (int e = 0; e < kFusedMaxKpt; ++e) {
+      const bool sel = key[e] > T || (key[e] == T && r++ < need);
+      if (sel && slot < static_cast<uint32_t>(k)) out[slot++] = tid * kpt + e;  // exactly k
+    }
+  }
+  if (tid == 0) a.counters[b] = 0u;  // ready for the next call
+  __syncthreads();                    // the shared scratch is reused by the caller
+}
+
+template <int J>  // float4s per thread and row: D / 4 <= J * kFusedThreads
+__global__ void __launch_bounds__(kFusedThreads, 2)
+score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
+  constexpr int RG = kFusedRows;  // rows per group
+  __shared__ float part[2][kFusedWarps][2 * RG];
+  __shared__ float qq_part[kFusedWarps];
+  __shared__ int last_flag;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int D4 = a.D >> 2;
+  const long long r_begin = static_cast<long long>(blockIdx.x) * a.rows_per_cta;
+  const long long r_end = min(r_begin + a.rows_per_cta, a.rows);
+  if (tid == 0 && r_end > r_begin) {
+    // L2 prefetch of the first two groups' rows (a hint: see above)
+    const long long n = min(r_end - r_begin, static_cast<long long>(2 * RG));
+    const char* src = reinterpret_cast<const char*>(a.bank + r_begin * a.D);
+    const unsigned long long bytes = static_cast<unsigned long long>(n) * a.D * 4;
+    for (unsigned long long off = 0; off < bytes; off += (1ull << 20)) {
+      const unsigned int sz = static_cast<unsigned int>(min(bytes - off, 1ull << 20));
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(src + off), "r"(sz) : "memory");
+    }
+  }
+  pdl_wait();
+  pdl_trigger();
+  int cur_b = -1;
+  float4 qr[J];
+  float qq = 0.f;
+  long long seg_begin = r_begin;
+  int g = 0;
+  for (long long r0 = r_begin; r0 < r_end; ++g) {
+    const int b = static_cast<int>(r0 / a.N);
+    const long long seq_end = static_cast<long long>(b + 1) * a.N;
+    const long long lim = min(r_end, seq_end);
+    const int nr = static_cast<int>(min(static_cast<long long>(RG), lim - r0));
+    if (b != cur_b) {  // this CTA's first rows of sequence b: its q_vec and q.q
+      cur_b = b;
+      const float4* q = reinterpret_cast<const float4*>(a.qv + static_cast<long long>(b) * a.D);
+      float acc = 0.f;
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        const int i4 = tid + j * kFusedThreads;
+        qr[j] = i4 < D4 ? __ldg(q + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
+        acc = fmaf(qr[j].x, qr[j].x, acc); acc = fmaf(qr[j].y, qr[j].y, acc);
+        acc = fmaf(qr[j].z, qr[j].z, acc); acc = fmaf(qr[j].w, qr[j].w, acc);
+      }
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+      if (lane == 0) qq_part[warp] = acc;
+      __syncthreads();
+      qq = qq_part[0];
+#pragma unroll
+      for (int w = 1; w < kFusedWarps; ++w) qq += qq_part[w];
+    }
+    float4 m[RG][J];
+#pragma unroll
+    for (int r = 0; r < RG; ++r)
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        const int i4 = tid + j * kFusedThreads;
+        m[r][j] = (r < nr && i4 < D4)
+                      ? ld_stream_f4(a.bank + (r0 + r) * a.D + 4 * static_cast<long long>(i4))
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    float dot[RG], mm[RG];
+#pragma unroll
+    for (int r = 0; r < RG; ++r) {
+      float d0 = 0.f, s0 = 0.f;
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        const float4 v = m[r][j], c = qr[j];
+        d0 = fmaf(v.x, c.x, d0); d0 = fmaf(v.y, c.y, d0); d0 = fmaf(v.z, c.z, d0); d0 = fmaf(v.w, c.w, d0);
+        s0 = fmaf(v.x, v.x, s0); s0 = fmaf(v.y, v.y, s0); s0 = fmaf(v.z, v.z, s0); s0 = fmaf(v.w, v.w, s0);
+      }
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) {
+        d0 += __shfl_xor_sync(0xffffffffu, d0, off);
+        s0 += __shfl_xor_sync(0xffffffffu, s0, off);
+      }
+      dot[r] = d0;
+      mm[r] = s0;
+    }
+    float* pg = &part[g & 1][0][0];
+    if (lane == 0) {
+#pragma unroll
+      for (int r = 0; r < RG; ++r) {
+        pg[warp * 2 * RG + 2 * r] = dot[r];
+        pg[warp * 2 * RG + 2 * r + 1] = mm[r];
+      }
+    }
+    __syncthreads();
+    if (tid < nr) {
+      float sd = pg[2 * tid], sm = pg[2 * tid + 1];
+#pragma unroll
+      for (int w = 1; w < kFusedWarps; ++w) {
+        sd += pg[w * 2 * RG + 2 * tid];
+        sm += pg[w * 2 * RG + 2 * tid + 1];
+      }
+      float sc = 0.f;
+      if (sm > 0.f && qq > 0.f) sc = sd / (sqrtf(sm) * sqrtf(qq));
+      if (sc == 0.f) sc = 0.f;  // -0 -> +0, so that -0 and +0 tie
+      a.scores[r0 + tid] = sc;
+      if (a.la.sqnorm) a.la.sqnorm[r0 + tid] = sm;
+    }
+    r0 += nr;
+    if (r0 == lim) {
+      // end of this CTA's run of sequence b: publish the scores, count the run
+      __threadfence();
+      __syncthreads();
+      if (tid == 0) {
+        const unsigned int run = static_cast<unsigned int>(r0 - seg_begin);
+        const unsigned int old = atomicAdd(a.counters + b, run);
+        last_flag = (old + run == static_cast<unsigned int>(a.N)) ? 1 : 0;
+      }
+      __syncthreads();
+      seg_begin = r0;
+      if (last_flag) fused_select(a, b);
+    }
+  }
+}
+
+// Launches score_select_fused_kernel; the caller has checked N <= kFusedMaxN
+// and D <= kFusedMaxD.
+static int launch_score_select_fused(const float* question_emb, const float* cme_bank, int B,
+                                     int N, int D, int k, int32_t* idx_out, float* sc,
+                                     unsigned int* counters, cudaStream_t s, const LocateArgs& la) {
+  const int J = (D / 4 <= kFusedThreads) ? 1 : 2;
+  const int RG = kFusedRows;
+  const long long rows = static_cast<long long>(B) * N;
+  const long long groups = (rows + RG - 1) / RG;
+  long long ctas = static_cast<long long>(sm_count()) * 2;
+  if (ctas > groups) ctas = groups;
+  const long long rows_per_cta = ((groups + ctas - 1) / ctas) * RG;
+  ctas = (rows + rows_per_cta - 1) / rows_per_cta;
+  FusedArgs a;
+  a.qv = question_emb;
+  a.bank = cme_bank;
+  a.N = N;
+  a.D = D;
+  a.k = k;
+  a.rows = rows;
+  a.rows_per_cta = rows_per_cta;
+  a.scores = sc;
+  a.counters = counters;
+  a.idx_out = idx_out;
+  a.la = la;
+  if (J == 1)
+    return launch_pdl(score_select_fused_kernel<1>, dim3(static_cast<unsigned>(ctas)),
+                      dim3(kFusedThreads), 0, s, a);
+  return launch_pdl(score_select_fused_kernel<2>, dim3(static_cast<unsigned>(ctas)),
+                    dim3(kFusedThreads), 0, s, a);
+}
+
 // The two selection kernels, scores written to `sc` (device, B * N floats);
 // with la.sqnorm set, the squared norms too and the localisation runs in the
 // selection kernel.
+// With `counters` (B zeroed words) and a bank of at most kFusedMaxN CMEs of
+// dimension at most kFusedMaxD, one launch (score_select_fused_kernel);
+// otherwise the two kernels.
 static int launch_score_select(const float* question_emb, const float* cme_bank, int B, int N,
                                int D, int k, int32_t* idx_out, float* sc, cudaStream_t s,
+                               unsigned int* counters = nullptr,
                                const LocateArgs& la = LocateArgs{nullptr, nullptr, nullptr, 0,
                                                                  nullptr, nullptr}) {
+  if (counters && N <= kFusedMaxN && D <= kFusedMaxD)
+    return launch_score_select_fused(question_emb, cme_bank, B, N, D, k, idx_out, sc, counters, s,
+                                     la);
   const long long rows = static_cast<long long>(B) * N;
   long long blocks = rows;
   const long long cap = static_cast<long long>(sm_count()) * (2048 / kScoreThreads);
@@ -585,7 +904,8 @@ extern "C" {
 
 size_t cmc_score_select_workspace_size(int B, int N) {
   if (B < 1 || N < 1) return 0;
-  return cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256);
+  return cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256) +
+         cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256);
 }
 
 int cmc_score_select(const float* question_emb, const float* cme_bank, int B, int N, int D, int k,
@@ -601,20 +921,28 @@ int cmc_score_select(const float* question_emb, const float* cme_bank, int B, in
   if ((scores_out && (reinterpret_cast<uintptr_t>(scores_out) & 3)) ||
       (idx_out && (reinterpret_cast<uintptr_t>(idx_out) & 3)))
     return CMC_ERR_ALIGN;
+  // Workspace: [B * N fp32 scores, 256-byte aligned][B completion counters].
+  // Without one (scores_out given) the two-launch path runs, which needs no
+  // counters.
   float* sc = scores_out;
-  if (!sc) {
-    if (!workspace) return CMC_ERR_WORKSPACE;
+  unsigned int* counters = nullptr;
+  if (workspace) {
     if (workspace_bytes < cmc_score_select_workspace_size(B, N)) return CMC_ERR_WORKSPACE;
     if (reinterpret_cast<uintptr_t>(workspace) & 3) return CMC_ERR_ALIGN;
-    sc = static_cast<float*>(workspace);
+    const size_t scores_bytes = align_up(static_cast<size_t>(B) * N * sizeof(float), 256);
+    counters = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + scores_bytes);
+    if (!sc) sc = static_cast<float*>(workspace);
+  } else if (!sc) {
+    return CMC_ERR_WORKSPACE;
   }
   return launch_score_select(question_emb, cme_bank, B, N, D, k, idx_out, sc,
-                             static_cast<cudaStream_t>(stream));
+                             static_cast<cudaStream_t>(stream), counters);
 }
 
 size_t cmc_question_select_workspace_size(int B, int N) {
   if (B < 1 || N < 1) return 0;
-  return 2 * cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256);
+  return 2 * cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256) +
+         cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256);
 }
 
 int cmc_question_select(const float* question_tokens, const int32_t* q_len, int Lq,
@@ -641,15 +969,20 @@ int cmc_question_select(const float* question_tokens, const int32_t* q_len, int 
                           static_cast<const void*>(alpha_out), static_cast<const void*>(start_out)})
     if (reinterpret_cast<uintptr_t>(ptr) & 3) return CMC_ERR_ALIGN;
   if (workspace_bytes < cmc_question_select_workspace_size(B, N)) return CMC_ERR_WORKSPACE;
+  // Workspace: [scores][squared norms] (B * N fp32 each, 256-byte aligned)
+  // [B completion counters].
+  const size_t scores_bytes = align_up(static_cast<size_t>(B) * N * sizeof(float), 256);
   float* sc = static_cast<float*>(workspace);
-  float* sq = sc + align_up(static_cast<size_t>(B) * N * sizeof(float), 256) / sizeof(float);
+  float* sq = sc + scores_bytes / sizeof(float);
+  unsigned int* counters =
+      reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + 2 * scores_bytes);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int D4 = D / 4;
   int st = launch_pdl(question_pool_kernel, dim3((D4 + 31) / 32, B),
                       dim3(kPoolThreads), 0, s, question_tokens, q_len, Lq, D, q_vec_out);
   if (st != CMC_OK) return st;
   LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out};
-  return launch_score_select(q_vec_out, cme_bank, B, N, D, k, idx_out, sc, s, la);
+  return launch_score_select(q_vec_out, cme_bank, B, N, D, k, idx_out, sc, s, counters, la);
 }
 
 }  // extern "C"

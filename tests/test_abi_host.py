@@ -76,10 +76,13 @@ def test_score_select_argument_checks(L):
     assert _sel(L, bank=FAKE + 4) == ALIGN
     assert _sel(L, ws=0) == WORKSPACE
     assert _sel(L, wsb=2 * 64 * 4 - 1) == WORKSPACE
+    assert _sel(L, wsb=512 + 255) == WORKSPACE  # room for the scores, not the counters
+    assert _sel(L, ws=0, scores=FAKE, wsb=0, bank=FAKE + 4) == ALIGN  # no workspace: scores_out
 
 
 def test_score_select_workspace_size(L):
-    assert L.cmc_score_select_workspace_size(3, 100) == 1280  # 1200 rounded up to 256
+    # 1200 bytes of scores rounded up to 256, then 3 counters rounded up to 256
+    assert L.cmc_score_select_workspace_size(3, 100) == 1280 + 256
     assert L.cmc_score_select_workspace_size(0, 100) == 0
 
 
@@ -211,7 +214,7 @@ def test_decode_step_rope_argument_checks(L):
 
 
 def test_question_select_workspace_size(L):
-    assert L.cmc_question_select_workspace_size(3, 100) == 2 * 1280
+    assert L.cmc_question_select_workspace_size(3, 100) == 2 * 1280 + 256
     assert L.cmc_question_select_workspace_size(0, 100) == 0
 
 

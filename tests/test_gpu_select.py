@@ -1,7 +1,14 @@
 """Tier-1 scoring and selection on the GPU against the fp64 oracle.
 
 The selected index set is compared bit-exactly (as an ordered array); scores
-within 1e-5 absolute (fp32 accumulation over D <= 4096 terms of a cosine)."""
+within 1e-5 absolute (fp32 accumulation over D <= 4096 terms of a cosine).
+
+Both launch paths run on every case: one launch (a workspace given, N <= 8192,
+D <= 4096: the CTA that completes a sequence's scores selects it) and two
+launches (no workspace, scores_out given, reached through the C ABI; also the
+path of larger banks).  They must select the same rows."""
+
+import ctypes
 
 import numpy as np
 import pytest
@@ -18,14 +25,32 @@ pytestmark = pytest.mark.gpu
 SCORE_ATOL = 1e-5
 
 
+def _two_launch(qd, bd, k):
+    """cmc_score_select without a workspace (scores_out given): the scoring
+    kernel, then the selection kernel."""
+    B, N, D = bd.shape
+    idx = torch.full((B, k), -1, dtype=torch.int32, device=bd.device)
+    sc = torch.empty((B, N), dtype=torch.float32, device=bd.device)
+    st = cmc.lib().cmc_score_select(
+        ctypes.c_void_p(qd.data_ptr()), ctypes.c_void_p(bd.data_ptr()), B, N, D, k,
+        ctypes.c_void_p(idx.data_ptr()), ctypes.c_void_p(sc.data_ptr()), None, 0,
+        ctypes.c_void_p(torch.cuda.current_stream(bd.device).cuda_stream))
+    assert st == 0
+    return idx, sc
+
+
 def _run(q, bank, k, dev):
     qd, bd = dev_f32(q, dev), dev_f32(bank, dev)
     scores = torch.empty(bank.shape[:2], dtype=torch.float32, device=dev)
     idx = cmc.score_select(qd, bd, k, scores_out=scores)
     # the workspace path (no scores_out) must select the same rows
     idx2 = cmc.score_select(qd, bd, k)
+    # and so must the two-launch path
+    idx3, scores3 = _two_launch(qd, bd, k)
     torch.cuda.synchronize()
     assert torch.equal(idx, idx2)
+    assert torch.equal(idx, idx3)
+    assert (scores - scores3).abs().max().item() <= 2 * SCORE_ATOL
     return idx.cpu().numpy(), scores.cpu().numpy()
 
 
@@ -81,12 +106,19 @@ def test_select_ties_go_to_lower_index(cuda_device):
 # the last three: a cluster of 8 selection CTAs per sequence (N > 8,192),
 # keys split across their shared memories (also unevenly: 50,001 = 8 x 6,250
 # + 1), and one CTA re-reading the keys from global memory (N / 8 > 49,152)
-@pytest.mark.parametrize("N,D,k", [(1, 4, 1), (1, 4, 0), (5, 8, 5), (1000, 36, 999),
-                                   (1025, 512, 17), (3000, 4, 1500), (4096, 128, 4095),
-                                   (9000, 8, 1234), (50001, 4, 777), (400003, 4, 1000)])
-def test_select_edge_shapes(cuda_device, N, D, k):
+#
+# One launch up to N = 8192 (16 keys per thread of the selecting CTA) and
+# D = 4096 (one or two float4s per thread and row: 2048 / 2052); two launches
+# above either limit (8193, 4100).
+@pytest.mark.parametrize("N,D,k,B", [
+    (1, 4, 1, 3), (1, 4, 0, 3), (5, 8, 5, 3), (1000, 36, 999, 3), (1025, 512, 17, 3),
+    (3000, 4, 1500, 3), (4096, 128, 4095, 3), (9000, 8, 1234, 3), (50001, 4, 777, 3),
+    (400003, 4, 1000, 3), (8192, 16, 4000, 2), (8193, 16, 100, 2), (777, 2048, 50, 2),
+    (777, 2052, 50, 2), (300, 4100, 50, 2), (33, 4096, 5, 7), (1024, 256, 100, 40)])
+def test_select_edge_shapes(cuda_device, N, D, k, B):
+    """Random banks (no planted margin).  Also CTAs whose rows span several
+    sequences (B = 7, N = 33; B = 40, N = 1024) in the one-launch path."""
     rng = np.random.default_rng(N + D + k)
-    B = 3
     q = rng.standard_normal((B, D)).astype(np.float32)
     bank = rng.standard_normal((B, N, D)).astype(np.float32)
     idx, scores = _run(q, bank, k, cuda_device)
@@ -127,3 +159,19 @@ def test_select_negative_and_signed_zero_scores(cuda_device):
     idx, scores = _run(q, bank, 3, cuda_device)
     assert idx[0].tolist() == [1, 2, 6]
     assert not np.signbit(scores[0, 3])
+
+
+def test_one_launch_counters_reset_across_calls(cuda_device):
+    """One workspace over calls on different banks: every call selects exactly
+    the planted set, and leaves the completion counters at zero."""
+    w = WORKLOADS["mistral_batched"]
+    ws = torch.zeros(cmc.score_select_workspace_size(8, w.N), dtype=torch.uint8,
+                     device=cuda_device)
+    for batch in (range(0, 8), range(8, 16), range(0, 8)):
+        si = selection_inputs(w, batch=batch)
+        idx = cmc.score_select(dev_f32(si.question_emb, cuda_device),
+                               dev_f32(si.cme_bank, cuda_device), w.k, workspace=ws)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(idx.cpu().numpy(), si.planted_idx)
+        counters = ws[-256:].view(torch.int32)[:8]
+        assert int(counters.abs().sum()) == 0
