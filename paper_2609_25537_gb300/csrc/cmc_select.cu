@@ -521,34 +521,39 @@ topk_select_cluster_kernel(const float* __restrict__ scores, int N, int k,
 
 // ---------------------------------------------------------------------------
 // One launch for scoring and selection (banks of at most kFusedMaxN CMEs of
-// dimension at most kFusedMaxD).
+// dimension at most kFusedMaxD, at most kFusedMaxRows CMEs in all).
 //
-// CTA c scores the contiguous rows [c R, (c+1) R) of the flattened [B, N]
-// bank (R a multiple of the group size), a group of rows at a time with
-// every load of the group in flight at once (the thread's share of each row
-// is J float4s, its share of q_vec the same J float4s, held in registers).
-// Before the grid dependency wait the CTA asks L2 to prefetch its first rows,
-// so under programmatic dependent launch the bank streams in while the
-// previous kernel drains (a prefetch is a hint and leaves L2 coherent with
-// that kernel's writes).  The sums meet in a fixed tree (xor shuffles, then
-// the warps in order), so equal rows get bit-identical scores.
+// CTA c (1,024 threads, one per SM) scores the contiguous rows
+// [c R, (c+1) R) of the flattened [B, N] bank in groups of up to kFusedRows
+// rows: thread t owns float4 t of every row and of q_vec, and copies its
+// float4s of two groups at a time into its own shared-memory slots with
+// cp.async, so every row of a CTA with at most two groups is requested at
+// once and no register holds data in flight.  Before the grid dependency wait the
+// CTA asks L2 to prefetch its rows, so under programmatic dependent launch
+// the bank streams in while the previous kernel drains (a prefetch is a hint
+// and leaves L2 coherent with that kernel's writes).  A row's partial sums
+// meet in the xor butterfly of the lanes, then the warps in order: equal rows
+// get bit-identical scores.
 //
 // At the end of each run of rows of one sequence the CTA fences its score
 // writes and adds the run's length to the sequence's counter; the CTA whose
-// addition completes N is the last to score that sequence and selects its
-// top k itself: keys are the order-preserving uint32 images of the scores,
-// a bit-by-bit search from the top bit finds the largest T with at least k
-// keys >= T (the k-th largest key), and an ordered compaction writes the keys
-// > T and the lowest-index keys == T in ascending index order.  It then puts
-// the counter back to zero for the next call.  No CTA waits on another.
+// addition completes N is the last to score that sequence and selects its top
+// k itself.  Keys are the order-preserving uint32 images of the scores; a
+// bit-by-bit search from the top bit finds the largest T with at least k keys
+// >= T (the k-th largest key), each round one counting barrier
+// (__syncthreads_count) per key a thread holds; an ordered compaction then
+// writes the keys > T and the lowest-index keys == T in ascending index
+// order.  It puts the counter back to zero for the next call.  No CTA waits
+// on another.
 // ---------------------------------------------------------------------------
 
-constexpr int kFusedThreads = 512;
+constexpr int kFusedThreads = 1024;
 constexpr int kFusedWarps = kFusedThreads / 32;
 constexpr int kFusedMaxN = 8192;                            // CMEs per sequence
 constexpr int kFusedMaxKpt = kFusedMaxN / kFusedThreads;    // keys per thread in the selection
-constexpr int kFusedMaxD = 4096;                            // J <= 2 float4s per thread and row
-constexpr int kFusedRows = 4;                               // rows per group (all loads in flight)
+constexpr int kFusedMaxD = 4 * kFusedThreads;               // one float4 per thread and row
+constexpr int kFusedRows = 8;                               // rows per group (all loads in flight)
+constexpr long long kFusedMaxRows = 16384;                  // larger banks: the two launches
 
 struct FusedArgs {
   const float* qv;        // [B, D]
@@ -562,31 +567,27 @@ struct FusedArgs {
   LocateArgs la;          // la.sqnorm: also write squared norms and localise
 };
 
-// Exclusive prefix sums over the block of two per-thread values (warps in
-// order); `ws` holds two kFusedWarps-entry arrays used by this call only.
-__device__ __forceinline__ void fused_scan2(uint32_t a, uint32_t b, uint32_t (*ws)[kFusedWarps],
-                                            uint32_t* a_before, uint32_t* b_before) {
+// Exclusive prefix sum over the block of one value per thread (warps in
+// order); `ws` is a kFusedWarps-entry array used by this call only.
+__device__ __forceinline__ uint32_t fused_scan(uint32_t v, uint32_t* ws) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t ia = a, ib = b;
+  uint32_t inc = v;
 #pragma unroll
   for (int off = 1; off < 32; off <<= 1) {
-    const uint32_t ta = __shfl_up_sync(0xffffffffu, ia, off);
-    const uint32_t tb = __shfl_up_sync(0xffffffffu, ib, off);
-    if (lane >= off) { ia += ta; ib += tb; }
+    const uint32_t t = __shfl_up_sync(0xffffffffu, inc, off);
+    if (lane >= off) inc += t;
   }
-  if (lane == 31) { ws[0][warp] = ia; ws[1][warp] = ib; }
+  if (lane == 31) ws[warp] = inc;
   __syncthreads();
-  uint32_t pa = 0, pb = 0;
-  for (int w = 0; w < warp; ++w) { pa += ws[0][w]; pb += ws[1][w]; }
-  *a_before = pa + ia - a;
-  *b_before = pb + ib - b;
+  uint32_t before = 0;
+  for (int w = 0; w < warp; ++w) before += ws[w];
+  return before + inc - v;
 }
 
 // The selection (and, with la.sqnorm, the localisation) of sequence b by the
 // CTA that completed its scores.  Every thread of the CTA calls it.
-__device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
-  __shared__ uint32_t cnt[2][kFusedWarps];
-  __shared__ uint32_t scan_a[2][kFusedWarps], scan_b[2][kFusedWarps];
+__device__ __forceinline__ void fused_select(const FusedArgs& a, int b) {
+  __shared__ uint32_t scan_eq[kFusedWarps], scan_sel[kFusedWarps];
   __shared__ float best_v[kFusedWarps];
   __shared__ int best_i[kFusedWarps];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -636,18 +637,11 @@ __device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
       const int j = tid * kpt + e;
       key[e] = (e < kpt && j < N) ? orderable(__ldcg(sc + j)) : 0u;
     }
-    int par = 0;
     auto count_ge = [&](uint32_t c) -> uint32_t {  // keys >= c over the block (c >= 1)
-      uint32_t n = 0;
-#pragma unroll
-      for (int e = 0; e < kFusedMaxKpt; ++e) n += key[e] >= c ? 1u : 0u;
-      n = __reduce_add_sync(0xffffffffu, n);
-      if (lane == 0) cnt[par][warp] = n;
-      __syncthreads();
       uint32_t tot = 0;
 #pragma unroll
-      for (int w = 0; w < kFusedWarps; ++w) tot += cnt[par][w];
-      par ^= 1;  // the other buffer: its readers passed this call's barrier
+      for (int e = 0; e < kFusedMaxKpt; ++e)
+        if (e < kpt) tot += static_cast<uint32_t>(__syncthreads_count(key[e] >= c));
       return tot;
     };
     // the k-th largest key: the largest T with at least k keys >= T
@@ -664,11 +658,9 @@ __device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
       n_gt += key[e] > T ? 1u : 0u;
       n_eq += key[e] == T ? 1u : 0u;
     }
-    uint32_t eq_before, unused;
-    fused_scan2(n_eq, 0u, scan_a, &eq_before, &unused);
+    const uint32_t eq_before = fused_scan(n_eq, scan_eq);
     const uint32_t take = need > eq_before ? min(need - eq_before, n_eq) : 0u;
-    uint32_t slot, unused2;
-    fused_scan2(n_gt + take, 0u, scan_b, &slot, &unused2);
+    uint32_t slot = fused_scan(n_gt + take, scan_sel);
     uint32_t r = eq_before;
 #pragma unroll
     for (int e = 0; e < kFusedMaxKpt; ++e) {
@@ -680,21 +672,43 @@ __device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
   __syncthreads();                    // the shared scratch is reused by the caller
 }
 
-template <int J>  // float4s per thread and row: D / 4 <= J * kFusedThreads
-__global__ void __launch_bounds__(kFusedThreads, 2)
+// 16-byte asynchronous copy global -> shared (cp.async, completion tracked
+// per thread by commit / wait groups), streaming through L2 only.
+__device__ __forceinline__ void sel_cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(
+                   static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
+               "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void sel_cp_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void sel_cp_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+constexpr int kFusedStages = 2;  // row groups in flight per CTA
+__host__ __device__ constexpr size_t fused_smem_bytes() {
+  return static_cast<size_t>(kFusedStages) * kFusedRows * kFusedThreads * 16;
+}
+
+__global__ void __launch_bounds__(kFusedThreads, 1)
 score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
   constexpr int RG = kFusedRows;  // rows per group
+  // [stage][row][thread]: thread t copies float4 t of each row into its own
+  // slots and reads only those back, so a stage needs no barrier to be reused
+  extern __shared__ float4 rows_s[];
   __shared__ float part[2][kFusedWarps][2 * RG];
   __shared__ float qq_part[kFusedWarps];
+  __shared__ float4 q_s[kFusedThreads];  // q_vec of the current sequence
   __shared__ int last_flag;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int D4 = a.D >> 2;
-  const long long r_begin = static_cast<long long>(blockIdx.x) * a.rows_per_cta;
-  const long long r_end = min(r_begin + a.rows_per_cta, a.rows);
+  const bool own = tid < D4;
+  // row indices fit in 32 bits: at most kFusedMaxRows rows
+  const int r_begin = static_cast<int>(blockIdx.x) * static_cast<int>(a.rows_per_cta);
+  const int r_end = min(r_begin + static_cast<int>(a.rows_per_cta), static_cast<int>(a.rows));
   if (tid == 0 && r_end > r_begin) {
-    // L2 prefetch of the first two groups' rows (a hint: see above)
-    const long long n = min(r_end - r_begin, static_cast<long long>(2 * RG));
-    const char* src = reinterpret_cast<const char*>(a.bank + r_begin * a.D);
+    // L2 prefetch of the rows of the first groups (a hint: see above)
+    const int n = min(r_end - r_begin, kFusedStages * RG);
+    const char* src = reinterpret_cast<const char*>(a.bank + static_cast<long long>(r_begin) * a.D);
     const unsigned long long bytes = static_cast<unsigned long long>(n) * a.D * 4;
     for (unsigned long long off = 0; off < bytes; off += (1ull << 20)) {
       const unsigned int sz = static_cast<unsigned int>(min(bytes - off, 1ull << 20));
@@ -703,75 +717,74 @@ score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
   }
   pdl_wait();
   pdl_trigger();
+  // a group: up to RG consecutive rows of one sequence within [r_begin, r_end)
+  auto group_len = [&](int r0) { return min(RG, min(r_end, (r0 / a.N + 1) * a.N) - r0); };
+  const float4* bank4 = reinterpret_cast<const float4*>(a.bank) + tid;
+  auto issue = [&](int r0, int st) {  // this thread's copies of a group, one commit group
+    const int nr = group_len(r0);
+    float4* dst = rows_s + st * RG * kFusedThreads + tid;
+    for (int r = 0; r < nr; ++r)
+      if (own) sel_cp_async16(dst + r * kFusedThreads, bank4 + static_cast<long long>(r0 + r) * D4);
+    sel_cp_commit();
+    return nr;
+  };
+  int ri = r_begin, gi = 0;  // next row to issue, groups issued
+  for (; gi < kFusedStages && ri < r_end; ++gi) ri += issue(ri, gi);
   int cur_b = -1;
-  float4 qr[J];
   float qq = 0.f;
-  long long seg_begin = r_begin;
-  int g = 0;
-  for (long long r0 = r_begin; r0 < r_end; ++g) {
-    const int b = static_cast<int>(r0 / a.N);
-    const long long seq_end = static_cast<long long>(b + 1) * a.N;
-    const long long lim = min(r_end, seq_end);
-    const int nr = static_cast<int>(min(static_cast<long long>(RG), lim - r0));
+  for (int r0 = r_begin, g = 0; r0 < r_end; ++g) {
+    const int b = r0 / a.N;
+    const int lim = min(r_end, (b + 1) * a.N);  // end of this CTA's run of sequence b
+    const int nr = group_len(r0);
     if (b != cur_b) {  // this CTA's first rows of sequence b: its q_vec and q.q
       cur_b = b;
-      const float4* q = reinterpret_cast<const float4*>(a.qv + static_cast<long long>(b) * a.D);
+      const float4 qr =
+          own ? __ldg(reinterpret_cast<const float4*>(a.qv + static_cast<long long>(b) * a.D) + tid)
+              : make_float4(0.f, 0.f, 0.f, 0.f);
+      q_s[tid] = qr;  // read back by this thread only
       float acc = 0.f;
-#pragma unroll
-      for (int j = 0; j < J; ++j) {
-        const int i4 = tid + j * kFusedThreads;
-        qr[j] = i4 < D4 ? __ldg(q + i4) : make_float4(0.f, 0.f, 0.f, 0.f);
-        acc = fmaf(qr[j].x, qr[j].x, acc); acc = fmaf(qr[j].y, qr[j].y, acc);
-        acc = fmaf(qr[j].z, qr[j].z, acc); acc = fmaf(qr[j].w, qr[j].w, acc);
-      }
+      acc = fmaf(qr.x, qr.x, acc); acc = fmaf(qr.y, qr.y, acc);
+      acc = fmaf(qr.z, qr.z, acc); acc = fmaf(qr.w, qr.w, acc);
 #pragma unroll
       for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
       if (lane == 0) qq_part[warp] = acc;
       __syncthreads();
       qq = qq_part[0];
-#pragma unroll
+#pragma unroll 4
       for (int w = 1; w < kFusedWarps; ++w) qq += qq_part[w];
     }
-    float4 m[RG][J];
-#pragma unroll
-    for (int r = 0; r < RG; ++r)
-#pragma unroll
-      for (int j = 0; j < J; ++j) {
-        const int i4 = tid + j * kFusedThreads;
-        m[r][j] = (r < nr && i4 < D4)
-                      ? ld_stream_f4(a.bank + (r0 + r) * a.D + 4 * static_cast<long long>(i4))
-                      : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-    float dot[RG], mm[RG];
+    // this group's copies have landed once at most (issued - g - 1) later groups are pending
+    if (gi - g - 1 >= 1) sel_cp_wait<1>(); else sel_cp_wait<0>();
+    // each row's dot and squared norm: this thread's partials, then the xor
+    // butterfly of the lanes; lane 0 leaves the warp's sums for the row
+    const float4 qr = q_s[tid];
+    const float4* src = rows_s + (g % kFusedStages) * RG * kFusedThreads + tid;
+    float* pg = &part[g & 1][0][0];
 #pragma unroll
     for (int r = 0; r < RG; ++r) {
+      const float4 m = (r < nr && own) ? src[r * kFusedThreads] : make_float4(0.f, 0.f, 0.f, 0.f);
       float d0 = 0.f, s0 = 0.f;
-#pragma unroll
-      for (int j = 0; j < J; ++j) {
-        const float4 v = m[r][j], c = qr[j];
-        d0 = fmaf(v.x, c.x, d0); d0 = fmaf(v.y, c.y, d0); d0 = fmaf(v.z, c.z, d0); d0 = fmaf(v.w, c.w, d0);
-        s0 = fmaf(v.x, v.x, s0); s0 = fmaf(v.y, v.y, s0); s0 = fmaf(v.z, v.z, s0); s0 = fmaf(v.w, v.w, s0);
-      }
+      d0 = fmaf(m.x, qr.x, d0); d0 = fmaf(m.y, qr.y, d0); d0 = fmaf(m.z, qr.z, d0); d0 = fmaf(m.w, qr.w, d0);
+      s0 = fmaf(m.x, m.x, s0); s0 = fmaf(m.y, m.y, s0); s0 = fmaf(m.z, m.z, s0); s0 = fmaf(m.w, m.w, s0);
 #pragma unroll
       for (int off = 16; off >= 1; off >>= 1) {
         d0 += __shfl_xor_sync(0xffffffffu, d0, off);
         s0 += __shfl_xor_sync(0xffffffffu, s0, off);
       }
-      dot[r] = d0;
-      mm[r] = s0;
-    }
-    float* pg = &part[g & 1][0][0];
-    if (lane == 0) {
-#pragma unroll
-      for (int r = 0; r < RG; ++r) {
-        pg[warp * 2 * RG + 2 * r] = dot[r];
-        pg[warp * 2 * RG + 2 * r + 1] = mm[r];
+      if (lane == 0) {
+        pg[warp * 2 * RG + 2 * r] = d0;
+        pg[warp * 2 * RG + 2 * r + 1] = s0;
       }
+    }
+    // the stage just read is this thread's own: refill it with a later group
+    if (ri < r_end) {
+      ri += issue(ri, g % kFusedStages);
+      ++gi;
     }
     __syncthreads();
     if (tid < nr) {
       float sd = pg[2 * tid], sm = pg[2 * tid + 1];
-#pragma unroll
+#pragma unroll 4
       for (int w = 1; w < kFusedWarps; ++w) {
         sd += pg[w * 2 * RG + 2 * tid];
         sm += pg[w * 2 * RG + 2 * tid + 1];
@@ -788,29 +801,36 @@ score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
       __threadfence();
       __syncthreads();
       if (tid == 0) {
-        const unsigned int run = static_cast<unsigned int>(r0 - seg_begin);
+        const unsigned int run = static_cast<unsigned int>(r0 - max(r_begin, b * a.N));
         const unsigned int old = atomicAdd(a.counters + b, run);
         last_flag = (old + run == static_cast<unsigned int>(a.N)) ? 1 : 0;
       }
       __syncthreads();
-      seg_begin = r0;
       if (last_flag) fused_select(a, b);
     }
   }
 }
 
-// Launches score_select_fused_kernel; the caller has checked N <= kFusedMaxN
-// and D <= kFusedMaxD.
+// Launches score_select_fused_kernel; the caller has checked the limits.
 static int launch_score_select_fused(const float* question_emb, const float* cme_bank, int B,
                                      int N, int D, int k, int32_t* idx_out, float* sc,
                                      unsigned int* counters, cudaStream_t s, const LocateArgs& la) {
-  const int J = (D / 4 <= kFusedThreads) ? 1 : 2;
-  const int RG = kFusedRows;
+  static std::once_flag attr_once[64];
+  int dev = 0;
+  int st = record_cuda_error(cudaGetDevice(&dev));
+  if (st != CMC_OK) return st;
+  if (dev < 0 || dev >= 64) return CMC_ERR_CUDA;
+  std::call_once(attr_once[dev], [&] {
+    st = record_cuda_error(cudaFuncSetAttribute(score_select_fused_kernel,
+                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                static_cast<int>(fused_smem_bytes())));
+  });
+  if (st != CMC_OK) return st;
+  // one CTA per SM at most, every CTA a contiguous run of rows
   const long long rows = static_cast<long long>(B) * N;
-  const long long groups = (rows + RG - 1) / RG;
-  long long ctas = static_cast<long long>(sm_count()) * 2;
-  if (ctas > groups) ctas = groups;
-  const long long rows_per_cta = ((groups + ctas - 1) / ctas) * RG;
+  long long ctas = (rows + kFusedRows - 1) / kFusedRows;
+  if (ctas > sm_count()) ctas = sm_count();
+  const long long rows_per_cta = (rows + ctas - 1) / ctas;
   ctas = (rows + rows_per_cta - 1) / rows_per_cta;
   FusedArgs a;
   a.qv = question_emb;
@@ -824,25 +844,22 @@ static int launch_score_select_fused(const float* question_emb, const float* cme
   a.counters = counters;
   a.idx_out = idx_out;
   a.la = la;
-  if (J == 1)
-    return launch_pdl(score_select_fused_kernel<1>, dim3(static_cast<unsigned>(ctas)),
-                      dim3(kFusedThreads), 0, s, a);
-  return launch_pdl(score_select_fused_kernel<2>, dim3(static_cast<unsigned>(ctas)),
-                    dim3(kFusedThreads), 0, s, a);
+  return launch_pdl(score_select_fused_kernel, dim3(static_cast<unsigned>(ctas)),
+                    dim3(kFusedThreads), fused_smem_bytes(), s, a);
 }
 
 // The two selection kernels, scores written to `sc` (device, B * N floats);
 // with la.sqnorm set, the squared norms too and the localisation runs in the
 // selection kernel.
-// With `counters` (B zeroed words) and a bank of at most kFusedMaxN CMEs of
-// dimension at most kFusedMaxD, one launch (score_select_fused_kernel);
-// otherwise the two kernels.
+// With `counters` (B zeroed words) and a bank within the limits of
+// score_select_fused_kernel, one launch; otherwise the two kernels.
 static int launch_score_select(const float* question_emb, const float* cme_bank, int B, int N,
                                int D, int k, int32_t* idx_out, float* sc, cudaStream_t s,
                                unsigned int* counters = nullptr,
                                const LocateArgs& la = LocateArgs{nullptr, nullptr, nullptr, 0,
                                                                  nullptr, nullptr}) {
-  if (counters && N <= kFusedMaxN && D <= kFusedMaxD)
+  if (counters && N <= kFusedMaxN && D <= kFusedMaxD &&
+      static_cast<long long>(B) * N <= kFusedMaxRows)
     return launch_score_select_fused(question_emb, cme_bank, B, N, D, k, idx_out, sc, counters, s,
                                      la);
   const long long rows = static_cast<long long>(B) * N;
