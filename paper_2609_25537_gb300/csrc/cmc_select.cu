@@ -552,7 +552,7 @@ constexpr int kFusedWarps = kFusedThreads / 32;
 constexpr int kFusedMaxN = 8192;                            // CMEs per sequence
 constexpr int kFusedMaxKpt = kFusedMaxN / kFusedThreads;    // keys per thread in the selection
 constexpr int kFusedMaxD = 4 * kFusedThreads;               // one float4 per thread and row
-constexpr int kFusedRows = 8;                               // rows per group (all loads in flight)
+constexpr int kFusedRows = 6;                               // rows per group (all loads in flight)
 constexpr long long kFusedMaxRows = 16384;                  // larger banks: the two launches
 
 struct FusedArgs {
@@ -586,7 +586,7 @@ __device__ __forceinline__ uint32_t fused_scan(uint32_t v, uint32_t* ws) {
 
 // The selection (and, with la.sqnorm, the localisation) of sequence b by the
 // CTA that completed its scores.  Every thread of the CTA calls it.
-__device__ __forceinline__ void fused_select(const FusedArgs& a, int b) {
+__device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
   __shared__ uint32_t scan_eq[kFusedWarps], scan_sel[kFusedWarps];
   __shared__ float best_v[kFusedWarps];
   __shared__ int best_i[kFusedWarps];
@@ -688,6 +688,8 @@ constexpr int kFusedStages = 2;  // row groups in flight per CTA
 __host__ __device__ constexpr size_t fused_smem_bytes() {
   return static_cast<size_t>(kFusedStages) * kFusedRows * kFusedThreads * 16;
 }
+// with the kernel's static shared memory (about 21 KB), within the 227 KB a CTA may use
+static_assert(fused_smem_bytes() <= 200 * 1024, "row stages do not fit in shared memory");
 
 __global__ void __launch_bounds__(kFusedThreads, 1)
 score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
