@@ -165,11 +165,12 @@ CMC_API size_t cmc_score_select_workspace_size(int B, int N);
  *                 at zero again (the scores part may hold anything).  It may
  *                 be NULL when scores_out is given.
  *
- * With a workspace, N <= 8192 and D <= 4096 the call is one kernel launch:
- * the CTA that writes the last score of a sequence (a counter in the
- * workspace tells it) selects that sequence's top k.  Otherwise (larger
- * banks, or no workspace) scoring and selection are two launches.  Both give
- * the same selection.
+ * Small banks with a workspace (D <= 4096, N <= 2048, and B * N rows that
+ * CTAs of at most 8 rows of one sequence cover in one wave of one CTA per SM)
+ * take one kernel launch: the CTA that writes the last score of a sequence (a
+ * counter in the workspace tells it) selects that sequence's top k.  Larger
+ * banks, or no workspace, take two launches (scoring, then selection).  Both
+ * give the same selection.
  *
  * Scores are computed in fp32 with a fixed summation order, so equal rows get
  * bit-identical scores.  Equal scores go to the lower index; -0 equals +0.  A

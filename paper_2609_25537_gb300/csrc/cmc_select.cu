@@ -520,47 +520,46 @@ topk_select_cluster_kernel(const float* __restrict__ scores, int N, int k,
 }
 
 // ---------------------------------------------------------------------------
-// One launch for scoring and selection (banks of at most kFusedMaxN CMEs of
-// dimension at most kFusedMaxD, at most kFusedMaxRows CMEs in all).
+// One launch for scoring and selection, for small banks: every CTA scores R
+// rows of one sequence (R <= kFusedRows divides N, and B N / R CTAs fit in one
+// wave of one CTA per SM).
 //
-// CTA c (1,024 threads, one per SM) scores the contiguous rows
-// [c R, (c+1) R) of the flattened [B, N] bank in groups of up to kFusedRows
-// rows: thread t owns float4 t of every row and of q_vec, and copies its
-// float4s of two groups at a time into its own shared-memory slots with
-// cp.async, so every row of a CTA with at most two groups is requested at
-// once and no register holds data in flight.  Before the grid dependency wait the
-// CTA asks L2 to prefetch its rows, so under programmatic dependent launch
-// the bank streams in while the previous kernel drains (a prefetch is a hint
-// and leaves L2 coherent with that kernel's writes).  A row's partial sums
-// meet in the xor butterfly of the lanes, then the warps in order: equal rows
-// get bit-identical scores.
+// CTA c (1,024 threads) copies its R rows into shared memory with cp.async,
+// thread t taking float4 t of each row, so all of them are requested at
+// once; while they are in flight it reduces q_vec . q_vec of its sequence.
+// Before the grid dependency wait the CTA asks L2 to prefetch its rows, so
+// under programmatic dependent launch the bank streams in while the previous
+// kernel drains (a prefetch is a hint and leaves L2 coherent with that
+// kernel's writes).  Each thread's partial dot and squared norm of the R rows
+// (16 values, zero past R) meet across the lanes in a halving butterfly -- at
+// lane offset o the lanes with bit o set keep the upper half of their values
+// and add their partner's upper half, then the lane pairs add -- which adds
+// the same pairs as a plain xor butterfly for every value, in a quarter of
+// the shuffles; then warp r adds row r's 32 warp sums in the same butterfly.
+// Equal rows thus get bit-identical scores.
 //
-// At the end of each run of rows of one sequence the CTA fences its score
-// writes and adds the run's length to the sequence's counter; the CTA whose
-// addition completes N is the last to score that sequence and selects its top
-// k itself.  Keys are the order-preserving uint32 images of the scores; a
-// bit-by-bit search from the top bit finds the largest T with at least k keys
-// >= T (the k-th largest key), each round one counting barrier
-// (__syncthreads_count) per key a thread holds; an ordered compaction then
-// writes the keys > T and the lowest-index keys == T in ascending index
-// order.  It puts the counter back to zero for the next call.  No CTA waits
-// on another.
+// The CTA then releases its score writes (fence.acq_rel.gpu) and adds R to
+// the sequence's counter; the CTA whose addition completes N is the last to
+// score that sequence and selects its top k itself.  Keys are the order-
+// preserving uint32 images of the scores; a bit-by-bit search from the top
+// bit finds the largest T with at least k keys >= T (the k-th largest key),
+// each round one counting barrier (__syncthreads_count) per key a thread
+// holds; an ordered compaction then writes the keys > T and the lowest-index
+// keys == T in ascending index order.  It puts the counter back to zero for
+// the next call.  No CTA waits on another.
 // ---------------------------------------------------------------------------
 
 constexpr int kFusedThreads = 1024;
 constexpr int kFusedWarps = kFusedThreads / 32;
-constexpr int kFusedMaxN = 8192;                            // CMEs per sequence
-constexpr int kFusedMaxKpt = kFusedMaxN / kFusedThreads;    // keys per thread in the selection
-constexpr int kFusedMaxD = 4 * kFusedThreads;               // one float4 per thread and row
-constexpr int kFusedRows = 6;                               // rows per group (all loads in flight)
-constexpr long long kFusedMaxRows = 16384;                  // larger banks: the two launches
+constexpr int kFusedRows = 8;                    // rows per CTA at most
+constexpr int kFusedMaxD = 4 * kFusedThreads;    // one float4 per thread and row
+constexpr int kFusedMaxN = 2 * kFusedThreads;    // two keys per thread in the selection
 
 struct FusedArgs {
   const float* qv;        // [B, D]
   const float* bank;      // [B, N, D]
   int N, D, k;
-  long long rows;         // B * N
-  long long rows_per_cta;
+  int rows_per_cta;       // R: divides N
   float* scores;          // [B, N]
   unsigned int* counters; // [B]: zero before the call, zero after it
   int32_t* idx_out;       // [B, k]
@@ -568,8 +567,12 @@ struct FusedArgs {
 };
 
 // Exclusive prefix sum over the block of one value per thread (warps in
-// order); `ws` is a kFusedWarps-entry array used by this call only.
+// order); `ws` is a kFusedWarps-entry array used by this call only.  Each
+// warp scans its values with shuffles, and after one barrier every warp scans
+// the 32 warp totals itself (kFusedWarps == 32) and takes the prefix at its
+// own index.
 __device__ __forceinline__ uint32_t fused_scan(uint32_t v, uint32_t* ws) {
+  static_assert(kFusedWarps == 32, "one warp total per lane");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t inc = v;
 #pragma unroll
@@ -579,9 +582,63 @@ __device__ __forceinline__ uint32_t fused_scan(uint32_t v, uint32_t* ws) {
   }
   if (lane == 31) ws[warp] = inc;
   __syncthreads();
-  uint32_t before = 0;
-  for (int w = 0; w < warp; ++w) before += ws[w];
+  const uint32_t tot = ws[lane];
+  uint32_t tinc = tot;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t t = __shfl_up_sync(0xffffffffu, tinc, off);
+    if (lane >= off) tinc += t;
+  }
+  const uint32_t before = __shfl_sync(0xffffffffu, tinc - tot, warp);
   return before + inc - v;
+}
+
+// Top k of one sequence's N scores (N <= KPT * kFusedThreads), written to
+// out[0..k) in ascending index order.  Thread t holds the keys of indices
+// t*KPT .. t*KPT + KPT - 1 in registers (index order is thread order, then
+// position); padding keys are 0, below every score's key.  Every thread of
+// the CTA calls it.
+template <int KPT>
+__device__ __forceinline__ void fused_topk(const float* sc, int N, int k, int32_t* out,
+                                           uint32_t* scan_eq, uint32_t* scan_sel) {
+  const int tid = threadIdx.x;
+  uint32_t key[KPT];
+#pragma unroll
+  for (int e = 0; e < KPT; ++e) {
+    const int j = tid * KPT + e;
+    key[e] = j < N ? orderable(__ldcg(sc + j)) : 0u;
+  }
+  // the k-th largest key: the largest T with at least k keys >= T, one bit a
+  // round from the top; a round counts over the block with KPT counting barriers
+  uint32_t T = 0u;
+  for (int bit = 31; bit >= 0; --bit) {
+    const uint32_t c = T | (1u << bit);
+    int n = 0;
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) n += __syncthreads_count(key[e] >= c);
+    if (n >= k) T = c;
+  }
+  int gt = 0;  // keys > T
+  if (T != 0xFFFFFFFFu) {
+#pragma unroll
+    for (int e = 0; e < KPT; ++e) gt += __syncthreads_count(key[e] > T);
+  }
+  const uint32_t need = static_cast<uint32_t>(k - gt);  // keys == T to keep, lowest index first
+  uint32_t n_gt = 0, n_eq = 0;
+#pragma unroll
+  for (int e = 0; e < KPT; ++e) {
+    n_gt += key[e] > T ? 1u : 0u;
+    n_eq += key[e] == T ? 1u : 0u;
+  }
+  const uint32_t eq_before = fused_scan(n_eq, scan_eq);
+  const uint32_t take = need > eq_before ? min(need - eq_before, n_eq) : 0u;
+  uint32_t slot = fused_scan(n_gt + take, scan_sel);
+  uint32_t r = eq_before;
+#pragma unroll
+  for (int e = 0; e < KPT; ++e) {
+    const bool sel = key[e] > T || (key[e] == T && r++ < need);
+    if (sel && slot < static_cast<uint32_t>(k)) out[slot++] = tid * KPT + e;  // exactly k
+  }
 }
 
 // The selection (and, with la.sqnorm, the localisation) of sequence b by the
@@ -592,7 +649,9 @@ __device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
   __shared__ int best_i[kFusedWarps];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int N = a.N, k = a.k;
-  __threadfence();  // the other CTAs' scores (published before their counter additions)
+  // acquire: thread 0 saw the last counter addition; the other CTAs released
+  // their score writes before theirs, and the barrier passes the order on
+  if (tid == 0) asm volatile("fence.acq_rel.gpu;\n" ::: "memory");
   __syncthreads();
   if (a.la.sqnorm) {
     // CME-guided localisation: argmax of the squared norms, ties to the lower index
@@ -624,199 +683,138 @@ __device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
     }
   }
   int32_t* out = a.idx_out + static_cast<long long>(b) * k;
+  const float* sc = a.scores + static_cast<long long>(b) * N;
   if (k >= N) {
     for (int j = tid; j < N; j += kFusedThreads) out[j] = j;
   } else if (k > 0) {
-    // thread t holds the keys of indices t*kpt .. t*kpt + kpt - 1 (index order
-    // is thread order, then position); padding keys are 0, below every score's key
-    const int kpt = (N + kFusedThreads - 1) / kFusedThreads;
-    const float* sc = a.scores + static_cast<long long>(b) * N;
-    uint32_t key[kFusedMaxKpt];
-#pragma unroll
-    for (int e = 0; e < kFusedMaxKpt; ++e) {
-      const int j = tid * kpt + e;
-      key[e] = (e < kpt && j < N) ? orderable(__ldcg(sc + j)) : 0u;
-    }
-    auto count_ge = [&](uint32_t c) -> uint32_t {  // keys >= c over the block (c >= 1)
-      uint32_t tot = 0;
-#pragma unroll
-      for (int e = 0; e < kFusedMaxKpt; ++e)
-        if (e < kpt) tot += static_cast<uint32_t>(__syncthreads_count(key[e] >= c));
-      return tot;
-    };
-    // the k-th largest key: the largest T with at least k keys >= T
-    uint32_t T = 0u;
-    for (int bit = 31; bit >= 0; --bit) {
-      const uint32_t c = T | (1u << bit);
-      if (count_ge(c) >= static_cast<uint32_t>(k)) T = c;
-    }
-    const uint32_t gt = T == 0xFFFFFFFFu ? 0u : count_ge(T + 1u);
-    const uint32_t need = static_cast<uint32_t>(k) - gt;  // keys == T to keep, lowest index first
-    uint32_t n_gt = 0, n_eq = 0;
-#pragma unroll
-    for (int e = 0; e < kFusedMaxKpt; ++e) {
-      n_gt += key[e] > T ? 1u : 0u;
-      n_eq += key[e] == T ? 1u : 0u;
-    }
-    const uint32_t eq_before = fused_scan(n_eq, scan_eq);
-    const uint32_t take = need > eq_before ? min(need - eq_before, n_eq) : 0u;
-    uint32_t slot = fused_scan(n_gt + take, scan_sel);
-    uint32_t r = eq_before;
-#pragma unroll
-    for (int e = 0; e < kFusedMaxKpt; ++e) {
-      const bool sel = key[e] > T || (key[e] == T && r++ < need);
-      if (sel && slot < static_cast<uint32_t>(k)) out[slot++] = tid * kpt + e;  // exactly k
-    }
+    if (N <= kFusedThreads) fused_topk<1>(sc, N, k, out, scan_eq, scan_sel);
+    else fused_topk<2>(sc, N, k, out, scan_eq, scan_sel);
   }
   if (tid == 0) a.counters[b] = 0u;  // ready for the next call
   __syncthreads();                    // the shared scratch is reused by the caller
 }
 
-// 16-byte asynchronous copy global -> shared (cp.async, completion tracked
-// per thread by commit / wait groups), streaming through L2 only.
+// 16-byte asynchronous copy global -> shared (cp.async), through L2 only.
 __device__ __forceinline__ void sel_cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(
                    static_cast<uint32_t>(__cvta_generic_to_shared(dst))),
                "l"(src)
                : "memory");
 }
-__device__ __forceinline__ void sel_cp_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void sel_cp_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
 
-constexpr int kFusedStages = 2;  // row groups in flight per CTA
 __host__ __device__ constexpr size_t fused_smem_bytes() {
-  return static_cast<size_t>(kFusedStages) * kFusedRows * kFusedThreads * 16;
+  return static_cast<size_t>(kFusedRows) * kFusedThreads * 16;
 }
-// with the kernel's static shared memory (about 21 KB), within the 227 KB a CTA may use
-static_assert(fused_smem_bytes() <= 200 * 1024, "row stages do not fit in shared memory");
 
 __global__ void __launch_bounds__(kFusedThreads, 1)
 score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
-  constexpr int RG = kFusedRows;  // rows per group
-  // [stage][row][thread]: thread t copies float4 t of each row into its own
-  // slots and reads only those back, so a stage needs no barrier to be reused
+  constexpr int RG = kFusedRows;
+  // [row][thread]: thread t copies float4 t of each row into its own slot
   extern __shared__ float4 rows_s[];
-  __shared__ float part[2][kFusedWarps][2 * RG];
+  __shared__ float part[kFusedWarps][2 * RG];
   __shared__ float qq_part[kFusedWarps];
-  __shared__ float4 q_s[kFusedThreads];  // q_vec of the current sequence
   __shared__ int last_flag;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int D4 = a.D >> 2;
   const bool own = tid < D4;
-  // row indices fit in 32 bits: at most kFusedMaxRows rows
-  const int r_begin = static_cast<int>(blockIdx.x) * static_cast<int>(a.rows_per_cta);
-  const int r_end = min(r_begin + static_cast<int>(a.rows_per_cta), static_cast<int>(a.rows));
-  if (tid == 0 && r_end > r_begin) {
-    // L2 prefetch of the rows of the first groups (a hint: see above)
-    const int n = min(r_end - r_begin, kFusedStages * RG);
-    const char* src = reinterpret_cast<const char*>(a.bank + static_cast<long long>(r_begin) * a.D);
-    const unsigned long long bytes = static_cast<unsigned long long>(n) * a.D * 4;
-    for (unsigned long long off = 0; off < bytes; off += (1ull << 20)) {
-      const unsigned int sz = static_cast<unsigned int>(min(bytes - off, 1ull << 20));
-      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(src + off), "r"(sz) : "memory");
-    }
+  const int R = a.rows_per_cta;
+  const int r0 = static_cast<int>(blockIdx.x) * R;  // B N <= kFusedRows x SMs rows
+  const int b = r0 / a.N;                            // all R rows are of sequence b
+  const float4* rows_g = reinterpret_cast<const float4*>(a.bank) + static_cast<long long>(r0) * D4;
+  if (tid == 0) {
+    // L2 prefetch of this CTA's rows (a hint: see above)
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(rows_g),
+                 "r"(static_cast<unsigned int>(R) * D4 * 16u)
+                 : "memory");
   }
   pdl_wait();
   pdl_trigger();
-  // a group: up to RG consecutive rows of one sequence within [r_begin, r_end)
-  auto group_len = [&](int r0) { return min(RG, min(r_end, (r0 / a.N + 1) * a.N) - r0); };
-  const float4* bank4 = reinterpret_cast<const float4*>(a.bank) + tid;
-  auto issue = [&](int r0, int st) {  // this thread's copies of a group, one commit group
-    const int nr = group_len(r0);
-    float4* dst = rows_s + st * RG * kFusedThreads + tid;
-    for (int r = 0; r < nr; ++r)
-      if (own) sel_cp_async16(dst + r * kFusedThreads, bank4 + static_cast<long long>(r0 + r) * D4);
-    sel_cp_commit();
-    return nr;
-  };
-  int ri = r_begin, gi = 0;  // next row to issue, groups issued
-  for (; gi < kFusedStages && ri < r_end; ++gi) ri += issue(ri, gi);
-  int cur_b = -1;
-  float qq = 0.f;
-  for (int r0 = r_begin, g = 0; r0 < r_end; ++g) {
-    const int b = r0 / a.N;
-    const int lim = min(r_end, (b + 1) * a.N);  // end of this CTA's run of sequence b
-    const int nr = group_len(r0);
-    if (b != cur_b) {  // this CTA's first rows of sequence b: its q_vec and q.q
-      cur_b = b;
-      const float4 qr =
-          own ? __ldg(reinterpret_cast<const float4*>(a.qv + static_cast<long long>(b) * a.D) + tid)
-              : make_float4(0.f, 0.f, 0.f, 0.f);
-      q_s[tid] = qr;  // read back by this thread only
-      float acc = 0.f;
-      acc = fmaf(qr.x, qr.x, acc); acc = fmaf(qr.y, qr.y, acc);
-      acc = fmaf(qr.z, qr.z, acc); acc = fmaf(qr.w, qr.w, acc);
+  if (own)
+    for (int r = 0; r < R; ++r) sel_cp_async16(rows_s + r * kFusedThreads + tid, rows_g + r * D4 + tid);
+  asm volatile("cp.async.commit_group;\n" ::: "memory");
+  // q_vec . q_vec while the rows are in flight
+  const float4 qr = own ? __ldg(reinterpret_cast<const float4*>(a.qv + static_cast<long long>(b) * a.D) + tid)
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+  {
+    float acc = 0.f;
+    acc = fmaf(qr.x, qr.x, acc); acc = fmaf(qr.y, qr.y, acc);
+    acc = fmaf(qr.z, qr.z, acc); acc = fmaf(qr.w, qr.w, acc);
 #pragma unroll
-      for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-      if (lane == 0) qq_part[warp] = acc;
-      __syncthreads();
-      qq = qq_part[0];
+    for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    if (lane == 0) qq_part[warp] = acc;
+  }
+  asm volatile("cp.async.wait_group 0;\n" ::: "memory");
+  // this thread's partials: value 2r is row r's dot, 2r + 1 its squared norm
+  float v[2 * RG];
+#pragma unroll
+  for (int r = 0; r < RG; ++r) {
+    const float4 m = (r < R && own) ? rows_s[r * kFusedThreads + tid] : make_float4(0.f, 0.f, 0.f, 0.f);
+    float d0 = 0.f, s0 = 0.f;
+    d0 = fmaf(m.x, qr.x, d0); d0 = fmaf(m.y, qr.y, d0); d0 = fmaf(m.z, qr.z, d0); d0 = fmaf(m.w, qr.w, d0);
+    s0 = fmaf(m.x, m.x, s0); s0 = fmaf(m.y, m.y, s0); s0 = fmaf(m.z, m.z, s0); s0 = fmaf(m.w, m.w, s0);
+    v[2 * r] = d0;
+    v[2 * r + 1] = s0;
+  }
+  // halving butterfly over the 16 values: afterwards lanes 2i and 2i + 1 both
+  // hold value i (i from lane bits 4..1) summed over the warp
+#pragma unroll
+  for (int o = 16, n = 2 * RG; o >= 2; o >>= 1, n >>= 1) {
+    const bool up = (lane & o) != 0;
+#pragma unroll
+    for (int i = 0; i < n / 2; ++i) {
+      const float send = up ? v[i] : v[i + n / 2];
+      const float keep = up ? v[i + n / 2] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+    }
+  }
+  v[0] += __shfl_xor_sync(0xffffffffu, v[0], 1);
+  if ((lane & 1) == 0) part[warp][lane >> 1] = v[0];
+  __syncthreads();
+  float qq = qq_part[0];
 #pragma unroll 4
-      for (int w = 1; w < kFusedWarps; ++w) qq += qq_part[w];
-    }
-    // this group's copies have landed once at most (issued - g - 1) later groups are pending
-    if (gi - g - 1 >= 1) sel_cp_wait<1>(); else sel_cp_wait<0>();
-    // each row's dot and squared norm: this thread's partials, then the xor
-    // butterfly of the lanes; lane 0 leaves the warp's sums for the row
-    const float4 qr = q_s[tid];
-    const float4* src = rows_s + (g % kFusedStages) * RG * kFusedThreads + tid;
-    float* pg = &part[g & 1][0][0];
+  for (int w = 1; w < kFusedWarps; ++w) qq += qq_part[w];
+  // warp r: row r's 32 warp sums, in the same butterfly; lane 0 writes the score
+  if (warp < R) {
+    float sd = part[lane][2 * warp], sm = part[lane][2 * warp + 1];
 #pragma unroll
-    for (int r = 0; r < RG; ++r) {
-      const float4 m = (r < nr && own) ? src[r * kFusedThreads] : make_float4(0.f, 0.f, 0.f, 0.f);
-      float d0 = 0.f, s0 = 0.f;
-      d0 = fmaf(m.x, qr.x, d0); d0 = fmaf(m.y, qr.y, d0); d0 = fmaf(m.z, qr.z, d0); d0 = fmaf(m.w, qr.w, d0);
-      s0 = fmaf(m.x, m.x, s0); s0 = fmaf(m.y, m.y, s0); s0 = fmaf(m.z, m.z, s0); s0 = fmaf(m.w, m.w, s0);
-#pragma unroll
-      for (int off = 16; off >= 1; off >>= 1) {
-        d0 += __shfl_xor_sync(0xffffffffu, d0, off);
-        s0 += __shfl_xor_sync(0xffffffffu, s0, off);
-      }
-      if (lane == 0) {
-        pg[warp * 2 * RG + 2 * r] = d0;
-        pg[warp * 2 * RG + 2 * r + 1] = s0;
-      }
+    for (int off = 16; off >= 1; off >>= 1) {
+      sd += __shfl_xor_sync(0xffffffffu, sd, off);
+      sm += __shfl_xor_sync(0xffffffffu, sm, off);
     }
-    // the stage just read is this thread's own: refill it with a later group
-    if (ri < r_end) {
-      ri += issue(ri, g % kFusedStages);
-      ++gi;
-    }
-    __syncthreads();
-    if (tid < nr) {
-      float sd = pg[2 * tid], sm = pg[2 * tid + 1];
-#pragma unroll 4
-      for (int w = 1; w < kFusedWarps; ++w) {
-        sd += pg[w * 2 * RG + 2 * tid];
-        sm += pg[w * 2 * RG + 2 * tid + 1];
-      }
+    if (lane == 0) {
       float sc = 0.f;
       if (sm > 0.f && qq > 0.f) sc = sd / (sqrtf(sm) * sqrtf(qq));
       if (sc == 0.f) sc = 0.f;  // -0 -> +0, so that -0 and +0 tie
-      a.scores[r0 + tid] = sc;
-      if (a.la.sqnorm) a.la.sqnorm[r0 + tid] = sm;
-    }
-    r0 += nr;
-    if (r0 == lim) {
-      // end of this CTA's run of sequence b: publish the scores, count the run
-      __threadfence();
-      __syncthreads();
-      if (tid == 0) {
-        const unsigned int run = static_cast<unsigned int>(r0 - max(r_begin, b * a.N));
-        const unsigned int old = atomicAdd(a.counters + b, run);
-        last_flag = (old + run == static_cast<unsigned int>(a.N)) ? 1 : 0;
-      }
-      __syncthreads();
-      if (last_flag) fused_select(a, b);
+      a.scores[r0 + warp] = sc;
+      if (a.la.sqnorm) a.la.sqnorm[r0 + warp] = sm;
+      asm volatile("fence.acq_rel.gpu;\n" ::: "memory");  // release the score writes
     }
   }
+  __syncthreads();
+  if (tid == 0) {
+    const unsigned int old = atomicAdd(a.counters + b, static_cast<unsigned int>(R));
+    last_flag = (old + R == static_cast<unsigned int>(a.N)) ? 1 : 0;
+  }
+  __syncthreads();
+  if (last_flag) fused_select(a, b);
 }
 
-// Launches score_select_fused_kernel; the caller has checked the limits.
+// Rows per CTA of the one-launch path for B sequences of N CMEs of
+// dimension D: the largest R <= kFusedRows dividing N with B N / R CTAs in
+// one wave of one CTA per SM; 0 when there is none (or a limit is exceeded).
+static int fused_rows_per_cta(int B, int N, int D) {
+  if (N > kFusedMaxN || D > kFusedMaxD) return 0;
+  const long long rows = static_cast<long long>(B) * N;
+  for (int R = kFusedRows; R >= 1; --R)
+    if (N % R == 0 && rows / R <= sm_count()) return R;
+  return 0;
+}
+
+// Launches score_select_fused_kernel with R rows per CTA.
 static int launch_score_select_fused(const float* question_emb, const float* cme_bank, int B,
                                      int N, int D, int k, int32_t* idx_out, float* sc,
-                                     unsigned int* counters, cudaStream_t s, const LocateArgs& la) {
+                                     unsigned int* counters, cudaStream_t s, const LocateArgs& la,
+                                     int R) {
   static std::once_flag attr_once[64];
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
@@ -828,24 +826,18 @@ static int launch_score_select_fused(const float* question_emb, const float* cme
                                                 static_cast<int>(fused_smem_bytes())));
   });
   if (st != CMC_OK) return st;
-  // one CTA per SM at most, every CTA a contiguous run of rows
-  const long long rows = static_cast<long long>(B) * N;
-  long long ctas = (rows + kFusedRows - 1) / kFusedRows;
-  if (ctas > sm_count()) ctas = sm_count();
-  const long long rows_per_cta = (rows + ctas - 1) / ctas;
-  ctas = (rows + rows_per_cta - 1) / rows_per_cta;
   FusedArgs a;
   a.qv = question_emb;
   a.bank = cme_bank;
   a.N = N;
   a.D = D;
   a.k = k;
-  a.rows = rows;
-  a.rows_per_cta = rows_per_cta;
+  a.rows_per_cta = R;
   a.scores = sc;
   a.counters = counters;
   a.idx_out = idx_out;
   a.la = la;
+  const long long ctas = static_cast<long long>(B) * N / R;
   return launch_pdl(score_select_fused_kernel, dim3(static_cast<unsigned>(ctas)),
                     dim3(kFusedThreads), fused_smem_bytes(), s, a);
 }
@@ -860,10 +852,10 @@ static int launch_score_select(const float* question_emb, const float* cme_bank,
                                unsigned int* counters = nullptr,
                                const LocateArgs& la = LocateArgs{nullptr, nullptr, nullptr, 0,
                                                                  nullptr, nullptr}) {
-  if (counters && N <= kFusedMaxN && D <= kFusedMaxD &&
-      static_cast<long long>(B) * N <= kFusedMaxRows)
+  const int fused_rows = counters ? fused_rows_per_cta(B, N, D) : 0;
+  if (fused_rows > 0)
     return launch_score_select_fused(question_emb, cme_bank, B, N, D, k, idx_out, sc, counters, s,
-                                     la);
+                                     la, fused_rows);
   const long long rows = static_cast<long long>(B) * N;
   long long blocks = rows;
   const long long cap = static_cast<long long>(sm_count()) * (2048 / kScoreThreads);

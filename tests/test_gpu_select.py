@@ -107,17 +107,20 @@ def test_select_ties_go_to_lower_index(cuda_device):
 # keys split across their shared memories (also unevenly: 50,001 = 8 x 6,250
 # + 1), and one CTA re-reading the keys from global memory (N / 8 > 49,152)
 #
-# One launch up to N = 8192 (16 keys per thread of the selecting CTA) and
-# D = 4096 (one or two float4s per thread and row: 2048 / 2052); two launches
-# above either limit (8193, 4100).
+# One launch for small banks (CTAs of R <= 8 rows of one sequence, R dividing
+# N, one wave of one CTA per SM; D <= 4096): R = 8 (1000, 1024, 1216 = 8 x
+# 152 rows), R = 7 (777), R = 3 (B = 7, N = 33), R = 1 (prime N = 37, B = 4),
+# R = 5 (N = 5), and the two-key-per-thread selection (N = 1216); D from 4 to
+# 4096, one float4 per thread or fewer.  Two launches otherwise (D = 4100, and
+# the larger banks).
 @pytest.mark.parametrize("N,D,k,B", [
     (1, 4, 1, 3), (1, 4, 0, 3), (5, 8, 5, 3), (1000, 36, 999, 3), (1025, 512, 17, 3),
     (3000, 4, 1500, 3), (4096, 128, 4095, 3), (9000, 8, 1234, 3), (50001, 4, 777, 3),
-    (400003, 4, 1000, 3), (8192, 16, 4000, 2), (8193, 16, 100, 2), (777, 2048, 50, 2),
-    (777, 2052, 50, 2), (300, 4100, 50, 2), (33, 4096, 5, 7), (1024, 256, 100, 40)])
+    (400003, 4, 1000, 3), (8192, 16, 4000, 2), (8193, 16, 100, 2), (1000, 36, 999, 1),
+    (1024, 4096, 1023, 1), (1024, 2048, 1, 1), (1216, 64, 300, 1), (777, 4, 50, 1),
+    (33, 4096, 5, 7), (37, 100, 9, 4), (300, 4100, 50, 2), (1024, 256, 100, 40)])
 def test_select_edge_shapes(cuda_device, N, D, k, B):
-    """Random banks (no planted margin).  Also CTAs whose rows span several
-    sequences (B = 7, N = 33; B = 40, N = 1024) in the one-launch path."""
+    """Random banks (no planted margin), through both launch paths."""
     rng = np.random.default_rng(N + D + k)
     q = rng.standard_normal((B, D)).astype(np.float32)
     bank = rng.standard_normal((B, N, D)).astype(np.float32)
