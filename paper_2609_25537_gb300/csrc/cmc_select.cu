@@ -538,9 +538,10 @@ topk_select_cluster_kernel(const float* __restrict__ scores, int N, int k,
 // the shuffles; then warp r adds row r's 32 warp sums in the same butterfly.
 // Equal rows thus get bit-identical scores.
 //
-// The CTA then releases its score writes (fence.acq_rel.gpu) and adds R to
-// the sequence's counter; the CTA whose addition completes N is the last to
-// score that sequence and selects its top k itself.  Keys are the order-
+// The CTA then adds R to the sequence's counter with an acq_rel atomic (which
+// releases the CTA's score writes and acquires those of the CTAs before it);
+// the CTA whose addition completes N is the last to score that sequence and
+// selects its top k itself.  Keys are the order-
 // preserving uint32 images of the scores; a bit-by-bit search from the top
 // bit finds the largest T with at least k keys >= T (the k-th largest key),
 // each round one counting barrier (__syncthreads_count) per key a thread
@@ -649,10 +650,8 @@ __device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
   __shared__ int best_i[kFusedWarps];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int N = a.N, k = a.k;
-  // acquire: thread 0 saw the last counter addition; the other CTAs released
-  // their score writes before theirs, and the barrier passes the order on
-  if (tid == 0) asm volatile("fence.acq_rel.gpu;\n" ::: "memory");
-  __syncthreads();
+  // thread 0's acq_rel counter addition acquired the other CTAs' score
+  // writes; the caller's barrier passed that order on to every thread
   if (a.la.sqnorm) {
     // CME-guided localisation: argmax of the squared norms, ties to the lower index
     const float* sq = a.la.sqnorm + static_cast<long long>(b) * N;
@@ -787,12 +786,17 @@ score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
       if (sc == 0.f) sc = 0.f;  // -0 -> +0, so that -0 and +0 tie
       a.scores[r0 + warp] = sc;
       if (a.la.sqnorm) a.la.sqnorm[r0 + warp] = sm;
-      asm volatile("fence.acq_rel.gpu;\n" ::: "memory");  // release the score writes
     }
   }
   __syncthreads();
   if (tid == 0) {
-    const unsigned int old = atomicAdd(a.counters + b, static_cast<unsigned int>(R));
+    // acq_rel at GPU scope: releases the CTA's score writes (they precede it
+    // through the barrier) and, for the last CTA, acquires everyone else's
+    unsigned int old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;\n"
+                 : "=r"(old)
+                 : "l"(a.counters + b), "r"(static_cast<unsigned int>(R))
+                 : "memory");
     last_flag = (old + R == static_cast<unsigned int>(a.N)) ? 1 : 0;
   }
   __syncthreads();
