@@ -33,10 +33,14 @@
 // bytes (expect_tx / complete_tx) and its cp.async copies
 // (cp.async.mbarrier.arrive) have landed; four consumer warps, each owning 16
 // keys of a tile, compute
-//   S = Q K^T   with mma.sync m16n8k16 (query heads as the M rows: the G
-//               heads sharing the KV head, padded to 16),
+//   S^T = K Q^T   with mma.sync m16n8k16: the warp's 16 keys as the M rows,
+//                 the G query heads sharing the KV head as the N = 8 columns
+//                 (padded to 8), d in k-steps of 16,
 // an online softmax in the log2 domain (running max / sum per head), and
-//   O += P V    with mma.sync, P taken straight from the S accumulators,
+//   O^T += V^T P^T  with mma.sync: 16 rows of the head dimension per m-tile,
+//                 the heads as columns, the 16 keys as the k-step; P^T comes
+//                 from the S^T accumulators, packed to bf16 and transposed in
+//                 registers (movmatrix),
 // reading K with ldmatrix and V with ldmatrix.trans, then hand the stage back
 // through an "empty" mbarrier.  Every mbarrier wait has a wall-time limit.
 // Warps are merged in shared memory at the end of a unit.
@@ -137,15 +141,22 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t&
                : "r"(addr));
 }
 
-// C[16x8] += A[16x16] B[16x8], bf16 inputs, fp32 accumulators.  A rows 8..15
-// are the padding heads (always zero), so a1 = a3 = 0.
-__device__ __forceinline__ void mma_rows0to7(float (&c)[4], uint32_t a0, uint32_t a2, uint32_t b0,
-                                             uint32_t b1) {
+// C[16x8] += A[16x16] B[16x8], bf16 inputs, fp32 accumulators (all 16 rows of A).
+__device__ __forceinline__ void mma_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                          uint32_t a3, uint32_t b0, uint32_t b1) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
       "{%8,%9}, {%0,%1,%2,%3};\n"
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a0), "r"(0u), "r"(a2), "r"(0u), "r"(b0), "r"(b1));
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Transpose of an 8x8 matrix of 16-bit elements held one pair per thread
+// (thread l: row l/4, columns 2(l%4) and 2(l%4)+1).
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;\n" : "=r"(d) : "r"(a));
+  return d;
 }
 
 // 2^x with the ex2.approx instruction (ex2(-inf) = +0).
@@ -325,12 +336,17 @@ struct Stage {
 // bit masks of rows 0-31 / 32-63 whose Tier-1 index is out of range.
 enum { H_NROWS = 0, H_NEWSLOT = 1, H_NEWROW = 2, H_MASKED = 3, H_BADLO = 4, H_BADHI = 5 };
 
+// Row length (floats) of the end-of-unit merge buffer: d + 4, so that the
+// rows of the four head pairs a warp stores to start 8 banks apart and its
+// 32 lanes hit distinct banks.
+__host__ __device__ constexpr int merge_row_floats(int D) { return D + 4; }
+
 template <int D, int G, int NST, bool ROPE>
 constexpr size_t attn_smem_bytes() {
   return 1024 /* alignment slack */ +
          static_cast<size_t>(NST) * (Stage<D, G, ROPE>::kBytes + Stage<D, G, ROPE>::kAuxBytes) +
          kMetaSlots * (kTileKeys * 4 + 16) +
-         static_cast<size_t>(kWarps) * (2 * 8 + G * D) * sizeof(float);
+         static_cast<size_t>(kWarps) * (2 * 8 + G * merge_row_floats(D)) * sizeof(float);
 }
 
 // Byte offset of 16-byte chunk c (0 .. D/8-1) of tile row r within a K or V
@@ -676,7 +692,7 @@ __global__ void __launch_bounds__(kThreads + 32)
 two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) {
   using S = Stage<D, G, ROPE>;
   constexpr int KS = D / 16;  // k-steps of the Q K^T product
-  constexpr int NT = D / 8;   // n8 tiles of the output
+  constexpr int DP = merge_row_floats(D);  // padded row of the merge buffer
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* aux0 = smem + NST * S::kBytes;                              // NST aux areas
@@ -841,16 +857,25 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
   }
 
   // ======================= consumer warps =======================
-  const int gq = lane >> 2;  // mma row (query head within the group)
-  const int tq = lane & 3;   // mma column pair
+  // Both products take the warp's 16 keys (S^T = K Q^T) or 16 rows of the
+  // head dimension (O^T = V^T P^T) as the M rows of m16n8k16 and the query
+  // heads of the group as the N = 8 columns, so no M row is padding.
+  // Fragment coordinates: gq = lane / 4, tq = lane % 4.  S^T: keys gq and
+  // gq + 8 of the warp's 16, heads 2 tq and 2 tq + 1.  O^T m-tile mt: head
+  // dimension rows 16 mt + gq and 16 mt + 8 + gq, heads 2 tq and 2 tq + 1.
+  // A thread keeps the running max and sum of heads 2 tq and 2 tq + 1
+  // (heads >= G are padding: zero queries, never written out).
+  const int gq = lane >> 2;
+  const int tq = lane & 3;
+  constexpr int MT = D / 16;  // m-tiles of O^T
   TileCursor cc;
   cc.init(t_begin, p);
   int cur_u = -1;
-  uint32_t qa[KS][2];
-  float m_run = -INFINITY, l_run = 0.f;
-  float o[NT][4];
+  uint32_t qa[KS][2];  // Q^T fragments (B operand): head gq, columns of k-step ks
+  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
+  float o[MT][4];
 #pragma unroll
-  for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+  for (int j = 0; j < MT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
 #pragma unroll
   for (int ks = 0; ks < KS; ++ks) qa[ks][0] = qa[ks][1] = 0u;
 
@@ -935,10 +960,10 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
           }
         }
       }
-      m_run = -INFINITY;
-      l_run = 0.f;
+      m_run[0] = m_run[1] = -INFINITY;
+      l_run[0] = l_run[1] = 0.f;
 #pragma unroll
-      for (int j = 0; j < NT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+      for (int j = 0; j < MT; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
     }
 
     if (n_rows > 0) {
@@ -957,68 +982,74 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
       }
       const uint32_t sK = smem_addr(stage + S::kK);
       const uint32_t sV = smem_addr(stage + S::kV);
-      // ---- S = Q K^T over this warp's 16 keys: two n8 blocks, two chains each ----
-      float sa[2][4], sb[2][4];
-#pragma unroll
-      for (int nb = 0; nb < 2; ++nb)
-#pragma unroll
-        for (int e = 0; e < 4; ++e) sa[nb][e] = sb[nb][e] = 0.f;
-#pragma unroll
-      for (int ks = 0; ks < KS; ks += 2) {
-#pragma unroll
-        for (int nb = 0; nb < 2; ++nb) {
-          const int key = 16 * warp + 8 * nb + (lane & 7);
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4(sK + swz(key, 2 * ks + (lane >> 3)), b0, b1, b2, b3);
-          mma_rows0to7(sa[nb], qa[ks][0], qa[ks][1], b0, b1);
-          mma_rows0to7(sb[nb], qa[ks + 1][0], qa[ks + 1][1], b2, b3);
-        }
-      }
-      // ---- online softmax (log2 domain) ----
-      float v[2][2];
-      float mx = -INFINITY;
-#pragma unroll
-      for (int nb = 0; nb < 2; ++nb) {
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int kk = 16 * warp + 8 * nb + 2 * tq + e;
-          const bool ok = (keys >> kk) & 1ull;
-          v[nb][e] = ok ? (sa[nb][e] + sb[nb][e]) * p.scale_log2 : -INFINITY;
-          mx = fmaxf(mx, v[nb][e]);
-        }
-      }
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      const float m_new = fmaxf(m_run, mx);
-      float alpha = 1.f;
-      float pr[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
-      if (m_new != -INFINITY) {
-        alpha = ex2(m_run - m_new);
-#pragma unroll
-        for (int nb = 0; nb < 2; ++nb)
-#pragma unroll
-          for (int e = 0; e < 2; ++e) pr[nb][e] = ex2(v[nb][e] - m_new);
-      }
-      m_run = m_new;
-      l_run = l_run * alpha + (pr[0][0] + pr[0][1]) + (pr[1][0] + pr[1][1]);
-      if (!__all_sync(0xffffffffu, alpha == 1.f)) {
-#pragma unroll
-        for (int j = 0; j < NT; ++j) {
-          o[j][0] *= alpha;
-          o[j][1] *= alpha;
-        }
-      }
-      // ---- O += P V ----
-      const uint32_t pa0 = pack_bf16_rn(pr[0][0], pr[0][1]);
-      const uint32_t pa2 = pack_bf16_rn(pr[1][0], pr[1][1]);
+      // ---- S^T = K Q^T over this warp's 16 keys: 16 x 8 per k-step, two chains ----
+      float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
       {
+        // ldmatrix x4: lanes 0-7 / 8-15 / 16-23 / 24-31 address keys 0-7 / 8-15 /
+        // 0-7 / 8-15 at columns 16 ks .. +7 / same / 16 ks + 8 .. +15 / same
         const int key = 16 * warp + (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
-        for (int j = 0; j < NT; j += 2) {
-          uint32_t b0, b1, b2, b3;
-          ldsm_x4_t(sV + swz(key, j + (lane >> 4)), b0, b1, b2, b3);
-          mma_rows0to7(o[j], pa0, pa2, b0, b1);
-          mma_rows0to7(o[j + 1], pa0, pa2, b2, b3);
+        for (int ks = 0; ks < KS; ++ks) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4(sK + swz(key, 2 * ks + (lane >> 4)), a0, a1, a2, a3);
+          if (ks & 1) mma_16816(sb, a0, a1, a2, a3, qa[ks][0], qa[ks][1]);
+          else mma_16816(sa, a0, a1, a2, a3, qa[ks][0], qa[ks][1]);
+        }
+      }
+      // ---- online softmax (log2 domain), heads 2 tq and 2 tq + 1 ----
+      const bool ok0 = (keys >> (16 * warp + gq)) & 1ull;
+      const bool ok1 = (keys >> (16 * warp + gq + 8)) & 1ull;
+      float v[4];
+      v[0] = ok0 ? (sa[0] + sb[0]) * p.scale_log2 : -INFINITY;
+      v[1] = ok0 ? (sa[1] + sb[1]) * p.scale_log2 : -INFINITY;
+      v[2] = ok1 ? (sa[2] + sb[2]) * p.scale_log2 : -INFINITY;
+      v[3] = ok1 ? (sa[3] + sb[3]) * p.scale_log2 : -INFINITY;
+      float mx0 = fmaxf(v[0], v[2]), mx1 = fmaxf(v[1], v[3]);
+#pragma unroll
+      for (int off = 4; off < 32; off <<= 1) {  // over the 8 key rows (lane bits 2-4)
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, off));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, off));
+      }
+      const float mn0 = fmaxf(m_run[0], mx0), mn1 = fmaxf(m_run[1], mx1);
+      float alpha0 = 1.f, alpha1 = 1.f;
+      float pr[4] = {0.f, 0.f, 0.f, 0.f};
+      if (mn0 != -INFINITY) {
+        alpha0 = ex2(m_run[0] - mn0);
+        pr[0] = ex2(v[0] - mn0);
+        pr[2] = ex2(v[2] - mn0);
+      }
+      if (mn1 != -INFINITY) {
+        alpha1 = ex2(m_run[1] - mn1);
+        pr[1] = ex2(v[1] - mn1);
+        pr[3] = ex2(v[3] - mn1);
+      }
+      m_run[0] = mn0;
+      m_run[1] = mn1;
+      l_run[0] = l_run[0] * alpha0 + (pr[0] + pr[2]);
+      l_run[1] = l_run[1] * alpha1 + (pr[1] + pr[3]);
+      if (!__all_sync(0xffffffffu, alpha0 == 1.f && alpha1 == 1.f)) {
+#pragma unroll
+        for (int j = 0; j < MT; ++j) {
+          o[j][0] *= alpha0;
+          o[j][1] *= alpha1;
+          o[j][2] *= alpha0;
+          o[j][3] *= alpha1;
+        }
+      }
+      // ---- O^T += V^T P^T ----
+      // P^T as the B operand: the S^T fragments (keys gq / gq + 8, heads
+      // 2 tq, 2 tq + 1) packed to bf16 and transposed (head gq, keys 2 tq, +1)
+      const uint32_t pb0 = movmatrix_trans(pack_bf16_rn(pr[0], pr[1]));
+      const uint32_t pb1 = movmatrix_trans(pack_bf16_rn(pr[2], pr[3]));
+      {
+        // ldmatrix x4 .trans of V: lanes 0-7 / 8-15 / 16-23 / 24-31 address
+        // keys 0-7 / 0-7 / 8-15 / 8-15 at columns 16 mt .. +7 / 16 mt + 8 .. +15 / ...
+        const int key = 16 * warp + (lane & 7) + ((lane >> 4) & 1) * 8;
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+          uint32_t a0, a1, a2, a3;
+          ldsm_x4_t(sV + swz(key, 2 * mt + ((lane >> 3) & 1)), a0, a1, a2, a3);
+          mma_16816(o[mt], a0, a1, a2, a3, pb0, pb1);
         }
       }
     }
@@ -1033,23 +1064,31 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     // ---- end of a unit within this CTA: merge warps, write out or a partial ----
     const bool unit_end = (i + 1 == n_tiles) || (cc.j == p.tpu - 1);
     if (unit_end) {
-      // Merge the four warps' states of each head: every warp rescales its
-      // output and sum to the heads' common running max, then each thread
-      // adds four columns across the warps in a fixed order.
-      l_run += __shfl_xor_sync(0xffffffffu, l_run, 1);
-      l_run += __shfl_xor_sync(0xffffffffu, l_run, 2);
-      if (gq < G && tq == 0) merge_m[warp * 8 + gq] = m_run;
-      consumer_sync();
-      if (gq < G) {
-        float M = merge_m[gq];
+      // Merge the four warps' states of each head: every warp leaves its
+      // running max, sum and unnormalised output (rows of DP floats, padded so
+      // that the warp's stores hit distinct banks); after one barrier each
+      // thread takes four columns of one head, rescales the warps' outputs and
+      // sums to the heads' common max and adds them in warp order.
 #pragma unroll
-        for (int w = 1; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + gq]);
-        const float f = (M == -INFINITY) ? 0.f : ex2(m_run - M);
-        float* ow = merge_o + (warp * G + gq) * D;
+      for (int off = 4; off < 32; off <<= 1) {  // sums over the 8 key rows
+        l_run[0] += __shfl_xor_sync(0xffffffffu, l_run[0], off);
+        l_run[1] += __shfl_xor_sync(0xffffffffu, l_run[1], off);
+      }
 #pragma unroll
-        for (int j = 0; j < NT; ++j)
-          *reinterpret_cast<float2*>(ow + 8 * j + 2 * tq) = make_float2(o[j][0] * f, o[j][1] * f);
-        if (tq == 0) merge_l[warp * 8 + gq] = l_run * f;
+      for (int e = 0; e < 2; ++e) {
+        const int hh = 2 * tq + e;
+        if (hh < G) {
+          float* ow = merge_o + (warp * G + hh) * DP;
+#pragma unroll
+          for (int j = 0; j < MT; ++j) {
+            ow[16 * j + gq] = o[j][e];
+            ow[16 * j + 8 + gq] = o[j][2 + e];
+          }
+          if (gq == 0) {
+            merge_m[warp * 8 + hh] = m_run[e];
+            merge_l[warp * 8 + hh] = l_run[e];
+          }
+        }
       }
       consumer_sync();
 
@@ -1070,16 +1109,23 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
         if (x >= NGR) break;
         const int hh = (4 * x) / D;
         const int c = (4 * x) % D;
-        float4 acc = *reinterpret_cast<const float4*>(merge_o + hh * D + c);
-        float Ls = merge_l[hh];
+        float M = merge_m[hh];
 #pragma unroll
-        for (int w = 1; w < kWarps; ++w) {
-          const float4 v = *reinterpret_cast<const float4*>(merge_o + (w * G + hh) * D + c);
-          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
-          Ls += merge_l[w * 8 + hh];
+        for (int w = 1; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + hh]);
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        float Ls = 0.f;
+        if (M != -INFINITY) {
+#pragma unroll
+          for (int w = 0; w < kWarps; ++w) {
+            const float f = ex2(merge_m[w * 8 + hh] - M);
+            const float4 v = *reinterpret_cast<const float4*>(merge_o + (w * G + hh) * DP + c);
+            acc.x = fmaf(f, v.x, acc.x); acc.y = fmaf(f, v.y, acc.y);
+            acc.z = fmaf(f, v.z, acc.z); acc.w = fmaf(f, v.w, acc.w);
+            Ls = fmaf(f, merge_l[w * 8 + hh], Ls);
+          }
         }
         if (whole) {
-          const float inv = Ls > 0.f ? __frcp_rn(Ls) : 0.f;
+          const float inv = Ls > 0.f ? __fdividef(1.f, Ls) : 0.f;
           *reinterpret_cast<uint2*>(p.out + out_base + hh * D + c) =
               make_uint2(pack_bf16_rn(acc.x * inv, acc.y * inv), pack_bf16_rn(acc.z * inv, acc.w * inv));
         } else if (clus) {  // merged across the cluster below
@@ -1089,9 +1135,6 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
           constexpr int PW = rec_floats(G, D);
           float* rec = p.partials + (ut0 + (ut0 > t_begin ? 0 : t_begin - ut0)) * PW;
           if (c == 0) {
-            float M = merge_m[hh];
-#pragma unroll
-            for (int w = 1; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + hh]);
             rec[hh] = M;
             rec[G + hh] = Ls;
           }
@@ -1113,7 +1156,7 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
           if (x >= NGR) break;
           const int hh = (4 * x) / D;
           const int c = (4 * x) % D;
-          if (c == 0) {
+          if (c == 0) {  // merge_m still holds the warps' maxima
             float M = merge_m[hh];
 #pragma unroll
             for (int w = 1; w < kWarps; ++w) M = fmaxf(M, merge_m[w * 8 + hh]);
