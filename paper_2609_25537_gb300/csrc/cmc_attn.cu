@@ -982,8 +982,12 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
       }
       const uint32_t sK = smem_addr(stage + S::kK);
       const uint32_t sV = smem_addr(stage + S::kV);
-      // ---- S^T = K Q^T over this warp's 16 keys: 16 x 8 per k-step, two chains ----
-      float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
+      // ---- S^T = K Q^T over this warp's 16 keys: 16 x 8 per k-step, in
+      // four independent accumulator chains (the last tile's latency is on
+      // every launch's critical path) ----
+      float sacc[4][4];
+#pragma unroll
+      for (int cidx = 0; cidx < 4; ++cidx) sacc[cidx][0] = sacc[cidx][1] = sacc[cidx][2] = sacc[cidx][3] = 0.f;
       {
         // ldmatrix x4: lanes 0-7 / 8-15 / 16-23 / 24-31 address keys 0-7 / 8-15 /
         // 0-7 / 8-15 at columns 16 ks .. +7 / same / 16 ks + 8 .. +15 / same
@@ -992,9 +996,14 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
         for (int ks = 0; ks < KS; ++ks) {
           uint32_t a0, a1, a2, a3;
           ldsm_x4(sK + swz(key, 2 * ks + (lane >> 4)), a0, a1, a2, a3);
-          if (ks & 1) mma_16816(sb, a0, a1, a2, a3, qa[ks][0], qa[ks][1]);
-          else mma_16816(sa, a0, a1, a2, a3, qa[ks][0], qa[ks][1]);
+          mma_16816(sacc[ks & 3], a0, a1, a2, a3, qa[ks][0], qa[ks][1]);
         }
+      }
+      float sa[4], sb[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        sa[e] = sacc[0][e] + sacc[2][e];
+        sb[e] = sacc[1][e] + sacc[3][e];
       }
       // ---- online softmax (log2 domain), heads 2 tq and 2 tq + 1 ----
       const bool ok0 = (keys >> (16 * warp + gq)) & 1ull;
@@ -1397,11 +1406,13 @@ static bool encode_rows(CUtensorMap* map, const void* base, long long rows, int 
 // ~110 KB of shared memory at d = 128, G <= 4, so two CTAs share an SM.
 constexpr int kStages = 3;
 // Box tiles per CTA prefetched into L2 before the grid dependency wait.  With
-// the streamed K/V loads marked evict-first, four tiles (128 KB per CTA, half
-// of them in free slots while the previous launch runs, the rest in its tail)
-// measured best at the model shapes; without the evict-first policy one tile
-// was best and deeper prefetch slower.
-constexpr int kL2PrefetchTiles = 4;
+// the streamed K/V loads marked evict-first, five tiles (160 KB per CTA, some
+// in free slots while the previous launch runs, most in its tail) measured
+// best at the Llama-3-8B shape (14.20 us against 14.34 for four, 14.30 for six,
+// 14.7 for three or eight); without the evict-first policy one tile was best.
+// A rolling prefetch a few tiles ahead of the TMA issue, on top, was slower at
+// every distance (16.2-16.9 us).
+constexpr int kL2PrefetchTiles = 5;
 
 // Launch plan of one attention call on the current device.
 struct AttnPlan {
