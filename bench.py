@@ -33,7 +33,7 @@ Reported (one JSON line on rank 0):
   e2e            the same metric through the Python API with host buffers
                  (question vector, CME bank and every step's q / new K,V
                  copied in from pinned memory, every step's output copied out,
-                 one copy each way per round of R decode steps);
+                 by one staging-copy launch per round of R decode steps);
   cpu_baseline   the fp64 oracle on the host, on a bounded sample.
 
 `--impl reference` times the fp64 oracle alone on the host cores (the
@@ -709,12 +709,15 @@ def run_e2e(args, w, reqs, dev, stream, world):
     the new token's K,V are copied in from pinned host memory and the output
     copied back to pinned host memory.  As a serving loop would, each
     scheduling round (one decode step of each of the R requests) moves its
-    inputs in one host-to-device copy and its outputs in one device-to-host
-    copy, on two side streams, double-buffered by round parity: the copy in
-    of round p+1 overlaps the decode kernels of round p, and only the first
-    decode of a round waits on a copy (the others follow their predecessor by
-    programmatic dependent launch).  P rounds are captured in one CUDA graph.
-    Selection and compaction run eagerly."""
+    inputs in together, and a round's outputs go out together: one staging-copy
+    launch per round (cmc.stage_copies) on the decode stream carries the
+    inputs of this round and the outputs of the round two back.  It copies
+    without waiting for the decode before it (inputs double-buffered, outputs
+    triple-buffered, so that decode never touches what it copies) and
+    completes after it, so every decode launch keeps programmatic dependent
+    launch and the copies overlap decode work.  A last launch after the P
+    rounds carries the last two rounds' outputs.  P rounds are captured in one
+    CUDA graph.  Selection and compaction run eagerly."""
     import paper_2609_25537_gb300 as cmc
     R, T, P = args.requests, args.decode_steps, args.pool
     steps = max(1, min(args.steps, args.e2e_steps))
@@ -728,49 +731,24 @@ def run_e2e(args, w, reqs, dev, stream, world):
     host_out = torch.empty((P, R) + out_shape, dtype=torch.bfloat16).pin_memory()
     host_sel = [(r.qemb.cpu().pin_memory(), r.bank.cpu().pin_memory()) for r in reqs]
     in_d = [torch.empty(R * per_req, dtype=torch.bfloat16, device=dev) for _ in range(2)]
-    out_d = [torch.empty((R,) + out_shape, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    out_d = [torch.empty((R,) + out_shape, dtype=torch.bfloat16, device=dev) for _ in range(3)]
 
     def views(par, i):
         base = in_d[par][i * per_req:(i + 1) * per_req]
         return (base[:nq].view(reqs[i].q[0].shape), base[nq:nq + nk].view(reqs[i].k_new[0].shape),
                 base[nq + nk:].view(reqs[i].v_new[0].shape))
 
-    s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
-
     def rounds():
-        """P rounds with their copies; returns after joining the side streams
-        back into `stream`."""
-        fork = torch.cuda.Event()
-        fork.record(stream)
-        s_in.wait_event(fork)
-        s_out.wait_event(fork)
-        decoded = [None, None]  # last round's decodes per buffer parity (inputs free)
-        copied = [None, None]   # last read-back per parity (output buffers free)
         for p in range(P):
-            par = p & 1
-            with torch.cuda.stream(s_in):
-                for ev in (decoded[par], copied[par]):
-                    if ev is not None:
-                        s_in.wait_event(ev)
-                in_d[par].copy_(host_in[p], non_blocking=True)
-                ready = torch.cuda.Event()
-                ready.record(s_in)
-            stream.wait_event(ready)
-            with torch.cuda.stream(stream):
-                for i, r in enumerate(reqs):
-                    q, k, v = views(par, i)
-                    r.decode(p, q=q, k_new=k, v_new=v, mode=args.tier1, out=out_d[par][i])
-            decoded[par] = torch.cuda.Event()
-            decoded[par].record(stream)
-            with torch.cuda.stream(s_out):
-                s_out.wait_event(decoded[par])
-                host_out[p].copy_(out_d[par], non_blocking=True)
-                copied[par] = torch.cuda.Event()
-                copied[par].record(s_out)
-        for side in (s_in, s_out):
-            j = torch.cuda.Event()
-            j.record(side)
-            stream.wait_event(j)
+            pairs = [(host_in[p], in_d[p % 2])]
+            if p >= 2:
+                pairs.append((out_d[(p - 2) % 3], host_out[p - 2]))
+            cmc.stage_copies(pairs, device=dev)
+            for i, r in enumerate(reqs):
+                q, k, v = views(p % 2, i)
+                r.decode(p, q=q, k_new=k, v_new=v, mode=args.tier1, out=out_d[p % 3][i])
+        tail = [(out_d[(p - 1) % 3], host_out[p - 1]) for p in (P - 1, P) if p >= 1]
+        cmc.stage_copies(tail, wait_first=True, device=dev)
 
     graph = None
     try:
@@ -809,7 +787,8 @@ def run_e2e(args, w, reqs, dev, stream, world):
     return {"value": world * steps * R * w.B * T / el, "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
             "per_step_graph": graph is not None,
-            "copies": "one host-to-device and one device-to-host copy per round of R decode steps"}
+            "copies": ("per round of R decode steps, one staging-copy launch on the decode "
+                       "stream: this round's inputs in, the outputs of the round two back out")}
 
 
 def run_ablation(args, dev):

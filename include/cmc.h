@@ -380,6 +380,44 @@ CMC_API int cmc_decode_step_rope(const void* q, const void* tier1_k, const void*
 CMC_API int cmc_read_status(void* workspace, int clear, uint32_t* flags, void* stream);
 
 /* ------------------------------------------------------------------------ *
+ * Staging copies for a serving loop (not a step of the paper's method: the  *
+ * input and output traffic of the decode loop around it)                    *
+ * ------------------------------------------------------------------------ */
+
+/* One byte range to copy. */
+typedef struct cmc_copy {
+  const void* src; /* device memory, or pinned host memory the device can address */
+  void* dst;       /* likewise                                                     */
+  size_t bytes;    /* a multiple of 16; src and dst 16-byte aligned                */
+} cmc_copy;
+
+/*
+ * Copies up to 4 byte ranges in one kernel launch, with 16-byte loads and
+ * stores, so either side may be pinned host memory (cudaHostAlloc, or
+ * cudaHostRegister with cudaHostRegisterMapped: on systems with unified
+ * addressing its host address is also its device address).  This moves the
+ * per-step inputs in and outputs out of a decode loop without a copy engine:
+ * a copy-engine copy between two kernels on the stream, or a wait on another
+ * stream's copy, ends programmatic dependent launch for the kernel after it,
+ * and with it the overlap of that kernel's start with its predecessor's end.
+ *
+ * wait_first == 0: the copies start without waiting for the work enqueued
+ * before them on `stream`, and the launch completes only after that work
+ * (it waits at its end), so the copies overlap the preceding kernel and
+ * everything enqueued after the call sees both.  The caller guarantees that
+ * the preceding work neither writes any source nor reads or writes any
+ * destination (double-buffer the device buffers).
+ * wait_first != 0: the copies start after the preceding work, like an
+ * ordinary stream operation.
+ *
+ * Errors: n outside [0, 4] -> CMC_ERR_RANGE; copies NULL with n > 0, or a NULL
+ * src / dst with bytes > 0 -> CMC_ERR_NULL; misaligned pointer or size ->
+ * CMC_ERR_ALIGN.  Copies of 0 bytes are skipped.  The library does not check
+ * that a host pointer is pinned and mapped: an unmapped one faults.
+ */
+CMC_API int cmc_stage_copies(const cmc_copy* copies, int n, int wait_first, void* stream);
+
+/* ------------------------------------------------------------------------ *
  * Allocation-free Tier-1 selection                                          *
  * ------------------------------------------------------------------------ */
 

@@ -32,6 +32,7 @@ EXPORTS = (
     "cmc_tier1_gather",
     "cmc_decode_attn_plan",
     "cmc_read_status",
+    "cmc_stage_copies",
     "cmc_score_select_static",
 )
 
@@ -48,6 +49,11 @@ STATUS = {
 DEVFLAG_BAD_INDEX = 1
 DEVFLAG_BAD_POS = 2
 DEVFLAG_TIMEOUT = 4
+
+
+class CmcCopy(ctypes.Structure):
+    """Mirror of `cmc_copy` (include/cmc.h)."""
+    _fields_ = [("src", ctypes.c_void_p), ("dst", ctypes.c_void_p), ("bytes", ctypes.c_size_t)]
 
 
 class CmcDims(ctypes.Structure):
@@ -100,6 +106,7 @@ _SIGNATURES = {
     "cmc_tier1_gather": (_i, [_vp, _vp, _vp, _dims_p, _vp, _vp, _vp, _vp]),
     "cmc_decode_attn_plan": (_i, [_dims_p, _i, ctypes.POINTER(_i), ctypes.POINTER(_i)]),
     "cmc_read_status": (_i, [_vp, _i, ctypes.POINTER(ctypes.c_uint32), _vp]),
+    "cmc_stage_copies": (_i, [_vp, _i, _i, _vp]),
     "cmc_score_select_static": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),
 }
 

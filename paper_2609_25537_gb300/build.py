@@ -19,7 +19,7 @@ CSRC = os.path.join(PKG_DIR, "csrc")
 BUILD_DIR = os.path.join(PKG_DIR, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "libcmc.so")
 
-SOURCES = ["cmc_abi.cu", "cmc_select.cu", "cmc_attn.cu", "cmc_bridge.cu", "cmc_denoise.cu"]
+SOURCES = ["cmc_abi.cu", "cmc_select.cu", "cmc_attn.cu", "cmc_bridge.cu", "cmc_denoise.cu", "cmc_io.cu"]
 
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON_FLAGS = [

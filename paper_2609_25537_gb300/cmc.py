@@ -26,7 +26,7 @@ from typing import Dict, Optional, Tuple
 
 import torch
 
-from ._lib import CmcDims, check, lib, DEVFLAG_BAD_INDEX, DEVFLAG_BAD_POS, DEVFLAG_TIMEOUT
+from ._lib import CmcCopy, CmcDims, check, lib, DEVFLAG_BAD_INDEX, DEVFLAG_BAD_POS, DEVFLAG_TIMEOUT
 
 __all__ = [
     "CmcDims",
@@ -43,6 +43,7 @@ __all__ = [
     "decode_attn_workspace_size",
     "decode_attn_plan",
     "dims_of",
+    "stage_copies",
     "DEVFLAG_BAD_INDEX",
     "DEVFLAG_BAD_POS",
     "DEVFLAG_TIMEOUT",
@@ -419,3 +420,43 @@ def window_append(ring_k: torch.Tensor, ring_v: torch.Tensor, pos: torch.Tensor,
     st = lib().cmc_window_append(_p(ring_k), _p(ring_v), _p(pos), _p(k_new), _p(v_new),
                                  ctypes.byref(dims), _stream(dev))
     check(st, "cmc_window_append")
+
+
+# ----------------------------------------------------------------------------
+# Staging copies (host <-> device traffic of a decode loop)
+# ----------------------------------------------------------------------------
+
+def stage_copies(pairs, *, wait_first: bool = False, device: Optional[torch.device] = None) -> None:
+    """Copy each (src, dst) tensor pair, byte for byte, in one kernel launch on
+    the current stream; see cmc_stage_copies.  Host tensors must be pinned
+    (their memory is then mapped for the device).  With wait_first=False the
+    copies overlap the kernel before the call on the stream (the caller keeps
+    that kernel off every source and destination) and the launch completes
+    after it."""
+    pairs = list(pairs)
+    if len(pairs) > 4:
+        raise ValueError("at most 4 copies per call")
+    arr = (CmcCopy * max(1, len(pairs)))()
+    dev = device
+    for i, (src, dst) in enumerate(pairs):
+        for t, name in ((src, "src"), (dst, "dst")):
+            if not isinstance(t, torch.Tensor) or not t.is_contiguous():
+                raise ValueError(f"{name} must be a contiguous tensor")
+            if not t.is_cuda and not t.is_pinned():
+                raise ValueError(f"{name} must be a CUDA tensor or pinned host memory")
+            if t.is_cuda:
+                if dev is None:
+                    dev = t.device
+                elif t.device != dev:
+                    raise ValueError("all device tensors must be on one device")
+        nb = src.numel() * src.element_size()
+        if dst.numel() * dst.element_size() != nb:
+            raise ValueError("src and dst sizes differ")
+        arr[i].src = src.data_ptr()
+        arr[i].dst = dst.data_ptr()
+        arr[i].bytes = nb
+    if dev is None:
+        dev = torch.device("cuda", torch.cuda.current_device())
+    st = lib().cmc_stage_copies(ctypes.cast(arr, ctypes.c_void_p), len(pairs),
+                                1 if wait_first else 0, _stream(dev))
+    check(st, "cmc_stage_copies")

@@ -278,3 +278,20 @@ def test_denoise_argument_checks(L):
     assert d(emb=FAKE + 4) == ALIGN
     assert d(cnt=FAKE + 2) == ALIGN
     assert d(wsb=100) == WORKSPACE
+
+
+@host_only
+def test_stage_copies_argument_checks(L):
+    def call(copies, n, wait_first=0):
+        arr = (_lib.CmcCopy * max(1, len(copies)))()
+        for i, (s, d, b) in enumerate(copies):
+            arr[i].src, arr[i].dst, arr[i].bytes = s, d, b
+        return L.cmc_stage_copies(ctypes.cast(arr, ctypes.c_void_p), n, wait_first, None)
+    assert call([(FAKE, FAKE, 64)] * 4, 5) == RANGE
+    assert call([(FAKE, FAKE, 64)], -1) == RANGE
+    assert L.cmc_stage_copies(None, 1, 0, None) == NULL
+    assert call([(0, FAKE, 64)], 1) == NULL
+    assert call([(FAKE, 0, 64)], 1) == NULL
+    assert call([(FAKE + 8, FAKE, 64)], 1) == ALIGN
+    assert call([(FAKE, FAKE + 4, 64)], 1) == ALIGN
+    assert call([(FAKE, FAKE, 40)], 1) == ALIGN
