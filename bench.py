@@ -715,18 +715,27 @@ def run_e2e(args, w, reqs, dev, stream, world):
     without waiting for the decode before it (inputs double-buffered, outputs
     triple-buffered, so that decode never touches what it copies) and
     completes after it, so every decode launch keeps programmatic dependent
-    launch and the copies overlap decode work.  A last launch after the P
-    rounds carries the last two rounds' outputs.  P rounds are captured in one
-    CUDA graph.  Selection and compaction run eagerly."""
+    launch and the copies overlap decode work.  12 rounds (6 when T is not a
+    multiple of 12) are captured in one CUDA graph; the buffers rotate across
+    replays, so a replay's first two copy launches carry the previous
+    replay's last two rounds' outputs, and one copy launch after the step's
+    last replay the step's last two.  Selection and compaction run
+    eagerly."""
     import paper_2609_25537_gb300 as cmc
-    R, T, P = args.requests, args.decode_steps, args.pool
+    R, T, P0 = args.requests, args.decode_steps, args.pool
+    # rounds per graph: a multiple of 6 when T allows, so that the double-
+    # buffered inputs and triple-buffered outputs continue across replays and
+    # only the step's last two rounds need a copy after the last replay
+    P = 12 if T % 12 == 0 else (6 if T % 6 == 0 else P0)
+    rotate = P % 6 == 0
     steps = max(1, min(args.steps, args.e2e_steps))
     nq, nk = reqs[0].q[0].numel(), reqs[0].k_new[0].numel()
     per_req = nq + 2 * nk
     # host: round p holds the R requests' packed (q, k_new, v_new) of step p
-    host_in = torch.cat([torch.cat([r.q.reshape(P, -1), r.k_new.reshape(P, -1),
-                                    r.v_new.reshape(P, -1)], dim=1) for r in reqs],
-                        dim=1).cpu().pin_memory()                      # [P, R * per_req]
+    # (the pool's P0 inputs, cycled)
+    host_in = torch.cat([torch.cat([r.q.reshape(P0, -1), r.k_new.reshape(P0, -1),
+                                    r.v_new.reshape(P0, -1)], dim=1) for r in reqs],
+                        dim=1)[[p % P0 for p in range(P)]].contiguous().pin_memory()  # [P, R*per_req]
     out_shape = tuple(reqs[0].out.shape)
     host_out = torch.empty((P, R) + out_shape, dtype=torch.bfloat16).pin_memory()
     host_sel = [(r.qemb.cpu().pin_memory(), r.bank.cpu().pin_memory()) for r in reqs]
@@ -738,17 +747,21 @@ def run_e2e(args, w, reqs, dev, stream, world):
         return (base[:nq].view(reqs[i].q[0].shape), base[nq:nq + nk].view(reqs[i].k_new[0].shape),
                 base[nq + nk:].view(reqs[i].v_new[0].shape))
 
+    def last_two():  # the outputs of the last two rounds, after every decode
+        cmc.stage_copies([(out_d[(P - 2) % 3], host_out[P - 2]),
+                          (out_d[(P - 1) % 3], host_out[P - 1])], wait_first=True, device=dev)
+
     def rounds():
         for p in range(P):
             pairs = [(host_in[p], in_d[p % 2])]
-            if p >= 2:
-                pairs.append((out_d[(p - 2) % 3], host_out[p - 2]))
+            if p >= 2 or rotate:  # rounds 0, 1: the previous replay's last two
+                pairs.append((out_d[(p - 2) % 3], host_out[(p - 2) % P]))
             cmc.stage_copies(pairs, device=dev)
             for i, r in enumerate(reqs):
                 q, k, v = views(p % 2, i)
-                r.decode(p, q=q, k_new=k, v_new=v, mode=args.tier1, out=out_d[p % 3][i])
-        tail = [(out_d[(p - 1) % 3], host_out[p - 1]) for p in (P - 1, P) if p >= 1]
-        cmc.stage_copies(tail, wait_first=True, device=dev)
+                r.decode(p % P0, q=q, k_new=k, v_new=v, mode=args.tier1, out=out_d[p % 3][i])
+        if not rotate:
+            last_two()
 
     graph = None
     try:
@@ -773,6 +786,8 @@ def run_e2e(args, w, reqs, dev, stream, world):
                     graph.replay()
                 else:
                     rounds()
+            if rotate:
+                last_two()
         stream.synchronize()
 
     step()  # warm-up
