@@ -735,7 +735,7 @@ def run_e2e(args, w, reqs, dev, stream, world):
     # (the pool's P0 inputs, cycled)
     host_in = torch.cat([torch.cat([r.q.reshape(P0, -1), r.k_new.reshape(P0, -1),
                                     r.v_new.reshape(P0, -1)], dim=1) for r in reqs],
-                        dim=1)[[p % P0 for p in range(P)]].contiguous().pin_memory()  # [P, R*per_req]
+                        dim=1)[[p % P0 for p in range(P)]].cpu().contiguous().pin_memory()  # [P, R*per_req]
     out_shape = tuple(reqs[0].out.shape)
     host_out = torch.empty((P, R) + out_shape, dtype=torch.bfloat16).pin_memory()
     host_sel = [(r.qemb.cpu().pin_memory(), r.bank.cpu().pin_memory()) for r in reqs]
