@@ -21,8 +21,8 @@ namespace cmc {
 
 constexpr int kMaxCopies = 4;
 constexpr int kIoThreads = 256;
-constexpr int kInFlight = 8;
-constexpr int kIoMaxCtas = 128;
+constexpr int kInFlight = 4;
+constexpr int kIoMaxCtas = 64;
 
 struct IoArgs {
   const uint4* src[kMaxCopies];
