@@ -23,12 +23,17 @@ Reported (one JSON line on rank 0):
                  included in the timed region;
   roofline       the fused decode-step kernel: algorithmic bytes per launch
                  / average launch time, against the measured HBM copy peak;
-  select_us      Tier-1 score + select per request (two launches), L2-cold;
+  select_us      Tier-1 score + select per request (one launch at this
+                 size), inside the benchmark step, L2-cold;
   tier1_gather_us  the once-per-request Tier-1 compaction;
-  question_prologue_us, bridge_epilogue_us, denoise_us
-                 one call each (the question-side prologue of a request, the
-                 MemoryBridge output of a bank, the denoising of a context of
-                 N * r tokens), L2-cold, median of 5;
+  question_prologue_us, bridge_epilogue_us, denoise_us, select_stream_us
+                 per call in a graph of back-to-back calls on distinct inputs
+                 (at least twice the L2 per replay: every call reads HBM):
+                 the question-side prologue of a request, the MemoryBridge
+                 output of a bank, the denoising of a context of N * r
+                 tokens, the selection alone;
+  *_cold_us      one isolated call after a 512 MB write that evicts the L2
+                 (median of 5; includes a launch's fixed cost);
   variant        the decode step with the other Tier-1 form, us per launch;
   e2e            the same metric through the Python API with host buffers
                  (question vector, CME bank and every step's q / new K,V
@@ -584,9 +589,15 @@ def run_gpu(args, w, world, rank, local):
                         "achieved_gbs": nbytes / (r_us * 1e-6) / 1e9}
         del g3
 
-    # Once-per-request kernels outside the decode loop, each timed L2-cold: a
-    # graph of one call, replayed after a 512 MB write that evicts the L2
-    # (the write also covers the CPU's enqueue of the replay); median of 5.
+    # Once-per-request kernels outside the decode loop.  Each is timed as a
+    # graph of back-to-back calls on distinct copies of its inputs -- enough
+    # copies that the calls of one replay read at least twice the L2 (129 MB),
+    # so every call reads HBM -- replayed after warm-up; per call = replay
+    # time / calls (a call's launch is amortised and, under programmatic
+    # dependent launch, overlaps the one before: the device-side cost of a
+    # stream of requests).  The bank-sized ones also report one isolated call
+    # after a 512 MB write that evicts the L2 (median of 5), which includes a
+    # launch's fixed cost of several microseconds.
     flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
 
     def cold_us(fn, reps=5):
@@ -608,7 +619,31 @@ def run_gpu(args, w, world, rank, local):
         stream.synchronize()
         return 1000.0 * statistics.median(a.elapsed_time(b) for a, b in times[1:])
 
-    prologue_us = bridge_us = denoise_us = None
+    def stream_us(fns, reps=10):
+        with torch.cuda.stream(stream):
+            for fn in fns:
+                fn()  # warm-up outside capture
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for fn in fns:
+                fn()
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g.replay()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        stream.synchronize()
+        return 1000.0 * e0.elapsed_time(e1) / (reps * len(fns))
+
+    def copies_for(nbytes):
+        return max(2, min(16, -(-2 * 129_000_000 // max(nbytes, 1))))
+
+    prologue_us = bridge_us = denoise_us = select_cold_us = None
+    prologue_cold_us = bridge_cold_us = None
     denoise_bytes = 0
     if not args.no_variant:
         # the question-side prologue of one request (pool q_vec, score + select,
@@ -618,16 +653,35 @@ def run_gpu(args, w, world, rank, local):
         qlen = torch.from_numpy(qi.q_len).to(dev)
         offs = torch.from_numpy(qi.chunk_offset).to(dev)
         clen = torch.from_numpy(qi.ctx_len).to(dev)
-        ws_q = torch.zeros(cmc.lib().cmc_question_select_workspace_size(w.B, w.N),
-                           dtype=torch.uint8, device=dev)
         r0 = reqs[0]
-        prologue_us = cold_us(lambda: cmc.question_select(
-            tok, r0.bank, w.k, q_len=qlen, chunk_offset=offs, ctx_len=clen, W=w.W, workspace=ws_q))
+        nc = copies_for(r0.bank.numel() * 4)
+        banks = [r0.bank] + [r0.bank.clone() for _ in range(nc - 1)]
+        toks = [tok] + [tok.clone() for _ in range(nc - 1)]
+        ws_qs = [torch.zeros(cmc.lib().cmc_question_select_workspace_size(w.B, w.N),
+                             dtype=torch.uint8, device=dev) for _ in range(nc)]
+        ws_ss = [torch.zeros(cmc.score_select_workspace_size(w.B, w.N), dtype=torch.uint8,
+                             device=dev) for _ in range(nc)]
+        idxs = [torch.empty_like(r0.idx) for _ in range(nc)]
+        # the selection alone, timed the same ways
+        select_cold_us = cold_us(lambda: cmc.score_select(r0.qemb, r0.bank, w.k, idx_out=r0.idx,
+                                                          workspace=r0.sel_ws))
+        sel_stream_us = stream_us([
+            (lambda i=i: cmc.score_select(r0.qemb, banks[i], w.k, idx_out=idxs[i],
+                                          workspace=ws_ss[i])) for i in range(nc)])
+        prologue_cold_us = cold_us(lambda: cmc.question_select(
+            tok, r0.bank, w.k, q_len=qlen, chunk_offset=offs, ctx_len=clen, W=w.W,
+            workspace=ws_qs[0]))
+        prologue_us = stream_us([
+            (lambda i=i: cmc.question_select(toks[i], banks[i], w.k, q_len=qlen,
+                                             chunk_offset=offs, ctx_len=clen, W=w.W,
+                                             workspace=ws_qs[i])) for i in range(nc)])
         # MemoryBridge output (LayerNorm, nu tanh, norm cap) on a bank-sized
         # MLP output, out of place
-        scratch = torch.empty_like(r0.bank)
-        bridge_us = cold_us(lambda: cmc.bridge_epilogue(r0.bank, 0.8, out=scratch))
-        del scratch
+        outs = [torch.empty_like(r0.bank) for _ in range(nc)]
+        bridge_cold_us = cold_us(lambda: cmc.bridge_epilogue(banks[0], 0.8, out=outs[0]))
+        bridge_us = stream_us([(lambda i=i: cmc.bridge_epilogue(banks[i], 0.8, out=outs[i]))
+                               for i in range(nc)])
+        del outs, banks, toks
         # graph-based denoising of one context of |C| = N * r tokens (H = 1280,
         # GPT2-Large's width; g = 3, tau = 0.05, keep-minimum 16)
         ratio = 8 if w.N >= 16384 else 4
@@ -635,11 +689,14 @@ def run_gpu(args, w, world, rank, local):
             ratio = max(1, args.denoise_tokens // w.N)
         ci = context_inputs(w.with_(B=1), H=1280, ratio=ratio)
         emb = torch.from_numpy(ci.emb).to(dev)
-        ws_d = torch.empty(cmc.lib().cmc_denoise_workspace_size(1, emb.shape[1]),
-                           dtype=torch.uint8, device=dev)
-        denoise_us = cold_us(lambda: cmc.denoise(emb, workspace=ws_d))
         denoise_bytes = emb.numel() * 4
-        del emb
+        nd = copies_for(denoise_bytes)
+        embs = [emb] + [emb.clone() for _ in range(nd - 1)]
+        ws_ds = [torch.empty(cmc.lib().cmc_denoise_workspace_size(1, emb.shape[1]),
+                             dtype=torch.uint8, device=dev) for _ in range(nd)]
+        denoise_us = stream_us([(lambda i=i: cmc.denoise(embs[i], workspace=ws_ds[i]))
+                                for i in range(nd)])
+        del emb, embs
     del flush
 
     # e2e through the Python API with pinned host buffers
@@ -674,7 +731,11 @@ def run_gpu(args, w, world, rank, local):
         "decode_us_per_launch": launch_us,
         "hbm_pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
         "select_us": select_us,
+        "select_cold_us": select_cold_us,
+        "select_stream_us": sel_stream_us if not args.no_variant else None,
         "question_prologue_us": prologue_us,
+        "question_prologue_cold_us": prologue_cold_us,
+        "bridge_epilogue_cold_us": bridge_cold_us,
         "bridge_epilogue_us": bridge_us,
         "bridge_epilogue_gbs": (8 * w.B * w.N * w.D / (bridge_us * 1e-6) / 1e9
                                 if bridge_us else None),

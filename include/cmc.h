@@ -215,6 +215,11 @@ CMC_API size_t cmc_question_select_workspace_size(int B, int N);
  *                    (as for cmc_score_select: scores, squared norms, then
  *                    B completion counters that every call leaves at zero)
  *
+ * Small banks (as for cmc_score_select) take one kernel launch for the whole
+ * prologue; larger ones three (pooling, scoring, selection).  q_vec is the
+ * fp32 mean in either case, summed in a fixed order (the two paths' orders
+ * differ, within fp32 rounding).
+ *
  * Limits: those of cmc_score_select, Lq >= 1, Lq * D <= 2^31, W >= 1 when
  * localising.
  */

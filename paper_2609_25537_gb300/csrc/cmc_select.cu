@@ -1,7 +1,14 @@
 // Tier-1 question-guided selection (Section 2.5, the score_j equation and the
-// top-K re-ordering by document position that follows it).
+// top-K re-ordering by document position that follows it), and the
+// question-side prologue before it (the mean-pooled question vector, and the
+// CME-guided start of the Tier-2 window).
 //
-// Two kernels:
+// Small banks (the request sizes of a single decode): one launch,
+// score_select_fused_kernel -- CTAs score a few rows each and the CTA that
+// completes a sequence's scores selects its top k (see there); the prologue's
+// pooling and localisation run in the same launch.
+//
+// Larger banks, two launches:
 //  1. cosine_scores_kernel -- one CTA of 256 threads per CME row (grid-stride
 //     over rows): every thread streams its share of the row with 16-byte loads
 //     issued four at a time, accumulating m.q, m.m and q.q in fp32; the
@@ -557,7 +564,11 @@ constexpr int kFusedMaxD = 4 * kFusedThreads;    // one float4 per thread and ro
 constexpr int kFusedMaxN = 2 * kFusedThreads;    // two keys per thread in the selection
 
 struct FusedArgs {
-  const float* qv;        // [B, D]
+  const float* qv;        // [B, D], or NULL: pooled from q_tokens
+  const float* q_tokens;  // [B, Lq, D] question-token embeddings (when qv is NULL)
+  const int32_t* q_len;   // [B] or NULL (Lq each)
+  int Lq;
+  float* q_vec_out;       // [B, D]: the pooled q_vec (when qv is NULL)
   const float* bank;      // [B, N, D]
   int N, D, k;
   int rows_per_cta;       // R: divides N
@@ -731,9 +742,35 @@ score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
   if (own)
     for (int r = 0; r < R; ++r) sel_cp_async16(rows_s + r * kFusedThreads + tid, rows_g + r * D4 + tid);
   asm volatile("cp.async.commit_group;\n" ::: "memory");
-  // q_vec . q_vec while the rows are in flight
-  const float4 qr = own ? __ldg(reinterpret_cast<const float4*>(a.qv + static_cast<long long>(b) * a.D) + tid)
-                        : make_float4(0.f, 0.f, 0.f, 0.f);
+  // q_vec and q_vec . q_vec while the rows are in flight
+  float4 qr = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (a.qv) {
+    if (own) qr = __ldg(reinterpret_cast<const float4*>(a.qv + static_cast<long long>(b) * a.D) + tid);
+  } else if (own) {
+    // the mean of the first n question-token rows: eight rows at a time,
+    // all eight loads in flight, added in a fixed tree, then divided by n
+    int n = a.q_len ? a.q_len[b] : a.Lq;
+    n = n < 0 ? 0 : (n > a.Lq ? a.Lq : n);
+    const float4* tk = reinterpret_cast<const float4*>(a.q_tokens + static_cast<long long>(b) * a.Lq * a.D) + tid;
+    for (int i0 = 0; i0 < n; i0 += 8) {
+      float4 v[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e)
+        v[e] = i0 + e < n ? __ldg(tk + static_cast<long long>(i0 + e) * D4) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int w = 1; w < 8; w <<= 1)
+#pragma unroll
+        for (int e = 0; e < 8; e += 2 * w) {
+          v[e].x += v[e + w].x; v[e].y += v[e + w].y; v[e].z += v[e + w].z; v[e].w += v[e + w].w;
+        }
+      qr.x += v[0].x; qr.y += v[0].y; qr.z += v[0].z; qr.w += v[0].w;
+    }
+    if (n > 0) {
+      const float fn = static_cast<float>(n);
+      qr.x /= fn; qr.y /= fn; qr.z /= fn; qr.w /= fn;
+    }
+    if (r0 == b * a.N) reinterpret_cast<float4*>(a.q_vec_out + static_cast<long long>(b) * a.D)[tid] = qr;
+  }
   {
     float acc = 0.f;
     acc = fmaf(qr.x, qr.x, acc); acc = fmaf(qr.y, qr.y, acc);
@@ -818,7 +855,9 @@ static int fused_rows_per_cta(int B, int N, int D) {
 static int launch_score_select_fused(const float* question_emb, const float* cme_bank, int B,
                                      int N, int D, int k, int32_t* idx_out, float* sc,
                                      unsigned int* counters, cudaStream_t s, const LocateArgs& la,
-                                     int R) {
+                                     int R, const float* q_tokens = nullptr,
+                                     const int32_t* q_len = nullptr, int Lq = 0,
+                                     float* q_vec_out = nullptr) {
   static std::once_flag attr_once[64];
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
@@ -832,6 +871,10 @@ static int launch_score_select_fused(const float* question_emb, const float* cme
   if (st != CMC_OK) return st;
   FusedArgs a;
   a.qv = question_emb;
+  a.q_tokens = q_tokens;
+  a.q_len = q_len;
+  a.Lq = Lq;
+  a.q_vec_out = q_vec_out;
   a.bank = cme_bank;
   a.N = N;
   a.D = D;
@@ -992,11 +1035,16 @@ int cmc_question_select(const float* question_tokens, const int32_t* q_len, int 
   unsigned int* counters =
       reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + 2 * scores_bytes);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out};
+  // small banks: pooling, scoring, selection and localisation in one launch
+  const int fused_rows = fused_rows_per_cta(B, N, D);
+  if (fused_rows > 0)
+    return launch_score_select_fused(nullptr, cme_bank, B, N, D, k, idx_out, sc, counters, s, la,
+                                     fused_rows, question_tokens, q_len, Lq, q_vec_out);
   const int D4 = D / 4;
   int st = launch_pdl(question_pool_kernel, dim3((D4 + 31) / 32, B),
                       dim3(kPoolThreads), 0, s, question_tokens, q_len, Lq, D, q_vec_out);
   if (st != CMC_OK) return st;
-  LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out};
   return launch_score_select(q_vec_out, cme_bank, B, N, D, k, idx_out, sc, s, counters, la);
 }
 
