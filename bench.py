@@ -692,7 +692,7 @@ def run_gpu(args, w, world, rank, local):
         denoise_bytes = emb.numel() * 4
         nd = copies_for(denoise_bytes)
         embs = [emb] + [emb.clone() for _ in range(nd - 1)]
-        ws_ds = [torch.empty(cmc.lib().cmc_denoise_workspace_size(1, emb.shape[1]),
+        ws_ds = [torch.zeros(cmc.lib().cmc_denoise_workspace_size(1, emb.shape[1]),
                              dtype=torch.uint8, device=dev) for _ in range(nd)]
         denoise_us = stream_us([(lambda i=i: cmc.denoise(embs[i], workspace=ws_ds[i]))
                                 for i in range(nd)])

@@ -105,9 +105,16 @@ CMC_API size_t cmc_denoise_workspace_size(int B, int n_max);
  *   kept_idx    int32 [B, n_max] output: the kept positions in ascending
  *               order, then -1
  *   kept_count  int32 [B] output: how many were kept
- *   workspace   >= cmc_denoise_workspace_size(B, n_max) bytes, any content;
+ *   workspace   >= cmc_denoise_workspace_size(B, n_max) bytes, zero-filled
+ *               before its first use: its last bytes hold one completion
+ *               counter per context, which every call leaves zero (calls
+ *               that share a workspace must be ordered, e.g. one stream);
  *               on completion its first B * n_max bytes hold each token's
  *               threshold-test result (1 passed, 0 not or past n_tokens)
+ *
+ * When the contexts' 32-token tiles fit one CTA per SM (B * ceil(n_max / 32)
+ * <= SM count), the whole call is one kernel launch: the CTA that finishes a
+ * context's last tile also walks its keep-minimum and writes kept_idx.
  *
  * Limits: 1 <= B <= 65535, 1 <= n_max <= 2^24, 4 <= H <= 65536, H % 4 == 0,
  * 1 <= g <= 8, keep_every >= 0, tau finite.
@@ -213,7 +220,8 @@ CMC_API size_t cmc_question_select_workspace_size(int B, int N);
  *   workspace        >= cmc_question_select_workspace_size(B, N) bytes,
  *                    16-byte aligned, zero-filled once before its first use
  *                    (as for cmc_score_select: scores, squared norms, then
- *                    B completion counters that every call leaves at zero)
+ *                    B completion counters and B 64-bit argmax slots, both
+ *                    left at zero by every call)
  *
  * Small banks (as for cmc_score_select) take one kernel launch for the whole
  * prologue; larger ones three (pooling, scoring, selection).  q_vec is the

@@ -82,7 +82,8 @@ def denoise(emb: torch.Tensor, *, n_tokens: Optional[torch.Tensor] = None, g: in
             workspace: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
     """Positions of the tokens kept by the graph-based denoising, int32
     [B, n_max] ascending then -1, and their counts int32 [B]; see
-    cmc_denoise.  Defaults: the paper's g = 3, tau = 0.05, keep-minimum 16."""
+    cmc_denoise.  Defaults: the paper's g = 3, tau = 0.05, keep-minimum 16.
+    A given ``workspace`` must have been zero-filled before its first use."""
     _need(emb, "emb", torch.float32, 3)
     dev = emb.device
     B, n_max, H = emb.shape
@@ -94,7 +95,7 @@ def denoise(emb: torch.Tensor, *, n_tokens: Optional[torch.Tensor] = None, g: in
     count = torch.empty(B, dtype=torch.int32, device=dev)
     need = int(lib().cmc_denoise_workspace_size(B, n_max))
     if workspace is None:
-        workspace = torch.empty(need, dtype=torch.uint8, device=dev)
+        workspace = _counter_workspace("denoise", need, dev)
     st = lib().cmc_denoise(_p(emb), _p(n_tokens), B, n_max, H, g, float(tau), keep_every,
                            _p(kept), _p(count), _p(workspace),
                            workspace.numel() * workspace.element_size(), _stream(dev))
@@ -139,17 +140,17 @@ def score_select_workspace_size(B: int, N: int) -> int:
     return int(lib().cmc_score_select_workspace_size(B, N))
 
 
-_sel_ws_cache: Dict[Tuple, torch.Tensor] = {}
+_counter_ws_cache: Dict[Tuple, torch.Tensor] = {}
 
 
-def _selection_workspace(kind: str, nbytes: int, device: torch.device) -> torch.Tensor:
-    """A zero-filled selection workspace, one per (kind, device, stream, size):
-    its completion counters start at zero, and every call leaves them so."""
+def _counter_workspace(kind: str, nbytes: int, device: torch.device) -> torch.Tensor:
+    """A zero-filled workspace, one per (kind, device, stream, size): its
+    completion counters start at zero, and every call leaves them so."""
     key = (kind, device.index, torch.cuda.current_stream(device).cuda_stream, nbytes)
-    ws = _sel_ws_cache.get(key)
+    ws = _counter_ws_cache.get(key)
     if ws is None:
         ws = torch.zeros(nbytes, dtype=torch.uint8, device=device)
-        _sel_ws_cache[key] = ws
+        _counter_ws_cache[key] = ws
     return ws
 
 
@@ -176,7 +177,7 @@ def score_select(question_emb: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
         if tuple(scores_out.shape) != (B, N):
             raise ValueError(f"scores_out shape {tuple(scores_out.shape)} != {(B, N)}")
     if workspace is None:
-        workspace = _selection_workspace("select", score_select_workspace_size(B, N), dev)
+        workspace = _counter_workspace("select", score_select_workspace_size(B, N), dev)
     ws_bytes = workspace.numel() * workspace.element_size()
     st = lib().cmc_score_select(_p(question_emb), _p(cme_bank), B, N, D, k, _p(idx_out),
                                 _p(scores_out), _p(workspace), ws_bytes, _stream(dev))
@@ -216,7 +217,7 @@ def question_select(question_tokens: torch.Tensor, cme_bank: torch.Tensor, k: in
     start = torch.empty(B, dtype=torch.int32, device=dev) if locate else None
     need = int(lib().cmc_question_select_workspace_size(B, N))
     if workspace is None:
-        workspace = _selection_workspace("question", need, dev)
+        workspace = _counter_workspace("question", need, dev)
     st = lib().cmc_question_select(
         _p(question_tokens), _p(q_len), Lq, _p(cme_bank), B, N, D, k, _p(chunk_offset),
         _p(ctx_len), int(W or 0), _p(q_vec), _p(idx), _p(alpha), _p(start), _p(workspace),

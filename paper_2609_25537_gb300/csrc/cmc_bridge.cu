@@ -8,8 +8,8 @@
 // are plain library GEMMs and stay with the caller; this is the row-wise
 // epilogue that turns their output into the bank the Tier-1 scoring reads.
 //
-// Rows of up to 4,096 features stay in registers (bridge_epilogue_reg_kernel,
-// below).  Longer rows: a CTA walks its rows (grid-stride) through three
+// Rows of up to 4,096 features stay in registers, one 128-thread CTA per
+// row (bridge_epilogue_reg_kernel, below).  Longer rows: a CTA walks its rows (grid-stride) through three
 // shared-memory row buffers: while it reduces and writes row r, rows r + grid and r + 2 grid are
 // already on their way (16-byte cp.async copies), so each SM overlaps the HBM
 // reads of later rows with the arithmetic and the writes of the current one.
@@ -145,20 +145,22 @@ bridge_epilogue_kernel(const float* x, const float* __restrict__ gamma,
   br_wait<0>();
 }
 
-// Rows of at most 4,096 features: a thread keeps its V float4s of the row in
-// registers and loads its share of the next row of the CTA (grid-stride)
-// before it works on the current one, so no shared-memory staging and no
-// refill barrier; each of the three reductions takes one barrier (its own
-// partials array, summed by every thread in the same order).
-constexpr int kBridgeRegMaxV = 4;  // float4s per thread: D <= 4 * 4 * kBridgeThreads
-constexpr int kBridgeRegCtasPerSm = 3;
+// Rows of at most 4,096 features: one CTA of 128 threads per row, a thread
+// keeping its V float4s of the row in registers; eight CTAs per SM, so that
+// a bank of up to 8 x SMs rows is one wave whose loads are all issued at
+// once (more rows: grid-stride).  No shared-memory staging; each of the
+// three reductions takes one barrier (its own partials array, summed by every
+// thread in the same order).
+constexpr int kBridgeRegThreads = 128;
+constexpr int kBridgeRegMaxV = 8;  // float4s per thread: D <= 4 * 8 * kBridgeRegThreads
+constexpr int kBridgeRegCtasPerSm = 8;
 
 template <int V>
-__global__ void __launch_bounds__(kBridgeThreads, kBridgeRegCtasPerSm)
+__global__ void __launch_bounds__(kBridgeRegThreads, kBridgeRegCtasPerSm)
 bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
                            const float* __restrict__ beta, long long rows, int D, float eps,
                            float nu, float* out) {
-  constexpr int NW = kBridgeThreads / 32;
+  constexpr int NW = kBridgeRegThreads / 32;
   __shared__ float red[3][NW];
   pdl_wait();
   pdl_trigger();
@@ -166,7 +168,6 @@ bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
   const int D4 = D >> 2;
   const float4* g4 = reinterpret_cast<const float4*>(gamma);
   const float4* b4 = reinterpret_cast<const float4*>(beta);
-  const long long step = gridDim.x;
   auto block_sum = [&](float v, float* part) {
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
@@ -177,19 +178,14 @@ bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
     for (int w = 1; w < NW; ++w) t += part[w];
     return t;
   };
-  auto load = [&](long long r, float4 (&v)[V]) {
+  for (long long r = blockIdx.x; r < rows; r += gridDim.x) {
+    float4 cur[V];
     const float4* src = reinterpret_cast<const float4*>(x + r * D);
 #pragma unroll
     for (int e = 0; e < V; ++e) {
-      const int i = tid + e * kBridgeThreads;
-      v[e] = i < D4 ? __ldcs(src + i) : make_float4(0.f, 0.f, 0.f, 0.f);  // coherent: x may be out
+      const int i = tid + e * kBridgeRegThreads;
+      cur[e] = i < D4 ? __ldcs(src + i) : make_float4(0.f, 0.f, 0.f, 0.f);  // coherent: x may be out
     }
-  };
-  float4 cur[V], nxt[V];
-  long long r = blockIdx.x;
-  if (r < rows) load(r, cur);
-  for (; r < rows; r += step) {
-    if (r + step < rows) load(r + step, nxt);
     float s = 0.f;
 #pragma unroll
     for (int e = 0; e < V; ++e) s += (cur[e].x + cur[e].y) + (cur[e].z + cur[e].w);
@@ -197,7 +193,7 @@ bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
     float q = 0.f;
 #pragma unroll
     for (int e = 0; e < V; ++e) {
-      if (tid + e * kBridgeThreads < D4) {
+      if (tid + e * kBridgeRegThreads < D4) {
         const float a = cur[e].x - mean, b = cur[e].y - mean, c = cur[e].z - mean, d = cur[e].w - mean;
         q += (a * a + b * b) + (c * c + d * d);
       }
@@ -207,7 +203,7 @@ bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
     float n2 = 0.f;
 #pragma unroll
     for (int e = 0; e < V; ++e) {
-      const int i = tid + e * kBridgeThreads;
+      const int i = tid + e * kBridgeRegThreads;
       if (i < D4) {
         const float4 g = gamma ? __ldg(g4 + i) : make_float4(1.f, 1.f, 1.f, 1.f);
         const float4 b = beta ? __ldg(b4 + i) : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -224,11 +220,10 @@ bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
     float4* orow = reinterpret_cast<float4*>(out + r * D);
 #pragma unroll
     for (int e = 0; e < V; ++e) {
-      const int i = tid + e * kBridgeThreads;
+      const int i = tid + e * kBridgeRegThreads;
       if (i < D4) orow[i] = make_float4(cur[e].x * f, cur[e].y * f, cur[e].z * f, cur[e].w * f);
     }
-#pragma unroll
-    for (int e = 0; e < V; ++e) cur[e] = nxt[e];
+    __syncthreads();  // red is rewritten by the next row of this CTA
   }
 }
 
@@ -246,17 +241,21 @@ int cmc_bridge_epilogue(const float* x, const float* gamma, const float* beta, i
     return CMC_ERR_ALIGN;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int D4 = D / 4;
-  if (D4 <= kBridgeRegMaxV * kBridgeThreads) {
+  if (D4 <= kBridgeRegMaxV * kBridgeRegThreads) {
     long long grid = rows;
     const long long cap = static_cast<long long>(sm_count()) * kBridgeRegCtasPerSm;
     if (grid > cap) grid = cap;
-    const dim3 gd(static_cast<unsigned>(grid)), bd(kBridgeThreads);
+    const dim3 gd(static_cast<unsigned>(grid)), bd(kBridgeRegThreads);
     const long long R = static_cast<long long>(rows);
-    switch ((D4 + kBridgeThreads - 1) / kBridgeThreads) {
+    switch ((D4 + kBridgeRegThreads - 1) / kBridgeRegThreads) {
       case 1: return launch_pdl(bridge_epilogue_reg_kernel<1>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
       case 2: return launch_pdl(bridge_epilogue_reg_kernel<2>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
       case 3: return launch_pdl(bridge_epilogue_reg_kernel<3>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
-      default: return launch_pdl(bridge_epilogue_reg_kernel<4>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      case 4: return launch_pdl(bridge_epilogue_reg_kernel<4>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      case 5: return launch_pdl(bridge_epilogue_reg_kernel<5>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      case 6: return launch_pdl(bridge_epilogue_reg_kernel<6>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      case 7: return launch_pdl(bridge_epilogue_reg_kernel<7>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
+      default: return launch_pdl(bridge_epilogue_reg_kernel<8>, gd, bd, 0, s, x, gamma, beta, R, D, eps, nu, out);
     }
   }
   const size_t smem = static_cast<size_t>(kBridgeBufs) * D * sizeof(float);

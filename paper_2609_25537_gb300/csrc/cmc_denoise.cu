@@ -8,26 +8,32 @@
 //     one context.  Their rows and the rows of the g tokens that follow the
 //     tile (together one contiguous span of the [n, H] matrix) are streamed
 //     through shared memory in chunks of 128 features (512 bytes per row),
-//     four stages of 16-byte cp.async copies; rows past the context's tokens
-//     are zero-filled, never read.  Each warp owns four tokens: per chunk a
-//     lane takes one float4 of each of the warp's rows and accumulates the
-//     squared norms and the dot products of every token with its g
-//     followers; lanes are reduced once per tile (fixed order), and lane 0
-//     writes the four pass flags (max cosine >= tau, decided in fp32).  Every
-//     row crosses from HBM once (the g halo rows are the next tile's first
-//     rows, read by the neighbouring CTA at about the same time).  The
-//     tile's 32 pass bits also go to a word of the workspace, and the tile's
-//     positions of kept_idx are set to -1 (the compaction overwrites the
-//     kept ones).
-//  2. denoise_compact_kernel -- one cluster of 8 CTAs per context.  Walking
-//     left to right, the keep-minimum forces token i exactly when it fails the test and its
-//     distance to the last token that passed (or to position -1) is a
-//     multiple of keep_every, so the walk is data-parallel.  A thread takes
-//     one 32-token pass word per segment of 262,144 tokens (the next
-//     segment's word is loaded ahead); a cluster-wide prefix maximum gives it
-//     the last passing position before its word, from which the forced
-//     positions of each gap follow with one division; a cluster-wide prefix
-//     sum places its kept positions; both carry from one segment to the next.
+//     four stages of 16-byte cp.async copies (two CTAs per SM); rows past the
+//     context's tokens are zero-filled, never read.  Each warp owns four
+//     tokens: per chunk a lane takes one float4 of each of the warp's rows
+//     and of the g rows after them, and accumulates their squared norms and
+//     the dot products of every token with its g followers; the lanes meet
+//     once per tile in a halving butterfly (fixed order), and lane t g + s
+//     decides the cosine of token t with follower s (>= tau, in fp32), one
+//     vote per warp giving its four pass flags.  Every row crosses from HBM
+//     once (the g halo rows are the next tile's first rows, read by the
+//     neighbouring CTA at about the same time).  The tile's 32 pass bits also
+//     go to a word of the workspace, and the tile's positions of kept_idx are
+//     set to -1 (the compaction overwrites the kept ones).  For a context of
+//     at most 256 tiles (8,192 tokens) the CTA that finishes its last tile (a
+//     counter per context, acq_rel) also runs the keep-minimum and the
+//     compaction below for that context (pass_compact_small: one pass word
+//     per thread, two barriers), and the second kernel is not launched.
+//  2. denoise_compact_kernel -- one cluster of 8 CTAs per longer context.
+//     Walking left to right, the keep-minimum forces token i exactly when it
+//     fails the test and its distance to the last token that passed (or to
+//     position -1) is a multiple of keep_every, so the walk is data-parallel.
+//     A thread takes one 32-token pass word per segment of 262,144 tokens
+//     (the next segment's word is loaded ahead); a cluster-wide prefix
+//     maximum gives it the last passing position before its word, from which
+//     the forced positions of each gap follow (keep_mask); a cluster-wide
+//     prefix sum places its kept positions; both carry from one segment to
+//     the next.
 #include <cuda_runtime.h>
 #include <math.h>
 #include <stdint.h>
@@ -45,8 +51,8 @@ constexpr int kPassTile = kPassTokPerWarp * (kPassThreads / 32);  // 32 tokens p
 constexpr int kPassChunk = 128;                                   // features per stage
 constexpr int kPassStageRows = kPassTile + kDenoiseMaxG;          // 40
 constexpr int kPassStageBytes = kPassStageRows * kPassChunk * 4;  // 20 KB
-constexpr int kPassStages = 4;
-constexpr int kPassSmem = kPassStages * kPassStageBytes;          // 80 KB
+constexpr int kPassStages = 4;                                    // two CTAs per SM
+__host__ __device__ constexpr int pass_smem(int stages) { return stages * kPassStageBytes; }
 constexpr int kCompactThreads = 1024;
 constexpr int kCompactWords = 4;  // pass words per 16-byte group of the word array's rows
 constexpr int kCompactCtas = 8;   // CTAs (one thread-block cluster) per context
@@ -64,19 +70,117 @@ __device__ __forceinline__ float dot4(const float4& a, const float4& b) {
   return (a.x * b.x + a.y * b.y) + (a.z * b.z + a.w * b.w);
 }
 
-template <int G>
+// Kept tokens among the 32 tokens i0 .. i0+31 whose pass bits are `m`, given
+// lp, the last passing position before i0 (-1: none): the passing tokens,
+// and in every gap between a passing token (or lp) and the next one, the
+// positions at multiples of K after it.  The gap from lp takes one division;
+// a later gap holds a forced position only when the K bits after its passing
+// token are all zero, which a run mask of the zero bits finds for the whole
+// word at once (bit x of r: bits x .. x+K-1 of ~m all set, built by doubling),
+// so the loop visits only those gaps.
+__device__ __forceinline__ uint32_t keep_mask(uint32_t m, int lp, int i0, int K) {
+  uint32_t kept = m;
+  if (K <= 0) return kept;
+  const int first = m ? __ffs(m) - 1 : 32;  // first passing token (word-relative)
+  for (int f = lp + K * ((i0 - lp + K - 1) / K) - i0; f < first; f += K) kept |= 1u << f;
+  if (K >= 32) return kept;  // a later gap fits no multiple of K inside the word
+  uint32_t r = ~m;
+  int len = 1;
+  while (2 * len <= K) {
+    r &= r >> len;
+    len *= 2;
+  }
+  if (K > len) r &= r >> (K - len);
+  uint32_t cand = m & (r >> 1);  // passing tokens followed by K failing ones
+  while (cand) {
+    const int p = __ffs(cand) - 1;
+    cand &= cand - 1;
+    const uint32_t after = m & ~((2u << p) - 1u);  // passing tokens after p
+    const int q = after ? __ffs(after) - 1 : 32;
+    for (int f = p + K; f < q; f += K) kept |= 1u << f;
+  }
+  return kept;
+}
+
+// The keep-minimum and the compaction of context b by the pass CTA that
+// finished its last tile, for a context of at most kPassThreads tiles:
+// thread t takes pass word t; the last passing position before its word is a
+// prefix maximum (a warp scan, then the warp totals before it from shared
+// memory), its kept positions follow from keep_mask, and their first slot in
+// kept_idx is a prefix sum in the same two steps; it writes its kept
+// positions itself.  Two barriers.  The words were written by the other CTAs
+// of this launch before their counter additions, which this CTA's thread 0
+// acquired.
+__device__ void pass_compact_small(const uint32_t* masks, int n, int keep_every,
+                                   int32_t* out, int32_t* count, int* wmax, int* wsum) {
+  constexpr int NW = kPassThreads / 32;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nw = (n + 31) / 32;  // words that hold tokens (at most kPassThreads)
+  const int i0 = 32 * tid;
+  const int nv = tid < nw ? min(n - i0, 32) : 0;
+  const uint32_t valid = nv >= 32 ? ~0u : ((1u << nv) - 1u);
+  const uint32_t m = tid < nw ? (__ldcg(masks + tid) & valid) : 0u;
+  int lp = m ? i0 + 31 - __clz(m) : -1;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, lp, off);
+    if (lane >= off) lp = max(lp, u);
+  }
+  if (lane == 31) wmax[warp] = lp;
+  lp = __shfl_up_sync(0xffffffffu, lp, 1);
+  if (lane == 0) lp = -1;
+  __syncthreads();
+#pragma unroll
+  for (int w = 0; w < NW; ++w)
+    if (w < warp) lp = max(lp, wmax[w]);
+  uint32_t kept = nv > 0 ? keep_mask(m, lp, i0, keep_every) & valid : 0u;
+  const int c = __popc(kept);
+  int incl = c;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += u;
+  }
+  if (lane == 31) wsum[warp] = incl;
+  __syncthreads();
+  int slot = incl - c, total = 0;
+#pragma unroll
+  for (int w = 0; w < NW; ++w) {
+    const int x = wsum[w];
+    slot += w < warp ? x : 0;
+    total += x;
+  }
+  while (kept) {
+    out[slot++] = i0 + __ffs(kept) - 1;
+    kept &= kept - 1;
+  }
+  if (tid == 0) *count = total;
+}
+
+// FUSE (a context of at most kPassThreads tiles): the CTA that finishes a
+// context's last tile also runs its keep-minimum and compaction
+// (pass_compact_small), counting finished tiles in `counters` (zero before
+// the call, zero after it).
+template <int G, int NST, bool FUSE>
 __global__ void __launch_bounds__(kPassThreads, 2)
 denoise_pass_kernel(const float* __restrict__ emb, const int32_t* __restrict__ n_tokens, int n_max,
                     int H, float tau, uint8_t* __restrict__ pass, uint32_t* __restrict__ masks,
                     int32_t* __restrict__ kept_idx, long long tiles, int tiles_per_ctx,
-                    int words_stride) {
+                    int words_stride, unsigned int* __restrict__ counters, int keep_every,
+                    int32_t* __restrict__ kept_count) {
   constexpr int TPW = kPassTokPerWarp;
   constexpr int SROWS = kPassTile + G;                                // rows staged per chunk
   constexpr int NCP = (SROWS * 32 + kPassThreads - 1) / kPassThreads;  // copies per thread
-  constexpr int kLast = kPassThreads / 32 - 1;                        // warp that owns the halo norms
+  // per warp: the squared norms of its TPW rows and the G rows after them,
+  // then the TPW x G dot products; padded to whole groups of 16
+  constexpr int NV = TPW + G + TPW * G;
+  constexpr int NV16 = (NV + 15) / 16 * 16;
+  constexpr int KV = NV16 / 16;  // values a lane holds after the halving rounds
   extern __shared__ __align__(16) float4 dn_stage[];
-  __shared__ float nrm_s[kPassTile + kDenoiseMaxG];  // squared norms of the staged rows
-  __shared__ uint32_t nib[kPassThreads / 32];         // each warp's four pass bits
+  __shared__ float red_s[kPassThreads / 32][NV16];  // each warp's reduced values
+  __shared__ uint32_t nib[kPassThreads / 32];        // each warp's four pass bits
+  __shared__ int wmax[kPassThreads / 32], wsum[kPassThreads / 32];  // the fused compaction's scans
+  __shared__ int last_flag;
   pdl_wait();
   pdl_trigger();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -91,9 +195,42 @@ denoise_pass_kernel(const float* __restrict__ emb, const int32_t* __restrict__ n
     uint8_t* pb = pass + static_cast<long long>(b) * n_max;
     // the compaction overwrites the kept positions; everything else stays -1
     if (tid < kPassTile && i0 + tid < n_max) kept_idx[static_cast<long long>(b) * n_max + i0 + tid] = -1;
+    // Thread 0 writes the tile's pass word (after the barrier that makes the
+    // warps' bits and every thread's writes precede it) and, fused, adds the
+    // tile to the context's count with an acq_rel atomic (releasing this CTA's
+    // writes, acquiring the other CTAs' for the last one); the CTA that
+    // completes the count compacts the context.
+    auto tile_done = [&](bool empty) {
+      __syncthreads();
+      if (tid == 0) {
+        uint32_t word = 0;
+        if (!empty) {
+#pragma unroll
+          for (int w = 0; w < kPassThreads / 32; ++w) word |= nib[w] << (w * TPW);
+        }
+        masks[static_cast<long long>(b) * words_stride + i0 / kPassTile] = word;
+        if (FUSE) {
+          unsigned int old;
+          asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;\n"
+                       : "=r"(old)
+                       : "l"(counters + b)
+                       : "memory");
+          last_flag = (old + 1 == static_cast<unsigned int>(tiles_per_ctx)) ? 1 : 0;
+        }
+      }
+      if (FUSE) {
+        __syncthreads();
+        if (last_flag) {
+          pass_compact_small(masks + static_cast<long long>(b) * words_stride, n, keep_every,
+                             kept_idx + static_cast<long long>(b) * n_max, kept_count + b, wmax,
+                             wsum);
+          if (tid == 0) counters[b] = 0u;  // ready for the next call
+        }
+      }
+    };
     if (i0 >= n) {  // a tile past the context's tokens: flags 0
       if (tid < kPassTile && i0 + tid < n_max) pb[i0 + tid] = 0;
-      if (tid == 0) masks[static_cast<long long>(b) * words_stride + i0 / kPassTile] = 0u;
+      tile_done(true);
       continue;
     }
     const int rows = min(SROWS, n - i0);  // staged rows that hold tokens
@@ -109,7 +246,7 @@ denoise_pass_kernel(const float* __restrict__ emb, const int32_t* __restrict__ n
       src[m] = src0 + static_cast<long long>(x >> 5) * H + 4 * (x & 31);
     }
     auto issue = [&](int c) {
-      const uint32_t dst0 = sbase + (c % kPassStages) * kPassStageBytes;
+      const uint32_t dst0 = sbase + (c % NST) * kPassStageBytes;
       const int col0 = c * kPassChunk;
 #pragma unroll
       for (int m = 0; m < NCP; ++m) {
@@ -121,84 +258,75 @@ denoise_pass_kernel(const float* __restrict__ emb, const int32_t* __restrict__ n
       }
     };
 #pragma unroll
-    for (int c = 0; c < kPassStages - 1; ++c) {
+    for (int c = 0; c < NST - 1; ++c) {
       if (c < nchunks) issue(c);
       dn_commit();
     }
-    float nrm[TPW + G], dt[TPW][G];
+    // v: the norms of rows r0 .. r0+TPW+G-1, then dot(t, s) at TPW + G + t G + s
+    float v[NV16];
 #pragma unroll
-    for (int j = 0; j < TPW + G; ++j) nrm[j] = 0.f;
-#pragma unroll
-    for (int t = 0; t < TPW; ++t)
-#pragma unroll
-      for (int s = 0; s < G; ++s) dt[t][s] = 0.f;
+    for (int j = 0; j < NV16; ++j) v[j] = 0.f;
     for (int c = 0; c < nchunks; ++c) {
-      dn_wait<kPassStages - 2>();  // chunk c has landed (this thread's copies)
+      dn_wait<NST - 2>();  // chunk c has landed (this thread's copies)
       __syncthreads();             // ... everyone's; and chunk c-1's stage is free
-      if (c + kPassStages - 1 < nchunks) issue(c + kPassStages - 1);
+      if (c + NST - 1 < nchunks) issue(c + NST - 1);
       dn_commit();
-      const float4* st = dn_stage + (c % kPassStages) * (kPassStageBytes / 16) + r0 * 32 + lane;
+      const float4* st = dn_stage + (c % NST) * (kPassStageBytes / 16) + r0 * 32 + lane;
       float4 x[TPW + G];
 #pragma unroll
       for (int j = 0; j < TPW + G; ++j) x[j] = st[j * 32];
 #pragma unroll
-      for (int j = 0; j < TPW; ++j) nrm[j] += dot4(x[j], x[j]);
-      if (warp == kLast) {  // the g rows after the tile
-#pragma unroll
-        for (int j = TPW; j < TPW + G; ++j) nrm[j] += dot4(x[j], x[j]);
-      }
+      for (int j = 0; j < TPW + G; ++j) v[j] += dot4(x[j], x[j]);
 #pragma unroll
       for (int t = 0; t < TPW; ++t)
 #pragma unroll
-        for (int s = 0; s < G; ++s) dt[t][s] += dot4(x[t], x[t + 1 + s]);
+        for (int s = 0; s < G; ++s) v[TPW + G + t * G + s] += dot4(x[t], x[t + 1 + s]);
     }
     dn_wait<0>();
+    // Halving butterfly over the lanes: at offset o the lanes with bit o set
+    // keep the upper half of their values and add their partner's upper
+    // half; the others the lower half.  It adds the same pairs as a plain xor
+    // butterfly for every value (so every warp that reduces a row's norm
+    // gets the same bits), in a fraction of the shuffles.  Afterwards lanes
+    // 2i and 2i+1 hold values KV i .. KV i + KV-1 summed over the warp.
 #pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) {
+    for (int o = 16, nh = NV16 / 2; o >= 2; o >>= 1, nh >>= 1) {
+      const bool up = (lane & o) != 0;
 #pragma unroll
-      for (int j = 0; j < TPW + G; ++j)
-        if (j < TPW || warp == kLast) nrm[j] += __shfl_xor_sync(0xffffffffu, nrm[j], off);
-#pragma unroll
-      for (int t = 0; t < TPW; ++t)
-#pragma unroll
-        for (int s = 0; s < G; ++s) dt[t][s] += __shfl_xor_sync(0xffffffffu, dt[t][s], off);
+      for (int i = 0; i < nh; ++i) {
+        const float send = up ? v[i] : v[i + nh];
+        const float keep = up ? v[i + nh] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+      }
     }
-    if (lane == 0) {
 #pragma unroll
-      for (int j = 0; j < TPW + G; ++j)
-        if (j < TPW || warp == kLast) nrm_s[r0 + j] = nrm[j];
+    for (int i = 0; i < KV; ++i) v[i] += __shfl_xor_sync(0xffffffffu, v[i], 1);
+    if ((lane & 1) == 0) {
+#pragma unroll
+      for (int i = 0; i < KV; ++i) red_s[warp][KV * (lane >> 1) + i] = v[i];
     }
-    __syncthreads();  // the norms are shared; the stages are refilled by the next tile
-    if (lane == 0) {
+    __syncwarp();
+    {
+      // the test of token t against its follower s on lane t G + s, then one
+      // vote per warp
+      const int my_t = lane / G, my_s = lane - (lane / G) * G;
+      const int i = i0 + r0 + my_t;
+      bool ok = false;
+      if (lane < TPW * G && i < n && my_s < min(G, n - 1 - i)) {
+        const float ni = red_s[warp][my_t], nj = red_s[warp][my_t + 1 + my_s];
+        const float d = red_s[warp][TPW + G + lane];
+        const float c = (ni > 0.f && nj > 0.f) ? d / (sqrtf(ni) * sqrtf(nj)) : 0.f;
+        ok = c >= tau;
+      }
+      const uint32_t vote = __ballot_sync(0xffffffffu, ok);
       uint32_t bits = 0;
 #pragma unroll
-      for (int t = 0; t < TPW; ++t) {
-        const int i = i0 + r0 + t;
-        if (i >= n_max) break;
-        bool ok = false;
-        if (i < n) {
-          const int gg = min(G, n - 1 - i);  // followers that exist
-#pragma unroll
-          for (int s = 0; s < G; ++s) {
-            if (s < gg) {
-              const float ni = nrm[t], nj = nrm_s[r0 + t + 1 + s];
-              const float c = (ni > 0.f && nj > 0.f) ? dt[t][s] / (sqrtf(ni) * sqrtf(nj)) : 0.f;
-              ok = ok || c >= tau;
-            }
-          }
-        }
-        pb[i] = ok ? 1 : 0;
-        bits |= ok ? (1u << t) : 0u;
-      }
-      nib[warp] = bits;
+      for (int t = 0; t < TPW; ++t)
+        bits |= ((vote >> (t * G)) & ((1u << G) - 1u)) ? (1u << t) : 0u;
+      if (lane < TPW && i0 + r0 + lane < n_max) pb[i0 + r0 + lane] = (bits >> lane) & 1u;
+      if (lane == 0) nib[warp] = bits;
     }
-    __syncthreads();
-    if (tid == 0) {
-      uint32_t word = 0;
-#pragma unroll
-      for (int w = 0; w < kPassThreads / 32; ++w) word |= nib[w] << (w * TPW);
-      masks[static_cast<long long>(b) * words_stride + i0 / kPassTile] = word;
-    }
+    tile_done(false);
   }
 }
 
@@ -249,26 +377,6 @@ __device__ __forceinline__ int block_excl_sum(int v, int* red, int* total) {
   *total = __shfl_sync(0xffffffffu, wv, 31);
   __syncthreads();
   return (warp > 0 ? before : 0) + v - mine;
-}
-
-// Kept tokens among the 32 tokens i0 .. i0+31 whose pass bits are `m`, given
-// lp, the last passing position before i0 (-1: none): the passing tokens,
-// and in every gap between a passing token (or lp) and the next one, the
-// positions at multiples of K after it.  One division per gap.
-__device__ __forceinline__ uint32_t keep_mask(uint32_t m, int lp, int i0, int K) {
-  uint32_t kept = m;
-  if (K <= 0) return kept;
-  int prev = lp, pos = i0;
-  uint32_t rest = m;
-  while (true) {
-    const int nxt = rest ? i0 + __ffs(rest) - 1 : i0 + 32;  // next passing token, or the end
-    for (int f = prev + K * ((pos - prev + K - 1) / K); f < nxt; f += K) kept |= 1u << (f - i0);
-    if (!rest) break;
-    prev = nxt;
-    pos = nxt + 1;
-    rest &= rest - 1;
-  }
-  return kept;
 }
 
 __device__ __forceinline__ void dn_cluster_sync() {
@@ -372,7 +480,9 @@ extern "C" {
 
 // [0, B * n_max): one pass byte per token; then, 256-byte aligned, one
 // 32-bit pass word per tile of 32 tokens, [B, words_stride] with the row
-// stride rounded up to whole 16-byte groups.
+// stride rounded up to whole 16-byte groups; then, 256-byte aligned, one
+// 32-bit tile counter per context (zero-filled once by the caller; every
+// call leaves them zero).
 static size_t dn_words_offset(int B, int n_max) {
   return cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(n_max), 256);
 }
@@ -381,10 +491,14 @@ static int dn_words_stride(int n_max) {
   return (words + cmc::kCompactWords - 1) / cmc::kCompactWords * cmc::kCompactWords;
 }
 
-size_t cmc_denoise_workspace_size(int B, int n_max) {
-  if (B < 1 || n_max < 1) return 0;
+static size_t dn_counters_offset(int B, int n_max) {
   const size_t words = static_cast<size_t>(B) * static_cast<size_t>(dn_words_stride(n_max));
   return cmc::align_up(dn_words_offset(B, n_max) + 4 * words, 256);
+}
+
+size_t cmc_denoise_workspace_size(int B, int n_max) {
+  if (B < 1 || n_max < 1) return 0;
+  return dn_counters_offset(B, n_max) + cmc::align_up(4 * static_cast<size_t>(B), 256);
 }
 
 int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int H, int g,
@@ -404,20 +518,24 @@ int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint8_t* pass = static_cast<uint8_t*>(workspace);
   uint32_t* masks = reinterpret_cast<uint32_t*>(pass + dn_words_offset(B, n_max));
+  unsigned int* counters = reinterpret_cast<unsigned int*>(pass + dn_counters_offset(B, n_max));
   static std::atomic<bool> attr_set[64];  // per device: the attribute is set (idempotent)
   int dev = 0;
   int st = record_cuda_error(cudaGetDevice(&dev));
   if (st != CMC_OK) return st;
   if (dev >= 0 && dev < 64 && !attr_set[dev].load(std::memory_order_acquire)) {
-    const void* kerns[8] = {
-        reinterpret_cast<const void*>(denoise_pass_kernel<1>), reinterpret_cast<const void*>(denoise_pass_kernel<2>),
-        reinterpret_cast<const void*>(denoise_pass_kernel<3>), reinterpret_cast<const void*>(denoise_pass_kernel<4>),
-        reinterpret_cast<const void*>(denoise_pass_kernel<5>), reinterpret_cast<const void*>(denoise_pass_kernel<6>),
-        reinterpret_cast<const void*>(denoise_pass_kernel<7>), reinterpret_cast<const void*>(denoise_pass_kernel<8>)};
-    for (const void* k : kerns) {
-      st = record_cuda_error(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, kPassSmem));
-      if (st != CMC_OK) return st;
-    }
+#define CMC_DN_ATTR(GG)                                                                                 \
+    st = record_cuda_error(cudaFuncSetAttribute(denoise_pass_kernel<GG, kPassStages, false>,           \
+                                                cudaFuncAttributeMaxDynamicSharedMemorySize,           \
+                                                pass_smem(kPassStages)));                               \
+    if (st != CMC_OK) return st;                                                                        \
+    st = record_cuda_error(cudaFuncSetAttribute(denoise_pass_kernel<GG, kPassStages, true>,       \
+                                                cudaFuncAttributeMaxDynamicSharedMemorySize,           \
+                                                pass_smem(kPassStages)));                          \
+    if (st != CMC_OK) return st;
+    CMC_DN_ATTR(1) CMC_DN_ATTR(2) CMC_DN_ATTR(3) CMC_DN_ATTR(4)
+    CMC_DN_ATTR(5) CMC_DN_ATTR(6) CMC_DN_ATTR(7) CMC_DN_ATTR(8)
+#undef CMC_DN_ATTR
     attr_set[dev].store(true, std::memory_order_release);
   }
   const int tiles_per_ctx = (n_max + kPassTile - 1) / kPassTile;
@@ -425,19 +543,29 @@ int cmc_denoise(const float* emb, const int32_t* n_tokens, int B, int n_max, int
   long long blocks = tiles;
   const long long cap = static_cast<long long>(sm_count()) * 2 * 64;  // grid-stride beyond
   if (blocks > cap) blocks = cap;
+  // Contexts of at most kPassThreads tiles (8,192 tokens): the compaction in
+  // the same launch; longer ones: the cluster compaction kernel after the pass.
+  const bool fuse = tiles_per_ctx <= kPassThreads;
   switch (g) {
 #define CMC_DN_CASE(GG)                                                                             \
   case GG:                                                                                          \
-    st = launch_pdl(denoise_pass_kernel<GG>, dim3(static_cast<unsigned>(blocks)), dim3(kPassThreads), \
-                    static_cast<size_t>(kPassSmem), s, emb, n_tokens, n_max, H, tau, pass, masks,  \
-                    kept_idx, tiles, tiles_per_ctx, dn_words_stride(n_max));                        \
+    st = fuse ? launch_pdl(denoise_pass_kernel<GG, kPassStages, true>,                         \
+                           dim3(static_cast<unsigned>(blocks)), dim3(kPassThreads),                 \
+                           static_cast<size_t>(pass_smem(kPassStages)), s, emb, n_tokens,      \
+                           n_max, H, tau, pass, masks, kept_idx, tiles, tiles_per_ctx,              \
+                           dn_words_stride(n_max), counters, keep_every, kept_count)                \
+              : launch_pdl(denoise_pass_kernel<GG, kPassStages, false>,                             \
+                           dim3(static_cast<unsigned>(blocks)), dim3(kPassThreads),                 \
+                           static_cast<size_t>(pass_smem(kPassStages)), s, emb, n_tokens, n_max, H, \
+                           tau, pass, masks, kept_idx, tiles, tiles_per_ctx,                        \
+                           dn_words_stride(n_max), counters, keep_every, kept_count);               \
     break;
     CMC_DN_CASE(1) CMC_DN_CASE(2) CMC_DN_CASE(3) CMC_DN_CASE(4)
     CMC_DN_CASE(5) CMC_DN_CASE(6) CMC_DN_CASE(7) CMC_DN_CASE(8)
 #undef CMC_DN_CASE
     default: return CMC_ERR_RANGE;
   }
-  if (st != CMC_OK) return st;
+  if (st != CMC_OK || fuse) return st;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;

@@ -207,6 +207,9 @@ struct LocateArgs {
   int W;
   int32_t* alpha_out;           // [B] (nullable)
   int32_t* start_out;           // [B] (nullable)
+  // [B] or NULL: the one-launch path's argmax slots, (orderable squared norm
+  // << 32) | ~index, raised by every scoring CTA (zero before, zero after)
+  unsigned long long* best = nullptr;
 };
 
 __device__ __forceinline__ void locate_window(const LocateArgs& la, int b, int N) {
@@ -611,15 +614,9 @@ __device__ __forceinline__ uint32_t fused_scan(uint32_t v, uint32_t* ws) {
 // position); padding keys are 0, below every score's key.  Every thread of
 // the CTA calls it.
 template <int KPT>
-__device__ __forceinline__ void fused_topk(const float* sc, int N, int k, int32_t* out,
+__device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int k, int32_t* out,
                                            uint32_t* scan_eq, uint32_t* scan_sel) {
   const int tid = threadIdx.x;
-  uint32_t key[KPT];
-#pragma unroll
-  for (int e = 0; e < KPT; ++e) {
-    const int j = tid * KPT + e;
-    key[e] = j < N ? orderable(__ldcg(sc + j)) : 0u;
-  }
   // the k-th largest key: the largest T with at least k keys >= T, one bit a
   // round from the top; a round counts over the block with KPT counting barriers
   uint32_t T = 0u;
@@ -654,54 +651,55 @@ __device__ __forceinline__ void fused_topk(const float* sc, int N, int k, int32_
 }
 
 // The selection (and, with la.sqnorm, the localisation) of sequence b by the
-// CTA that completed its scores.  Every thread of the CTA calls it.
-__device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
+// CTA that completed its scores.  Every thread of the CTA calls it.  Thread
+// 0's acq_rel counter addition acquired the other CTAs' writes (scores, and
+// their raises of the argmax slot); the caller's barrier passed that order on
+// to every thread.  The localisation is one slot read by thread 0, issued
+// with the score loads; its chunk-offset load then runs under the search and
+// its result is written at the end.
+template <int KPT>
+__device__ __forceinline__ void fused_select_impl(const FusedArgs& a, int b) {
   __shared__ uint32_t scan_eq[kFusedWarps], scan_sel[kFusedWarps];
-  __shared__ float best_v[kFusedWarps];
-  __shared__ int best_i[kFusedWarps];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x;
   const int N = a.N, k = a.k;
-  // thread 0's acq_rel counter addition acquired the other CTAs' score
-  // writes; the caller's barrier passed that order on to every thread
-  if (a.la.sqnorm) {
-    // CME-guided localisation: argmax of the squared norms, ties to the lower index
-    const float* sq = a.la.sqnorm + static_cast<long long>(b) * N;
-    float best = -1.f;
-    int bi = 0x7fffffff;
-    for (int j = tid; j < N; j += kFusedThreads) {
-      const float v = __ldcg(sq + j);
-      if (v > best) { best = v; bi = j; }
-    }
+  const bool topk = k > 0 && k < N;
+  const float* sc = a.scores + static_cast<long long>(b) * N;
+  uint32_t key[KPT];
 #pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, best, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-      if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
-    }
-    if (lane == 0) { best_v[warp] = best; best_i[warp] = bi; }
-    __syncthreads();
-    if (tid == 0) {
-      for (int w = 1; w < kFusedWarps; ++w)
-        if (best_v[w] > best || (best_v[w] == best && best_i[w] < bi)) { best = best_v[w]; bi = best_i[w]; }
-      const long long alpha = a.la.chunk_offset[static_cast<long long>(b) * N + bi];
-      long long st = static_cast<long long>(a.la.ctx_len[b]) - a.la.W;
-      const long long centred = alpha - a.la.W / 2;
-      if (centred < st) st = centred;
-      if (st < 0) st = 0;
-      if (a.la.alpha_out) a.la.alpha_out[b] = static_cast<int32_t>(alpha);
-      if (a.la.start_out) a.la.start_out[b] = static_cast<int32_t>(st);
-    }
+  for (int e = 0; e < KPT; ++e) {
+    const int j = tid * KPT + e;
+    key[e] = (topk && j < N) ? orderable(__ldcg(sc + j)) : 0u;
+  }
+  const bool locate = a.la.sqnorm && tid == 0;
+  int32_t alpha = 0, clen = 0;
+  if (locate) {
+    const unsigned long long packed = __ldcg(a.la.best + b);
+    a.la.best[b] = 0ull;  // ready for the next call
+    const int bi = static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(packed & 0xFFFFFFFFull));
+    alpha = __ldg(a.la.chunk_offset + static_cast<long long>(b) * N + bi);
+    clen = __ldg(a.la.ctx_len + b);
   }
   int32_t* out = a.idx_out + static_cast<long long>(b) * k;
-  const float* sc = a.scores + static_cast<long long>(b) * N;
   if (k >= N) {
     for (int j = tid; j < N; j += kFusedThreads) out[j] = j;
   } else if (k > 0) {
-    if (N <= kFusedThreads) fused_topk<1>(sc, N, k, out, scan_eq, scan_sel);
-    else fused_topk<2>(sc, N, k, out, scan_eq, scan_sel);
+    fused_topk<KPT>(key, k, out, scan_eq, scan_sel);
+  }
+  if (locate) {
+    long long st = static_cast<long long>(clen) - a.la.W;
+    const long long centred = static_cast<long long>(alpha) - a.la.W / 2;
+    if (centred < st) st = centred;
+    if (st < 0) st = 0;
+    if (a.la.alpha_out) a.la.alpha_out[b] = alpha;
+    if (a.la.start_out) a.la.start_out[b] = static_cast<int32_t>(st);
   }
   if (tid == 0) a.counters[b] = 0u;  // ready for the next call
   __syncthreads();                    // the shared scratch is reused by the caller
+}
+
+__device__ __noinline__ void fused_select(const FusedArgs& a, int b) {
+  if (a.N <= kFusedThreads) fused_select_impl<1>(a, b);
+  else fused_select_impl<2>(a, b);
 }
 
 // 16-byte asynchronous copy global -> shared (cp.async), through L2 only.
@@ -723,6 +721,7 @@ score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
   extern __shared__ float4 rows_s[];
   __shared__ float part[kFusedWarps][2 * RG];
   __shared__ float qq_part[kFusedWarps];
+  __shared__ float rsq_s[kFusedRows];  // the rows' squared norms (localisation)
   __shared__ int last_flag;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int D4 = a.D >> 2;
@@ -823,12 +822,27 @@ score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
       if (sc == 0.f) sc = 0.f;  // -0 -> +0, so that -0 and +0 tie
       a.scores[r0 + warp] = sc;
       if (a.la.sqnorm) a.la.sqnorm[r0 + warp] = sm;
+      rsq_s[warp] = sm;
     }
   }
   __syncthreads();
   if (tid == 0) {
-    // acq_rel at GPU scope: releases the CTA's score writes (they precede it
-    // through the barrier) and, for the last CTA, acquires everyone else's
+    if (a.la.sqnorm) {
+      // this CTA's largest squared norm (lowest index on ties, NaN lowest),
+      // raised into the sequence's argmax slot
+      unsigned long long top = 0ull;
+      for (int r = 0; r < R; ++r) {
+        const float v = rsq_s[r];
+        const unsigned long long key = isnan(v) ? 0ull : orderable(v);
+        const unsigned long long p =
+            (key << 32) | (0xFFFFFFFFu - static_cast<uint32_t>(r0 + r - b * a.N));
+        top = p > top ? p : top;
+      }
+      atomicMax(a.la.best + b, top);
+    }
+    // acq_rel at GPU scope: releases the CTA's writes (they precede it through
+    // the barrier, and this thread's raise in program order) and, for the
+    // last CTA, acquires everyone else's
     unsigned int old;
     asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], %2;\n"
                  : "=r"(old)
@@ -1000,7 +1014,8 @@ int cmc_score_select(const float* question_emb, const float* cme_bank, int B, in
 size_t cmc_question_select_workspace_size(int B, int N) {
   if (B < 1 || N < 1) return 0;
   return 2 * cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256) +
-         cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256);
+         cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256) +
+         cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned long long), 256);
 }
 
 int cmc_question_select(const float* question_tokens, const int32_t* q_len, int Lq,
@@ -1028,14 +1043,17 @@ int cmc_question_select(const float* question_tokens, const int32_t* q_len, int 
     if (reinterpret_cast<uintptr_t>(ptr) & 3) return CMC_ERR_ALIGN;
   if (workspace_bytes < cmc_question_select_workspace_size(B, N)) return CMC_ERR_WORKSPACE;
   // Workspace: [scores][squared norms] (B * N fp32 each, 256-byte aligned)
-  // [B completion counters].
+  // [B completion counters][B argmax slots] (the last two zero between calls).
   const size_t scores_bytes = align_up(static_cast<size_t>(B) * N * sizeof(float), 256);
   float* sc = static_cast<float*>(workspace);
   float* sq = sc + scores_bytes / sizeof(float);
   unsigned int* counters =
       reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + 2 * scores_bytes);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out};
+  unsigned long long* best = reinterpret_cast<unsigned long long*>(
+      static_cast<char*>(workspace) + 2 * scores_bytes +
+      align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256));
+  LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out, best};
   // small banks: pooling, scoring, selection and localisation in one launch
   const int fused_rows = fused_rows_per_cta(B, N, D);
   if (fused_rows > 0)

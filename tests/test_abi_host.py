@@ -214,7 +214,8 @@ def test_decode_step_rope_argument_checks(L):
 
 
 def test_question_select_workspace_size(L):
-    assert L.cmc_question_select_workspace_size(3, 100) == 2 * 1280 + 256
+    # scores and squared norms (1,200 bytes each -> 1,280), 3 counters, 3 slots
+    assert L.cmc_question_select_workspace_size(3, 100) == 2 * 1280 + 256 + 256
     assert L.cmc_question_select_workspace_size(0, 100) == 0
 
 
@@ -257,8 +258,8 @@ def test_bridge_epilogue_argument_checks(L):
 
 
 def test_denoise_workspace_size(L):
-    # 2,000 pass bytes (to 2,048), then 2 x 32 pass words of 4 bytes
-    assert L.cmc_denoise_workspace_size(2, 1000) == 2048 + 256
+    # flags 2,000 -> 2,048; words 2 x 32 -> 256; counters 2 x 4 -> 256
+    assert L.cmc_denoise_workspace_size(2, 1000) == 2048 + 256 + 256
     assert L.cmc_denoise_workspace_size(0, 10) == 0
 
 

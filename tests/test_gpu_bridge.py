@@ -29,10 +29,11 @@ def _case(rows, D, nu, scale, affine, dev, seed=0, in_place=False):
     return ref
 
 
-# D = 64 and 36: one float4 per thread; 2048, 3072, 4096: two to four (rows in
-# registers); 16384: rows staged in shared memory
+# rows in registers, one 128-thread CTA per row: D = 64 and 36 take one float4
+# per thread, 1028 three (the last one partial), 2048 four, 2600 six, 3072 six,
+# 3588 eight (partial), 4096 eight; 16384: rows staged in shared memory
 @pytest.mark.parametrize("rows,D", [(1024, 4096), (300, 64), (7, 16384), (50, 36), (33, 2048),
-                                    (17, 3072)])
+                                    (17, 3072), (29, 1028), (21, 2600), (13, 3588)])
 @pytest.mark.parametrize("affine", [False, True])
 def test_bridge_epilogue_shapes(cuda_device, rows, D, affine):
     ref = _case(rows, D, 0.8, 2.0, affine, cuda_device)

@@ -32,9 +32,11 @@ def _ambiguous(emb_b, n, g, tau):
     return amb
 
 
-def _check(emb, n_tok, g, tau, every, dev, pass_n_tokens=True, whole=True):
+def _check(emb, n_tok, g, tau, every, dev, pass_n_tokens=True, whole=True, ws=None):
     B, n_max, _ = emb.shape
-    ws = torch.empty(cmc.lib().cmc_denoise_workspace_size(B, n_max), dtype=torch.uint8, device=dev)
+    if ws is None:
+        ws = torch.zeros(cmc.lib().cmc_denoise_workspace_size(B, n_max), dtype=torch.uint8,
+                         device=dev)
     kept, cnt = cmc.denoise(torch.from_numpy(emb).to(dev),
                             n_tokens=torch.from_numpy(n_tok).to(dev) if pass_n_tokens else None,
                             g=g, tau=tau, keep_every=every, workspace=ws)
@@ -87,3 +89,23 @@ def test_denoise_edge_cases(cuda_device):
     assert cnt.tolist() == [300 // 16, 217 // 16, 0, 0]
     full = np.nan_to_num(emb, nan=1.0)
     _check(full, np.full(B, n, dtype=np.int32), 3, 0.3, 16, cuda_device, pass_n_tokens=False)
+
+
+def test_denoise_one_launch_and_two_launch_paths(cuda_device):
+    """Contexts of 256 tiles of 32 tokens (the compaction runs in the pass
+    launch, counted per context in the workspace) and of 257 (the cluster
+    compaction kernel), one and several contexts, ragged last tiles; the same
+    workspace serves repeated calls and its counters are zero after each."""
+    rng = np.random.default_rng(5)
+    H = 128
+    for B, tiles in ((1, 256), (1, 257), (3, 256), (2, 3)):
+        n_max = 32 * tiles - 7                     # a ragged last tile
+        steps = rng.standard_normal((B, n_max, H)).astype(np.float32)
+        emb = np.cumsum(steps, axis=1).astype(np.float32)
+        n_tok = np.array([n_max - 45 * b for b in range(B)], dtype=np.int32)
+        ws = torch.zeros(cmc.lib().cmc_denoise_workspace_size(B, n_max), dtype=torch.uint8,
+                         device=cuda_device)
+        for rep in range(3):
+            _check(emb, n_tok, 3, 0.3, 16, cuda_device, whole=rep == 0, ws=ws)
+            tail = ws[-256:].cpu().numpy()
+            assert not tail.any(), "completion counters not left at zero"

@@ -78,3 +78,34 @@ def test_question_prologue_edge_cases(cuda_device):
     assert int(start[2]) == 0 and int(start[3]) == 400 - W
     # no q_len: every question uses all Lq rows
     _check(tokens, None, bank, 5, offs, clen, W, cuda_device)
+
+
+def test_question_prologue_ties_inside_a_cta_and_workspace_reuse(cuda_device):
+    """Largest norms tied inside one CTA's rows and across CTAs (the lowest
+    index wins), in the one-launch path; the same workspace serves repeated
+    calls and its completion counters and argmax slots are zero after each."""
+    rng = np.random.default_rng(12)
+    B, Lq, N, D, W, k = 3, 5, 64, 48, 16, 9
+    tokens = rng.standard_normal((B, Lq, D)).astype(np.float32)
+    bank = rng.standard_normal((B, N, D)).astype(np.float32)
+    big = np.abs(bank).max() * 4.0
+    bank[0, 13] = bank[0, 12] = big       # the same CTA for every rows-per-CTA up to 8: 12 wins
+    bank[1, 40] = bank[1, 3] = big        # different CTAs: 3 wins
+    bank[2, 63] = big                     # the last row
+    q_len = np.array([5, 2, 4], dtype=np.int32)
+    offs = np.tile(np.arange(N, dtype=np.int32) * 7, (B, 1))
+    clen = np.full(B, 7 * N, dtype=np.int32)
+    ws = torch.zeros(cmc.lib().cmc_question_select_workspace_size(B, N), dtype=torch.uint8,
+                     device=cuda_device)
+    rq, ridx, _, ralpha, rstart = oracle.question_select(tokens, q_len, bank, k, offs, clen, W)
+    assert ralpha.tolist() == [offs[0, 12], offs[1, 3], offs[2, 63]]
+    for _ in range(3):
+        q, idx, alpha, start = cmc.question_select(
+            _dev(tokens, cuda_device), _dev(bank, cuda_device), k,
+            q_len=_dev(q_len, cuda_device), chunk_offset=_dev(offs, cuda_device),
+            ctx_len=_dev(clen, cuda_device), W=W, workspace=ws)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(idx.cpu().numpy(), ridx)
+        np.testing.assert_array_equal(alpha.cpu().numpy(), ralpha)
+        np.testing.assert_array_equal(start.cpu().numpy(), rstart)
+        assert not ws[-512:].cpu().numpy().any(), "counters or argmax slots not left at zero"
