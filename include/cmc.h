@@ -153,7 +153,7 @@ CMC_API int cmc_bridge_epilogue(const float* x, const float* gamma, const float*
 
 /* Bytes of workspace cmc_score_select needs for B sequences of N CMEs: the
  * B * N fp32 scores (rounded up to 256 bytes), then B completion counters
- * (rounded up to 256 bytes). */
+ * (rounded up to 256 bytes), then B histograms of 2,048 32-bit counts. */
 CMC_API size_t cmc_score_select_workspace_size(int B, int N);
 
 /*
@@ -168,14 +168,17 @@ CMC_API size_t cmc_score_select_workspace_size(int B, int N);
  *   scores_out    fp32 [B, N]       optional output (NULL: not written)
  *   workspace     >= cmc_score_select_workspace_size(B, N) bytes, 16-byte
  *                 aligned, ZERO-FILLED ONCE before its first use: it holds
- *                 one completion counter per sequence, which every call leaves
- *                 at zero again (the scores part may hold anything).  It may
+ *                 one completion counter and one histogram of the scores'
+ *                 top 11 key bits per sequence, which every call leaves at
+ *                 zero again (the scores part may hold anything).  Calls that
+ *                 share a workspace must be ordered (e.g. one stream).  It may
  *                 be NULL when scores_out is given.
  *
  * Small banks with a workspace (D <= 4096, N <= 2048, and B * N rows that
  * CTAs of at most 8 rows of one sequence cover in one wave of one CTA per SM)
  * take one kernel launch: the CTA that writes the last score of a sequence (a
- * counter in the workspace tells it) selects that sequence's top k.  Larger
+ * counter in the workspace tells it) selects that sequence's top k, starting
+ * from the histogram the scoring CTAs built.  Larger
  * banks, or no workspace, take two launches (scoring, then selection).  Both
  * give the same selection.
  *
@@ -220,8 +223,8 @@ CMC_API size_t cmc_question_select_workspace_size(int B, int N);
  *   workspace        >= cmc_question_select_workspace_size(B, N) bytes,
  *                    16-byte aligned, zero-filled once before its first use
  *                    (as for cmc_score_select: scores, squared norms, then
- *                    B completion counters and B 64-bit argmax slots, both
- *                    left at zero by every call)
+ *                    B completion counters, B histograms of 2,048 counts and
+ *                    B 64-bit argmax slots, all left at zero by every call)
  *
  * Small banks (as for cmc_score_select) take one kernel launch for the whole
  * prologue; larger ones three (pooling, scoring, selection).  q_vec is the

@@ -552,11 +552,11 @@ topk_select_cluster_kernel(const float* __restrict__ scores, int N, int k,
 // releases the CTA's score writes and acquires those of the CTAs before it);
 // the CTA whose addition completes N is the last to score that sequence and
 // selects its top k itself.  Keys are the order-
-// preserving uint32 images of the scores; a bit-by-bit search from the top
-// bit finds the largest T with at least k keys >= T (the k-th largest key),
-// each round one counting barrier (__syncthreads_count) per key a thread
-// holds; an ordered compaction then writes the keys > T and the lowest-index
-// keys == T in ascending index order.  It puts the counter back to zero for
+// preserving uint32 images of the scores; each scoring CTA adds its rows to a
+// histogram of the top 11 key bits in the workspace, and the selecting CTA
+// finds the k-th largest key T from it and two shared-memory histogram levels
+// (bits 20..10, 9..0); an ordered compaction then writes the keys > T and
+// the lowest-index keys == T in ascending index order.  It puts the counter back to zero for
 // the next call.  No CTA waits on another.
 // ---------------------------------------------------------------------------
 
@@ -565,6 +565,7 @@ constexpr int kFusedWarps = kFusedThreads / 32;
 constexpr int kFusedRows = 8;                    // rows per CTA at most
 constexpr int kFusedMaxD = 4 * kFusedThreads;    // one float4 per thread and row
 constexpr int kFusedMaxN = 2 * kFusedThreads;    // two keys per thread in the selection
+constexpr int kHistTop = 2048;                   // bins of the top 11 bits of a key
 
 struct FusedArgs {
   const float* qv;        // [B, D], or NULL: pooled from q_tokens
@@ -579,6 +580,7 @@ struct FusedArgs {
   unsigned int* counters; // [B]: zero before the call, zero after it
   int32_t* idx_out;       // [B, k]
   LocateArgs la;          // la.sqnorm: also write squared norms and localise
+  unsigned int* hist;     // [B, kHistTop]: counts of the scores' top 11 key bits (zero before, zero after)
 };
 
 // Exclusive prefix sum over the block of one value per thread (warps in
@@ -608,31 +610,73 @@ __device__ __forceinline__ uint32_t fused_scan(uint32_t v, uint32_t* ws) {
   return before + inc - v;
 }
 
+// One level of the histogram search for the k-th largest key: thread t holds
+// the counts of bins bin_a > bin_b (the bins in descending order across the
+// threads); an exclusive prefix sum over the block gives the keys in the bins
+// above, and the thread whose bins hold the rem-th key (counting from the
+// top) publishes the bin and the rank of that key within it.
+__device__ __forceinline__ void hist_level(uint32_t ha, uint32_t bin_a, uint32_t hb, uint32_t bin_b,
+                                           uint32_t& rem, uint32_t& digit, uint32_t* ws,
+                                           uint32_t* pick) {
+  const uint32_t above = fused_scan(ha + hb, ws);
+  if (above < rem && rem <= above + ha) {
+    pick[0] = bin_a;
+    pick[1] = rem - above;
+  } else if (above + ha < rem && rem <= above + ha + hb) {
+    pick[0] = bin_b;
+    pick[1] = rem - above - ha;
+  }
+  __syncthreads();
+  digit = pick[0];
+  rem = pick[1];
+}
+
 // Top k of one sequence's N scores (N <= KPT * kFusedThreads), written to
 // out[0..k) in ascending index order.  Thread t holds the keys of indices
 // t*KPT .. t*KPT + KPT - 1 in registers (index order is thread order, then
-// position); padding keys are 0, below every score's key.  Every thread of
-// the CTA calls it.
+// position).  Every thread of the CTA calls it.
+//
+// The k-th largest key T is found in three histogram levels: its top 11 bits
+// from the histogram the scoring CTAs built in `ghist` (read, then zeroed for
+// the next call), bits 20..10 from a shared-memory histogram of the keys with
+// those top bits, bits 9..0 likewise; each level is one prefix sum over the
+// bins (two a thread) -- eight barriers in all, against 32 counting barriers
+// for a bit-by-bit search.  The ordered compaction then writes the keys > T
+// and the lowest-index keys == T.
 template <int KPT>
-__device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int k, int32_t* out,
-                                           uint32_t* scan_eq, uint32_t* scan_sel) {
+__device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int N, int k, int32_t* out,
+                                           uint32_t* ghist, uint32_t* scan_eq,
+                                           uint32_t* scan_sel) {
+  __shared__ uint32_t h2[kHistTop], h3[kHistTop / 2], pick[2];
   const int tid = threadIdx.x;
-  // the k-th largest key: the largest T with at least k keys >= T, one bit a
-  // round from the top; a round counts over the block with KPT counting barriers
-  uint32_t T = 0u;
-  for (int bit = 31; bit >= 0; --bit) {
-    const uint32_t c = T | (1u << bit);
-    int n = 0;
+  static_assert(kHistTop == 2 * kFusedThreads, "two top bins a thread");
+  h2[2 * tid] = 0u;
+  h2[2 * tid + 1] = 0u;
+  h3[tid] = 0u;
+  // level 1 (bits 31..21): thread t takes bins 2047 - 2t and 2046 - 2t
+  const uint32_t ba = kHistTop - 1 - 2 * tid, bb = ba - 1;
+  const uint32_t ga = __ldcg(ghist + ba), gb = __ldcg(ghist + bb);
+  ghist[ba] = 0u;
+  ghist[bb] = 0u;
+  uint32_t rem = static_cast<uint32_t>(k), d;
+  hist_level(ga, ba, gb, bb, rem, d, scan_sel, pick);
+  uint32_t T = d << 21;
+  // level 2 (bits 20..10) among the keys with those top bits
 #pragma unroll
-    for (int e = 0; e < KPT; ++e) n += __syncthreads_count(key[e] >= c);
-    if (n >= k) T = c;
-  }
-  int gt = 0;  // keys > T
-  if (T != 0xFFFFFFFFu) {
+  for (int e = 0; e < KPT; ++e)
+    if (tid * KPT + e < N && (key[e] >> 21) == (T >> 21)) atomicAdd(h2 + ((key[e] >> 10) & 2047u), 1u);
+  __syncthreads();
+  hist_level(h2[ba], ba, h2[bb], bb, rem, d, scan_sel, pick);
+  T |= d << 10;
+  // level 3 (bits 9..0): thread t takes bin 1023 - t
 #pragma unroll
-    for (int e = 0; e < KPT; ++e) gt += __syncthreads_count(key[e] > T);
-  }
-  const uint32_t need = static_cast<uint32_t>(k - gt);  // keys == T to keep, lowest index first
+  for (int e = 0; e < KPT; ++e)
+    if (tid * KPT + e < N && (key[e] >> 10) == (T >> 10)) atomicAdd(h3 + (key[e] & 1023u), 1u);
+  __syncthreads();
+  const uint32_t bc = kHistTop / 2 - 1 - tid;
+  hist_level(h3[bc], bc, 0u, 0u, rem, d, scan_sel, pick);
+  T |= d;
+  const uint32_t need = rem;  // keys == T to keep, lowest index first (k - need keys are > T)
   uint32_t n_gt = 0, n_eq = 0;
 #pragma unroll
   for (int e = 0; e < KPT; ++e) {
@@ -683,7 +727,7 @@ __device__ __forceinline__ void fused_select_impl(const FusedArgs& a, int b) {
   if (k >= N) {
     for (int j = tid; j < N; j += kFusedThreads) out[j] = j;
   } else if (k > 0) {
-    fused_topk<KPT>(key, k, out, scan_eq, scan_sel);
+    fused_topk<KPT>(key, N, k, out, a.hist + static_cast<long long>(b) * kHistTop, scan_eq, scan_sel);
   }
   if (locate) {
     long long st = static_cast<long long>(clen) - a.la.W;
@@ -821,6 +865,7 @@ score_select_fused_kernel(const __grid_constant__ FusedArgs a) {
       if (sm > 0.f && qq > 0.f) sc = sd / (sqrtf(sm) * sqrtf(qq));
       if (sc == 0.f) sc = 0.f;  // -0 -> +0, so that -0 and +0 tie
       a.scores[r0 + warp] = sc;
+      atomicAdd(a.hist + static_cast<long long>(b) * kHistTop + (orderable(sc) >> 21), 1u);
       if (a.la.sqnorm) a.la.sqnorm[r0 + warp] = sm;
       rsq_s[warp] = sm;
     }
@@ -898,6 +943,9 @@ static int launch_score_select_fused(const float* question_emb, const float* cme
   a.counters = counters;
   a.idx_out = idx_out;
   a.la = la;
+  // the histograms follow the counters in the workspace
+  a.hist = reinterpret_cast<unsigned int*>(reinterpret_cast<char*>(counters) +
+                                           align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256));
   const long long ctas = static_cast<long long>(B) * N / R;
   return launch_pdl(score_select_fused_kernel, dim3(static_cast<unsigned>(ctas)),
                     dim3(kFusedThreads), fused_smem_bytes(), s, a);
@@ -974,10 +1022,13 @@ static int launch_score_select(const float* question_emb, const float* cme_bank,
 
 extern "C" {
 
+// [scores: B N fp32][B completion counters][B x kHistTop histogram counts],
+// each part 256-byte aligned; the last two zero between calls.
 size_t cmc_score_select_workspace_size(int B, int N) {
   if (B < 1 || N < 1) return 0;
   return cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256) +
-         cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256);
+         cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256) +
+         static_cast<size_t>(B) * cmc::kHistTop * sizeof(unsigned int);
 }
 
 int cmc_score_select(const float* question_emb, const float* cme_bank, int B, int N, int D, int k,
@@ -1015,6 +1066,7 @@ size_t cmc_question_select_workspace_size(int B, int N) {
   if (B < 1 || N < 1) return 0;
   return 2 * cmc::align_up(static_cast<size_t>(B) * static_cast<size_t>(N) * sizeof(float), 256) +
          cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256) +
+         static_cast<size_t>(B) * cmc::kHistTop * sizeof(unsigned int) +
          cmc::align_up(static_cast<size_t>(B) * sizeof(unsigned long long), 256);
 }
 
@@ -1043,7 +1095,8 @@ int cmc_question_select(const float* question_tokens, const int32_t* q_len, int 
     if (reinterpret_cast<uintptr_t>(ptr) & 3) return CMC_ERR_ALIGN;
   if (workspace_bytes < cmc_question_select_workspace_size(B, N)) return CMC_ERR_WORKSPACE;
   // Workspace: [scores][squared norms] (B * N fp32 each, 256-byte aligned)
-  // [B completion counters][B argmax slots] (the last two zero between calls).
+  // [B completion counters][B x kHistTop histogram counts][B argmax slots]
+  // (the last three zero between calls).
   const size_t scores_bytes = align_up(static_cast<size_t>(B) * N * sizeof(float), 256);
   float* sc = static_cast<float*>(workspace);
   float* sq = sc + scores_bytes / sizeof(float);
@@ -1052,7 +1105,8 @@ int cmc_question_select(const float* question_tokens, const int32_t* q_len, int 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   unsigned long long* best = reinterpret_cast<unsigned long long*>(
       static_cast<char*>(workspace) + 2 * scores_bytes +
-      align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256));
+      align_up(static_cast<size_t>(B) * sizeof(unsigned int), 256) +
+      static_cast<size_t>(B) * kHistTop * sizeof(unsigned int));
   LocateArgs la{locate ? sq : nullptr, chunk_offset, ctx_len, W, alpha_out, start_out, best};
   // small banks: pooling, scoring, selection and localisation in one launch
   const int fused_rows = fused_rows_per_cta(B, N, D);

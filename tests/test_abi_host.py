@@ -81,8 +81,9 @@ def test_score_select_argument_checks(L):
 
 
 def test_score_select_workspace_size(L):
-    # 1200 bytes of scores rounded up to 256, then 3 counters rounded up to 256
-    assert L.cmc_score_select_workspace_size(3, 100) == 1280 + 256
+    # 1200 bytes of scores rounded up to 256, 3 counters rounded up to 256,
+    # then 3 histograms of 2,048 counts
+    assert L.cmc_score_select_workspace_size(3, 100) == 1280 + 256 + 3 * 8192
     assert L.cmc_score_select_workspace_size(0, 100) == 0
 
 
@@ -214,8 +215,9 @@ def test_decode_step_rope_argument_checks(L):
 
 
 def test_question_select_workspace_size(L):
-    # scores and squared norms (1,200 bytes each -> 1,280), 3 counters, 3 slots
-    assert L.cmc_question_select_workspace_size(3, 100) == 2 * 1280 + 256 + 256
+    # scores and squared norms (1,200 bytes each -> 1,280), 3 counters, 3
+    # histograms of 2,048 counts, 3 argmax slots
+    assert L.cmc_question_select_workspace_size(3, 100) == 2 * 1280 + 256 + 3 * 8192 + 256
     assert L.cmc_question_select_workspace_size(0, 100) == 0
 
 

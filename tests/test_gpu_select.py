@@ -164,17 +164,20 @@ def test_select_negative_and_signed_zero_scores(cuda_device):
     assert not np.signbit(scores[0, 3])
 
 
-def test_one_launch_counters_reset_across_calls(cuda_device):
-    """One workspace over calls on different banks: every call selects exactly
-    the planted set, and leaves the completion counters at zero."""
-    w = WORKLOADS["mistral_batched"]
-    ws = torch.zeros(cmc.score_select_workspace_size(8, w.N), dtype=torch.uint8,
+@pytest.mark.parametrize("name,B", [("mistral_batched", 8), ("llama3_8b", 1), ("tiny", 2)])
+def test_one_launch_counters_reset_across_calls(cuda_device, name, B):
+    """One workspace over calls on different banks (the one-launch path at the
+    Llama and tiny shapes, two launches for the Mistral batch): every call
+    selects exactly the planted set, and leaves the completion counters and
+    the score histograms at zero."""
+    w = WORKLOADS[name]
+    ws = torch.zeros(cmc.score_select_workspace_size(B, w.N), dtype=torch.uint8,
                      device=cuda_device)
-    for batch in (range(0, 8), range(8, 16), range(0, 8)):
+    scores_bytes = -(-B * w.N * 4 // 256) * 256
+    for batch in (range(0, B), range(B, 2 * B), range(0, B)):
         si = selection_inputs(w, batch=batch)
         idx = cmc.score_select(dev_f32(si.question_emb, cuda_device),
                                dev_f32(si.cme_bank, cuda_device), w.k, workspace=ws)
         torch.cuda.synchronize()
         np.testing.assert_array_equal(idx.cpu().numpy(), si.planted_idx)
-        counters = ws[-256:].view(torch.int32)[:8]
-        assert int(counters.abs().sum()) == 0
+        assert not ws[scores_bytes:].cpu().numpy().any(), "counters or histograms left non-zero"
