@@ -22,6 +22,8 @@ made once per question by :func:`tier1_gather` is passed.
 from __future__ import annotations
 
 import ctypes
+import functools
+import os
 from typing import Dict, Optional, Tuple
 
 import torch
@@ -48,6 +50,27 @@ __all__ = [
     "DEVFLAG_BAD_POS",
     "DEVFLAG_TIMEOUT",
 ]
+
+
+# With CMC_NVTX set (not "0") when the module is imported, every device call
+# below is wrapped in an NVTX range named after it ("cmc.decode_step", ...),
+# for profiler timelines; otherwise the functions are left as they are.
+_NVTX = os.environ.get("CMC_NVTX", "") not in ("", "0")
+
+
+def _ranged(fn):
+    if not _NVTX:
+        return fn
+    name = "cmc." + fn.__name__
+
+    @functools.wraps(fn)
+    def wrapped(*args, **kwargs):
+        torch.cuda.nvtx.range_push(name)
+        try:
+            return fn(*args, **kwargs)
+        finally:
+            torch.cuda.nvtx.range_pop()
+    return wrapped
 
 
 def _p(t: Optional[torch.Tensor]) -> ctypes.c_void_p:
@@ -77,6 +100,7 @@ def _need(t: torch.Tensor, name: str, dtype: torch.dtype, ndim: int, device=None
 # Graph-based context denoising
 # ----------------------------------------------------------------------------
 
+@_ranged
 def denoise(emb: torch.Tensor, *, n_tokens: Optional[torch.Tensor] = None, g: int = 3,
             tau: float = 0.05, keep_every: int = 16,
             workspace: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, torch.Tensor]:
@@ -107,6 +131,7 @@ def denoise(emb: torch.Tensor, *, n_tokens: Optional[torch.Tensor] = None, g: in
 # MemoryBridge output
 # ----------------------------------------------------------------------------
 
+@_ranged
 def bridge_epilogue(x: torch.Tensor, nu: float, *, gamma: Optional[torch.Tensor] = None,
                     beta: Optional[torch.Tensor] = None, eps: float = 1e-5,
                     out: Optional[torch.Tensor] = None) -> torch.Tensor:
@@ -154,6 +179,7 @@ def _counter_workspace(kind: str, nbytes: int, device: torch.device) -> torch.Te
     return ws
 
 
+@_ranged
 def score_select(question_emb: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
                  idx_out: Optional[torch.Tensor] = None,
                  scores_out: Optional[torch.Tensor] = None,
@@ -185,6 +211,7 @@ def score_select(question_emb: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
     return idx_out
 
 
+@_ranged
 def question_select(question_tokens: torch.Tensor, cme_bank: torch.Tensor, k: int, *,
                     q_len: Optional[torch.Tensor] = None,
                     chunk_offset: Optional[torch.Tensor] = None,
@@ -321,6 +348,7 @@ def _scale(scale: Optional[float]) -> float:
     return 0.0 if scale is None else float(scale)
 
 
+@_ranged
 def two_tier_decode_attn(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, *,
                          scale: Optional[float] = None, out: Optional[torch.Tensor] = None,
                          workspace: Optional[DecodeWorkspace] = None) -> torch.Tensor:
@@ -335,6 +363,7 @@ def two_tier_decode_attn(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, *,
     return out
 
 
+@_ranged
 def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, *,
                 scale: Optional[float] = None, out: Optional[torch.Tensor] = None,
                 workspace: Optional[DecodeWorkspace] = None,
@@ -367,6 +396,7 @@ def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, *,
     return out
 
 
+@_ranged
 def tier1_gather(bank_k: torch.Tensor, bank_v: torch.Tensor, idx: torch.Tensor, *,
                  out_k: Optional[torch.Tensor] = None, out_v: Optional[torch.Tensor] = None,
                  workspace: Optional[DecodeWorkspace] = None
@@ -401,6 +431,7 @@ def tier1_gather(bank_k: torch.Tensor, bank_v: torch.Tensor, idx: torch.Tensor, 
     return out_k, out_v
 
 
+@_ranged
 def window_append(ring_k: torch.Tensor, ring_v: torch.Tensor, pos: torch.Tensor,
                   k_new: torch.Tensor, v_new: torch.Tensor) -> None:
     """Append one token per sequence to the Tier-2 ring; see cmc_window_append."""
@@ -427,6 +458,7 @@ def window_append(ring_k: torch.Tensor, ring_v: torch.Tensor, pos: torch.Tensor,
 # Staging copies (host <-> device traffic of a decode loop)
 # ----------------------------------------------------------------------------
 
+@_ranged
 def stage_copies(pairs, *, wait_first: bool = False, device: Optional[torch.device] = None) -> None:
     """Copy each (src, dst) tensor pair, byte for byte, in one kernel launch on
     the current stream; see cmc_stage_copies.  Host tensors must be pinned
