@@ -654,7 +654,7 @@ def run_gpu(args, w, world, rank, local):
     def copies_for(nbytes):
         return max(2, min(16, -(-2 * 129_000_000 // max(nbytes, 1))))
 
-    prologue_us = bridge_us = denoise_us = select_cold_us = None
+    prologue_us = bridge_us = denoise_us = select_cold_us = batched = None
     prologue_cold_us = bridge_cold_us = None
     denoise_bytes = 0
     if not args.no_variant:
@@ -709,6 +709,56 @@ def run_gpu(args, w, world, rank, local):
         denoise_us = stream_us([(lambda i=i: cmc.denoise(embs[i], workspace=ws_ds[i]))
                                 for i in range(nd)])
         del emb, embs
+        if w.B == 1:
+            # the same calls with the inputs of RB requests in each (B = RB), as
+            # a server that batches arriving requests would issue them; per
+            # request = per call / RB, back to back on distinct inputs
+            RB = 4
+            wb = w.with_(B=RB)
+            sib = selection_inputs(wb)
+            qb = torch.from_numpy(sib.question_emb).to(dev)
+            bb = torch.from_numpy(sib.cme_bank).to(dev)
+            nb = copies_for(bb.numel() * 4)
+            bbs = [bb] + [bb.clone() for _ in range(nb - 1)]
+            wsb = [torch.zeros(cmc.score_select_workspace_size(RB, w.N), dtype=torch.uint8,
+                               device=dev) for _ in range(nb)]
+            sel_b = stream_us([(lambda i=i: cmc.score_select(qb, bbs[i], w.k, workspace=wsb[i]))
+                               for i in range(nb)]) / RB
+            qib = question_inputs(wb, sib, ratio=ratio)
+            tkb = torch.from_numpy(qib.tokens).to(dev)
+            tkbs = [tkb] + [tkb.clone() for _ in range(nb - 1)]
+            qlb = torch.from_numpy(qib.q_len).to(dev)
+            ofb = torch.from_numpy(qib.chunk_offset).to(dev)
+            clb = torch.from_numpy(qib.ctx_len).to(dev)
+            wqb = [torch.zeros(cmc.lib().cmc_question_select_workspace_size(RB, w.N),
+                               dtype=torch.uint8, device=dev) for _ in range(nb)]
+            pro_b = stream_us([(lambda i=i: cmc.question_select(
+                tkbs[i], bbs[i], w.k, q_len=qlb, chunk_offset=ofb, ctx_len=clb, W=w.W,
+                workspace=wqb[i])) for i in range(nb)]) / RB
+            outs = [torch.empty_like(bb) for _ in range(nb)]
+            br_b = stream_us([(lambda i=i: cmc.bridge_epilogue(bbs[i], 0.8, out=outs[i]))
+                              for i in range(nb)]) / RB
+            del outs, bbs, tkbs
+            cib = context_inputs(wb, H=1280, ratio=ratio)
+            eb = torch.from_numpy(cib.emb).to(dev)
+            ntb = torch.from_numpy(cib.n_tokens).to(dev)
+            tok_bytes = int(cib.n_tokens.sum()) * cib.emb.shape[2] * 4
+            ndb = copies_for(eb.numel() * 4)
+            ebs = [eb] + [eb.clone() for _ in range(ndb - 1)]
+            wsd = [torch.zeros(cmc.lib().cmc_denoise_workspace_size(RB, eb.shape[1]),
+                               dtype=torch.uint8, device=dev) for _ in range(ndb)]
+            dn_b = stream_us([(lambda i=i: cmc.denoise(ebs[i], n_tokens=ntb, workspace=wsd[i]))
+                              for i in range(ndb)]) / RB
+            del ebs
+            bank_bytes = 4 * w.N * w.D
+            batched = {
+                "requests_per_call": RB,
+                "note": "per request, calls of RB requests back to back on distinct inputs",
+                "select_us": sel_b, "select_gbs": bank_bytes / (sel_b * 1e-6) / 1e9,
+                "question_prologue_us": pro_b,
+                "bridge_epilogue_us": br_b, "bridge_epilogue_gbs": 2 * bank_bytes / (br_b * 1e-6) / 1e9,
+                "denoise_us": dn_b, "denoise_gbs": tok_bytes / RB / (dn_b * 1e-6) / 1e9,
+                "denoise_tokens": [int(x) for x in cib.n_tokens]}
     del flush
 
     # e2e through the Python API with pinned host buffers
@@ -756,6 +806,7 @@ def run_gpu(args, w, world, rank, local):
         "tier1_gather_us": gather_us,
         "tier1_gather_gbs": (tier1_gather_bytes(w.B, w.L, w.Hkv, w.d, w.k) / (gather_us * 1e-6)
                              / 1e9 if gather_us > 0 else None),
+        "batched_requests": batched,
         "variant": variant,
         "rope_variant": rope_variant,
         "warm_l2": warm_l2,
