@@ -676,3 +676,41 @@ def test_rope_stream_k_and_combine(cuda_device, mode):
     np.testing.assert_array_equal(host_bits(P.ring_v), P.o_ring_v)
     _ring_close_bf16(host_bits(P.ring_k), P.o_ring_k, "stream-K rotated keys")
     assert P.ws.status() == 0
+
+
+def test_rope_frequency_table_in_device_memory_or_parameters(cuda_device):
+    """The rotary frequencies come from a device table written on a theta's
+    first use outside graph capture, or from the kernel parameters when that
+    first use is being captured: both give bit-identical steps."""
+    w = WORKLOADS["tiny"].with_(B=2, T=1)
+    theta = 23456.789  # used by no other test
+    A = Problem(w, cuda_device, mode="dense")
+    Bp = Problem(w, cuda_device, mode="dense")
+    st = step_inputs(w, 0)
+    q, kn, vn = (dev_bf16(x, cuda_device) for x in (st.q, st.k_new, st.v_new))
+    out_a = torch.empty_like(q)
+    stream = torch.cuda.Stream(device=cuda_device)
+    stream.wait_stream(torch.cuda.current_stream(cuda_device))
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        cmc.decode_step(q, A.t1k, A.t1v, A.idx, A.ring_k, A.ring_v, A.pos, kn, vn, out=out_a,
+                        workspace=A.ws, rope_theta=theta, rope_offset=w.k)
+    g.replay()
+    torch.cuda.synchronize()
+    out_b = cmc.decode_step(q, Bp.t1k, Bp.t1v, Bp.idx, Bp.ring_k, Bp.ring_v, Bp.pos, kn, vn,
+                            workspace=Bp.ws, rope_theta=theta, rope_offset=w.k)
+    torch.cuda.synchronize()
+    assert torch.equal(out_a.view(torch.int16), out_b.view(torch.int16))
+    assert torch.equal(A.ring_k, Bp.ring_k) and torch.equal(A.pos, Bp.pos)
+    ref = oracle.decode_step_rope(st.q, A.kv.tier1_k, A.kv.tier1_v, A.idx_host, A.o_ring_k,
+                                  A.o_ring_v, A.o_pos, st.k_new, st.v_new, theta=theta,
+                                  rope_offset=w.k)
+    assert_attn_close(to_f64(out_b), ref, "rope table paths")
+
+
+def test_rope_many_thetas(cuda_device):
+    """More distinct thetas than device table slots: the later ones use the
+    kernel parameters; every step matches the oracle."""
+    w = WORKLOADS["tiny"].with_(B=1, T=1)
+    for j in range(20):
+        _rope_run(w, cuda_device, "dense", theta=1000.0 + 97.5 * j, offset=w.k)
