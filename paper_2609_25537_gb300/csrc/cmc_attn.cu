@@ -958,24 +958,31 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     if (u != cur_u) {  // first tile of a unit in this CTA
       cur_u = u;
       const uint8_t* qs = aux + S::kQ;
+      if (ROPE && gq < G && !dead) {
+        // rotate the query: column c of the first half pairs with c + d/2,
+        // and k-step ks + KS/2 holds exactly those partners, so each pair of
+        // columns is read once and gives both rotated values
+        const float2* tab = reinterpret_cast<const float2*>(aux + S::kRope);
+#pragma unroll
+        for (int ks = 0; ks < KS / 2; ++ks) {
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {
+            const int c = 16 * ks + 2 * tq + 8 * hf;  // < d/2
+            const uint32_t xv = *reinterpret_cast<const uint32_t*>(qs + (gq * D + c) * 2);
+            const uint32_t pv = *reinterpret_cast<const uint32_t*>(qs + (gq * D + c + D / 2) * 2);
+            const float2 t0 = tab[c], t1 = tab[c + 1];
+            const float xl = bf16lo_to_f32(xv), xh = bf16hi_to_f32(xv);
+            const float pl = bf16lo_to_f32(pv), ph = bf16hi_to_f32(pv);
+            qa[ks][hf] = pack_bf16_rn(fmaf(xl, t0.x, -1.f * pl * t0.y), fmaf(xh, t1.x, -1.f * ph * t1.y));
+            qa[ks + KS / 2][hf] = pack_bf16_rn(fmaf(pl, t0.x, 1.f * xl * t0.y), fmaf(ph, t1.x, 1.f * xh * t1.y));
+          }
+        }
+      }
 #pragma unroll
       for (int ks = 0; ks < KS; ++ks) {
         if (gq < G && !dead) {
           if (ROPE) {
-            // rotate the query: column c pairs with c ^ d/2 (the other half)
-            const float2* tab = reinterpret_cast<const float2*>(aux + S::kRope);
-#pragma unroll
-            for (int hf = 0; hf < 2; ++hf) {
-              const int c = 16 * ks + 2 * tq + 8 * hf;
-              const uint32_t xv = *reinterpret_cast<const uint32_t*>(qs + (gq * D + c) * 2);
-              const uint32_t pv = *reinterpret_cast<const uint32_t*>(qs + (gq * D + (c ^ (D / 2))) * 2);
-              const int i = c & (D / 2 - 1);
-              const float sg = (c < D / 2) ? -1.f : 1.f;
-              const float2 t0 = tab[i], t1 = tab[i + 1];
-              const float lo = fmaf(bf16lo_to_f32(xv), t0.x, sg * bf16lo_to_f32(pv) * t0.y);
-              const float hi = fmaf(bf16hi_to_f32(xv), t1.x, sg * bf16hi_to_f32(pv) * t1.y);
-              qa[ks][hf] = pack_bf16_rn(lo, hi);
-            }
+            // rotated above
           } else {
             qa[ks][0] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq) * 2);
             qa[ks][1] = *reinterpret_cast<const uint32_t*>(qs + gq * D * 2 + (16 * ks + 2 * tq + 8) * 2);
