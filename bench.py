@@ -11,7 +11,10 @@ scoring + top-k selection on its own CME bank and compacts the selected K/V
 rows into its dense Tier-1 cache (cmc_tier1_gather: the cache the paper's
 prefill of the selected CMEs leaves), then the R requests run their 3,000
 fused decode steps (ring append + two-tier attention over all 32 layers, one
-launch per request per step) round-robin.  `--tier1 gather` instead passes the
+launch per request per step) round-robin, request r's launches on stream
+r % S (S = --streams, default 2: a server runs independent requests
+concurrently; each request's steps stay in order on its stream, so a launch
+of one stream overlaps the completion of the other's).  `--tier1 gather` instead passes the
 bank and idx to every decode step (the gather inside the attention kernel).  Each request's KV
 state (84.5 MB read per step) fits in the 129 MB L2 by itself; interleaving R
 requests puts (R-1) x 84.5 MB of other traffic between two steps of the same
@@ -38,7 +41,8 @@ Reported (one JSON line on rank 0):
   e2e            the same metric through the Python API with host buffers
                  (question vector, CME bank and every step's q / new K,V
                  copied in from pinned memory, every step's output copied out,
-                 by one staging-copy launch per round of R decode steps);
+                 by one staging-copy launch per R decode launches on each
+                 stream);
   cpu_baseline   the fp64 oracle on the host, on a bounded sample.
 
 `--impl reference` times the fp64 oracle alone on the host cores (the
@@ -461,6 +465,11 @@ def run_gpu(args, w, world, rank, local):
     # the oracle's copy of request 0, taken before any kernel of ours touches it
     cpu_state = reqs[0].host_state() if want_cpu else None
     stream = torch.cuda.Stream(device=dev)
+    # the decode launches of the R independent requests go to S streams
+    # (request r to stream r % S), as a server runs independent requests
+    # concurrently; every request's steps stay in order on its stream
+    S = max(1, min(args.streams, R))
+    streams = [stream] + [torch.cuda.Stream(device=dev) for _ in range(S - 1)]
 
     mode = args.tier1
     other = "gather" if mode == "dense" else "dense"
@@ -474,13 +483,19 @@ def run_gpu(args, w, world, rank, local):
             r.decode(0, mode=mode, rope=True)
     stream.synchronize()
 
-    # one graph = P rounds of R decode launches; replayed T / P times per step
+    # one graph = P rounds of R decode launches (forked over the S streams and
+    # joined again at its end); replayed T / P times per step
     def capture(m, rope=False):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
+            for st in streams[1:]:
+                st.wait_stream(stream)
             for p in range(P):
-                for r in reqs:
-                    r.decode(p, mode=m, rope=rope)
+                for ri, r in enumerate(reqs):
+                    with torch.cuda.stream(streams[ri % S]):
+                        r.decode(p, mode=m, rope=rope)
+            for st in streams[1:]:
+                stream.wait_stream(st)
         return g
     graph = capture(mode)
     replays = T // P
@@ -762,7 +777,7 @@ def run_gpu(args, w, world, rank, local):
     del flush
 
     # e2e through the Python API with pinned host buffers
-    e2e = run_e2e(args, w, reqs, dev, stream, world) if not args.no_e2e else None
+    e2e = run_e2e(args, w, reqs, dev, stream, world, streams) if not args.no_e2e else None
 
     # CPU oracle baseline (rank 0, N = 1)
     cpu = None
@@ -790,6 +805,7 @@ def run_gpu(args, w, world, rank, local):
         "dtype": "bf16", "data": "synthetic",
         "config": dict(workload_config(w, R), tier1=mode),
         "tier1": mode,
+        "decode_streams": S,
         "decode_us_per_launch": launch_us,
         "hbm_pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
         "select_us": select_us,
@@ -828,63 +844,101 @@ def run_gpu(args, w, world, rank, local):
     return 0
 
 
-def run_e2e(args, w, reqs, dev, stream, world):
+def run_e2e(args, w, reqs, dev, stream, world, streams):
     """Same metric through the public Python API with host buffers: the
     question vector and CME bank of each request and, every decode step, q and
     the new token's K,V are copied in from pinned host memory and the output
-    copied back to pinned host memory.  As a serving loop would, each
-    scheduling round (one decode step of each of the R requests) moves its
-    inputs in together, and a round's outputs go out together: one staging-copy
-    launch per round (cmc.stage_copies) on the decode stream carries the
-    inputs of this round and the outputs of the round two back.  It copies
-    without waiting for the decode before it (inputs double-buffered, outputs
-    triple-buffered, so that decode never touches what it copies) and
-    completes after it, so every decode launch keeps programmatic dependent
-    launch and the copies overlap decode work.  12 rounds (6 when T is not a
-    multiple of 12) are captured in one CUDA graph; the buffers rotate across
-    replays, so a replay's first two copy launches carry the previous
-    replay's last two rounds' outputs, and one copy launch after the step's
-    last replay the step's last two.  Selection and compaction run
-    eagerly."""
+    copied back to pinned host memory.  The requests are split over the same
+    streams as the device-resident loop (request r on stream r % S), each
+    stream a serving loop of its own: every scheduling round (one decode step
+    of each of its requests) moves their inputs in together, and a round's
+    outputs go out together -- one staging-copy launch per round
+    (cmc.stage_copies) on that stream carries the inputs of this round and the
+    outputs of the round two back.  It copies without waiting for the decode
+    before it (inputs double-buffered, outputs triple-buffered, so that decode
+    never touches what it copies) and completes after it, so every decode
+    launch keeps programmatic dependent launch and the copies overlap decode
+    work.  12 rounds (6 when T is not a multiple of 12) are captured in one
+    CUDA graph; the buffers rotate across replays, so a replay's first two
+    copy launches carry the previous replay's last two rounds' outputs, and
+    one copy launch after the step's last replay the step's last two.
+    Selection and compaction run eagerly."""
     import paper_2609_25537_gb300 as cmc
     R, T, P0 = args.requests, args.decode_steps, args.pool
-    # rounds per graph: a multiple of 6 when T allows, so that the double-
-    # buffered inputs and triple-buffered outputs continue across replays and
-    # only the step's last two rounds need a copy after the last replay
-    P = 12 if T % 12 == 0 else (6 if T % 6 == 0 else P0)
-    rotate = P % 6 == 0
+    S = len(streams)
+    groups = [[i for i in range(R) if i % S == j] for j in range(S)]
+    # a stream's staging copy carries `spr` rounds of its requests, so that
+    # every copy launch still serves R decode launches
+    spr = max(1, R // max(len(g) for g in groups)) * max(1, args.e2e_copy_rounds)
+    # rounds per graph: a multiple of 6 super-rounds of spr rounds when T
+    # allows, so that the double-buffered inputs and triple-buffered outputs
+    # continue across replays and only the step's last two need a copy after
+    # the last replay
+    P = next((c for c in (12 * spr, 6 * spr, 2 * spr) if T % c == 0), None)
+    if P is None:  # one round per copy
+        spr = 1
+        P = next(c for c in (12, 6, P0, 2, T) if T % c == 0)
+    Q = P // spr  # super-rounds per graph (>= 2 unless T = 1)
+    rotate = Q % 6 == 0
     steps = max(1, min(args.steps, args.e2e_steps))
     nq, nk = reqs[0].q[0].numel(), reqs[0].k_new[0].numel()
     per_req = nq + 2 * nk
-    # host: round p holds the R requests' packed (q, k_new, v_new) of step p
-    # (the pool's P0 inputs, cycled)
-    host_in = torch.cat([torch.cat([r.q.reshape(P0, -1), r.k_new.reshape(P0, -1),
-                                    r.v_new.reshape(P0, -1)], dim=1) for r in reqs],
-                        dim=1)[[p % P0 for p in range(P)]].cpu().contiguous().pin_memory()  # [P, R*per_req]
     out_shape = tuple(reqs[0].out.shape)
-    host_out = torch.empty((P, R) + out_shape, dtype=torch.bfloat16).pin_memory()
+    # per stream: host round p holds its requests' packed (q, k_new, v_new) of
+    # step p (the pool's P0 inputs, cycled); device buffers of one super-round
+    host_in, host_out, in_d, out_d = [], [], [], []
+    for grp in groups:
+        host_in.append(torch.cat([torch.cat([reqs[i].q.reshape(P0, -1), reqs[i].k_new.reshape(P0, -1),
+                                             reqs[i].v_new.reshape(P0, -1)], dim=1) for i in grp],
+                                 dim=1)[[p % P0 for p in range(P)]].cpu().contiguous().pin_memory())
+        host_out.append(torch.empty((P, len(grp)) + out_shape, dtype=torch.bfloat16).pin_memory())
+        in_d.append([torch.empty(spr * len(grp) * per_req, dtype=torch.bfloat16, device=dev)
+                     for _ in range(2)])
+        out_d.append([torch.empty((spr, len(grp)) + out_shape, dtype=torch.bfloat16, device=dev)
+                      for _ in range(3)])
     host_sel = [(r.qemb.cpu().pin_memory(), r.bank.cpu().pin_memory()) for r in reqs]
-    in_d = [torch.empty(R * per_req, dtype=torch.bfloat16, device=dev) for _ in range(2)]
-    out_d = [torch.empty((R,) + out_shape, dtype=torch.bfloat16, device=dev) for _ in range(3)]
 
-    def views(par, i):
-        base = in_d[par][i * per_req:(i + 1) * per_req]
+    def views(gi, par, j, k):
+        i = groups[gi][k]
+        base = in_d[gi][par][(j * len(groups[gi]) + k) * per_req:(j * len(groups[gi]) + k + 1) * per_req]
         return (base[:nq].view(reqs[i].q[0].shape), base[nq:nq + nk].view(reqs[i].k_new[0].shape),
                 base[nq + nk:].view(reqs[i].v_new[0].shape))
 
-    def last_two():  # the outputs of the last two rounds, after every decode
-        cmc.stage_copies([(out_d[(P - 2) % 3], host_out[P - 2]),
-                          (out_d[(P - 1) % 3], host_out[P - 1])], wait_first=True, device=dev)
+    def fork():
+        for st in streams[1:]:
+            st.wait_stream(stream)
+
+    def join():
+        for st in streams[1:]:
+            stream.wait_stream(st)
+
+    def rows(sr):  # host rows of super-round sr
+        return slice(sr * spr, (sr + 1) * spr)
+
+    def last_two():  # the outputs of the last two super-rounds, after every decode
+        fork()
+        for gi in range(S):
+            with torch.cuda.stream(streams[gi]):
+                cmc.stage_copies([(out_d[gi][(Q - 2) % 3], host_out[gi][rows(Q - 2)]),
+                                  (out_d[gi][(Q - 1) % 3], host_out[gi][rows(Q - 1)])],
+                                 wait_first=True, device=dev)
+        join()
 
     def rounds():
-        for p in range(P):
-            pairs = [(host_in[p], in_d[p % 2])]
-            if p >= 2 or rotate:  # rounds 0, 1: the previous replay's last two
-                pairs.append((out_d[(p - 2) % 3], host_out[(p - 2) % P]))
-            cmc.stage_copies(pairs, device=dev)
-            for i, r in enumerate(reqs):
-                q, k, v = views(p % 2, i)
-                r.decode(p % P0, q=q, k_new=k, v_new=v, mode=args.tier1, out=out_d[p % 3][i])
+        fork()
+        for sr in range(Q):
+            for gi, grp in enumerate(groups):
+                with torch.cuda.stream(streams[gi]):
+                    pairs = [(host_in[gi][rows(sr)], in_d[gi][sr % 2])]
+                    if sr >= 2 or rotate:  # super-rounds 0, 1: the previous replay's last two
+                        pairs.append((out_d[gi][(sr - 2) % 3], host_out[gi][rows((sr - 2) % Q)]))
+                    cmc.stage_copies(pairs, device=dev)
+                    for j in range(spr):
+                        for k, i in enumerate(grp):
+                            q, kn, vn = views(gi, sr % 2, j, k)
+                            reqs[i].decode((sr * spr + j) % P0, q=q, k_new=kn, v_new=vn,
+                                           mode=args.tier1, out=out_d[gi][sr % 3][j, k])
+        join()
         if not rotate:
             last_two()
 
@@ -926,9 +980,10 @@ def run_e2e(args, w, reqs, dev, stream, world):
     d2h = R * T * reqs[0].out.numel() * 2
     return {"value": world * steps * R * w.B * T / el, "unit": "tokens/s",
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": steps,
-            "per_step_graph": graph is not None,
-            "copies": ("per round of R decode steps, one staging-copy launch on the decode "
-                       "stream: this round's inputs in, the outputs of the round two back out")}
+            "per_step_graph": graph is not None, "streams": S,
+            "copies": ("per round of decode steps of each stream's requests, one staging-copy "
+                       "launch on that stream: this round's inputs in, the outputs of the "
+                       "round two back out")}
 
 
 def run_ablation(args, dev):
@@ -1025,7 +1080,11 @@ def main(argv=None):
     ap.add_argument("--requests", type=int, default=4)
     ap.add_argument("--decode-steps", type=int, default=None)
     ap.add_argument("--pool", type=int, default=8)
+    ap.add_argument("--streams", type=int, default=2,
+                    help="streams the independent requests' decode launches are spread over")
     ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--e2e-copy-rounds", type=int, default=1,
+                    help="rounds of R decode steps each staging copy of the e2e loop carries")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--tier1", choices=("dense", "gather"), default="dense",
