@@ -12,9 +12,9 @@ rows into its dense Tier-1 cache (cmc_tier1_gather: the cache the paper's
 prefill of the selected CMEs leaves), then the R requests run their 3,000
 fused decode steps (ring append + two-tier attention over all 32 layers, one
 launch per request per step) round-robin, request r's launches on stream
-r % S (S = --streams, default 2: a server runs independent requests
+r % S (S = --streams, default 3: a server runs independent requests
 concurrently; each request's steps stay in order on its stream, so a launch
-of one stream overlaps the completion of the other's).  `--tier1 gather` instead passes the
+of one stream overlaps the completion of another's).  `--tier1 gather` instead passes the
 bank and idx to every decode step (the gather inside the attention kernel).  Each request's KV
 state (84.5 MB read per step) fits in the 129 MB L2 by itself; interleaving R
 requests puts (R-1) x 84.5 MB of other traffic between two steps of the same
@@ -1080,7 +1080,7 @@ def main(argv=None):
     ap.add_argument("--requests", type=int, default=4)
     ap.add_argument("--decode-steps", type=int, default=None)
     ap.add_argument("--pool", type=int, default=8)
-    ap.add_argument("--streams", type=int, default=2,
+    ap.add_argument("--streams", type=int, default=3,
                     help="streams the independent requests' decode launches are spread over")
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--e2e-copy-rounds", type=int, default=1,
