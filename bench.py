@@ -12,7 +12,7 @@ rows into its dense Tier-1 cache (cmc_tier1_gather: the cache the paper's
 prefill of the selected CMEs leaves), then the R requests run their 3,000
 fused decode steps (ring append + two-tier attention over all 32 layers, one
 launch per request per step) round-robin, request r's launches on stream
-r % S (S = --streams, default 3: a server runs independent requests
+r % S (S = --streams, default 4: a server runs independent requests
 concurrently; each request's steps stay in order on its stream, so a launch
 of one stream overlaps the completion of another's).  `--tier1 gather` instead passes the
 bank and idx to every decode step (the gather inside the attention kernel).  Each request's KV
@@ -867,9 +867,10 @@ def run_e2e(args, w, reqs, dev, stream, world, streams):
     R, T, P0 = args.requests, args.decode_steps, args.pool
     S = len(streams)
     groups = [[i for i in range(R) if i % S == j] for j in range(S)]
-    # a stream's staging copy carries `spr` rounds of its requests, so that
-    # every copy launch still serves R decode launches
-    spr = max(1, R // max(len(g) for g in groups)) * max(1, args.e2e_copy_rounds)
+    # a stream's staging copy carries `spr` rounds of its requests (one by
+    # default: with one request a stream, one copy launch per decode launch
+    # measured faster than one per two or four)
+    spr = max(1, args.e2e_copy_rounds)
     # rounds per graph: a multiple of 6 super-rounds of spr rounds when T
     # allows, so that the double-buffered inputs and triple-buffered outputs
     # continue across replays and only the step's last two need a copy after
@@ -1080,11 +1081,12 @@ def main(argv=None):
     ap.add_argument("--requests", type=int, default=4)
     ap.add_argument("--decode-steps", type=int, default=None)
     ap.add_argument("--pool", type=int, default=8)
-    ap.add_argument("--streams", type=int, default=3,
+    ap.add_argument("--streams", type=int, default=4,
                     help="streams the independent requests' decode launches are spread over")
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--e2e-copy-rounds", type=int, default=1,
-                    help="rounds of R decode steps each staging copy of the e2e loop carries")
+                    help="rounds (one decode step of each of a stream's requests) that each "
+                         "staging copy of the e2e loop carries")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--tier1", choices=("dense", "gather"), default="dense",
