@@ -637,15 +637,17 @@ __device__ __forceinline__ void hist_level(uint32_t ha, uint32_t bin_a, uint32_t
 // position).  Every thread of the CTA calls it.
 //
 // The k-th largest key T is found in three histogram levels: its top 11 bits
-// from the histogram the scoring CTAs built in `ghist` (read, then zeroed for
-// the next call), bits 20..10 from a shared-memory histogram of the keys with
-// those top bits, bits 9..0 likewise; each level is one prefix sum over the
-// bins (two a thread) -- eight barriers in all, against 32 counting barriers
-// for a bit-by-bit search.  The ordered compaction then writes the keys > T
-// and the lowest-index keys == T.
+// from the histogram the scoring CTAs built in `ghist` (thread t's two bins
+// 2047 - 2t and 2046 - 2t read by the caller with the keys, as ga and gb;
+// zeroed here for the next call), bits 20..10 from a shared-memory histogram
+// of the keys with those top bits, bits 9..0 likewise; each level is one
+// prefix sum over the bins (two a thread) -- eight barriers in all, against
+// 32 counting barriers for a bit-by-bit search.  The ordered compaction then
+// writes the keys > T and the lowest-index keys == T, its output slots from
+// one prefix sum of both counts packed in a word.
 template <int KPT>
 __device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int N, int k, int32_t* out,
-                                           uint32_t* ghist, uint32_t* scan_eq,
+                                           uint32_t* ghist, uint32_t ga, uint32_t gb,
                                            uint32_t* scan_sel) {
   __shared__ uint32_t h2[kHistTop], h3[kHistTop / 2], pick[2];
   const int tid = threadIdx.x;
@@ -655,7 +657,6 @@ __device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int N, in
   h3[tid] = 0u;
   // level 1 (bits 31..21): thread t takes bins 2047 - 2t and 2046 - 2t
   const uint32_t ba = kHistTop - 1 - 2 * tid, bb = ba - 1;
-  const uint32_t ga = __ldcg(ghist + ba), gb = __ldcg(ghist + bb);
   ghist[ba] = 0u;
   ghist[bb] = 0u;
   uint32_t rem = static_cast<uint32_t>(k), d;
@@ -683,9 +684,12 @@ __device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int N, in
     n_gt += key[e] > T ? 1u : 0u;
     n_eq += key[e] == T ? 1u : 0u;
   }
-  const uint32_t eq_before = fused_scan(n_eq, scan_eq);
-  const uint32_t take = need > eq_before ? min(need - eq_before, n_eq) : 0u;
-  uint32_t slot = fused_scan(n_gt + take, scan_sel);
+  // the keys > T and == T before this thread's, from one prefix sum: both
+  // counts total at most N <= 2048 < 2^16, so the low half never carries
+  const uint32_t before = fused_scan(n_gt | (n_eq << 16), scan_sel);
+  const uint32_t eq_before = before >> 16;
+  // the keys > T before this thread's, and the first `need` keys == T
+  uint32_t slot = (before & 0xFFFFu) + min(eq_before, need);
   uint32_t r = eq_before;
 #pragma unroll
   for (int e = 0; e < KPT; ++e) {
@@ -703,16 +707,23 @@ __device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int N, in
 // its result is written at the end.
 template <int KPT>
 __device__ __forceinline__ void fused_select_impl(const FusedArgs& a, int b) {
-  __shared__ uint32_t scan_eq[kFusedWarps], scan_sel[kFusedWarps];
+  __shared__ uint32_t scan_sel[kFusedWarps];
   const int tid = threadIdx.x;
   const int N = a.N, k = a.k;
   const bool topk = k > 0 && k < N;
   const float* sc = a.scores + static_cast<long long>(b) * N;
+  uint32_t* ghist = a.hist + static_cast<long long>(b) * kHistTop;
   uint32_t key[KPT];
 #pragma unroll
   for (int e = 0; e < KPT; ++e) {
     const int j = tid * KPT + e;
     key[e] = (topk && j < N) ? orderable(__ldcg(sc + j)) : 0u;
+  }
+  // this thread's two bins of the top-bits histogram, in flight with the keys
+  uint32_t ga = 0u, gb = 0u;
+  if (topk) {
+    ga = __ldcg(ghist + (kHistTop - 1 - 2 * tid));
+    gb = __ldcg(ghist + (kHistTop - 2 - 2 * tid));
   }
   const bool locate = a.la.sqnorm && tid == 0;
   int32_t alpha = 0, clen = 0;
@@ -727,7 +738,7 @@ __device__ __forceinline__ void fused_select_impl(const FusedArgs& a, int b) {
   if (k >= N) {
     for (int j = tid; j < N; j += kFusedThreads) out[j] = j;
   } else if (k > 0) {
-    fused_topk<KPT>(key, N, k, out, a.hist + static_cast<long long>(b) * kHistTop, scan_eq, scan_sel);
+    fused_topk<KPT>(key, N, k, out, ghist, ga, gb, scan_sel);
   }
   if (locate) {
     long long st = static_cast<long long>(clen) - a.la.W;
