@@ -150,7 +150,10 @@ bridge_epilogue_kernel(const float* x, const float* __restrict__ gamma,
 // a bank of up to 8 x SMs rows is one wave whose loads are all issued at
 // once (more rows: grid-stride).  No shared-memory staging; each of the
 // three reductions takes one barrier (its own partials array, summed by every
-// thread in the same order).
+// thread in the same order).  Before the grid dependency wait a CTA asks L2
+// to prefetch its first row, so that under programmatic dependent launch the
+// row streams in while the kernel before drains (a prefetch is a hint: L2
+// stays coherent with that kernel's writes to x).
 constexpr int kBridgeRegThreads = 128;
 constexpr int kBridgeRegMaxV = 8;  // float4s per thread: D <= 4 * 8 * kBridgeRegThreads
 constexpr int kBridgeRegCtasPerSm = 8;
@@ -162,6 +165,13 @@ bridge_epilogue_reg_kernel(const float* x, const float* __restrict__ gamma,
                            float nu, float* out) {
   constexpr int NW = kBridgeRegThreads / 32;
   __shared__ float red[3][NW];
+  if (threadIdx.x == 0 && static_cast<long long>(blockIdx.x) < rows)
+    // D * 4 bytes of a 16-byte aligned row (D a multiple of 4): the bulk
+    // prefetch's alignment and size rules hold
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;\n" ::"l"(
+                     x + static_cast<long long>(blockIdx.x) * D),
+                 "r"(static_cast<unsigned int>(D) * 4u)
+                 : "memory");
   pdl_wait();
   pdl_trigger();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
