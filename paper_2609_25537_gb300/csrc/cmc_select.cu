@@ -614,21 +614,24 @@ __device__ __forceinline__ uint32_t fused_scan(uint32_t v, uint32_t* ws) {
 // the counts of bins bin_a > bin_b (the bins in descending order across the
 // threads); an exclusive prefix sum over the block gives the keys in the bins
 // above, and the thread whose bins hold the rem-th key (counting from the
-// top) publishes the bin and the rank of that key within it.
+// top) publishes the bin, the rank of that key within it and the bin's count.
 __device__ __forceinline__ void hist_level(uint32_t ha, uint32_t bin_a, uint32_t hb, uint32_t bin_b,
-                                           uint32_t& rem, uint32_t& digit, uint32_t* ws,
-                                           uint32_t* pick) {
+                                           uint32_t& rem, uint32_t& digit, uint32_t& count,
+                                           uint32_t* ws, uint32_t* pick) {
   const uint32_t above = fused_scan(ha + hb, ws);
   if (above < rem && rem <= above + ha) {
     pick[0] = bin_a;
     pick[1] = rem - above;
+    pick[2] = ha;
   } else if (above + ha < rem && rem <= above + ha + hb) {
     pick[0] = bin_b;
     pick[1] = rem - above - ha;
+    pick[2] = hb;
   }
   __syncthreads();
   digit = pick[0];
   rem = pick[1];
+  count = pick[2];
 }
 
 // Top k of one sequence's N scores (N <= KPT * kFusedThreads), written to
@@ -636,20 +639,26 @@ __device__ __forceinline__ void hist_level(uint32_t ha, uint32_t bin_a, uint32_t
 // t*KPT .. t*KPT + KPT - 1 in registers (index order is thread order, then
 // position).  Every thread of the CTA calls it.
 //
-// The k-th largest key T is found in three histogram levels: its top 11 bits
-// from the histogram the scoring CTAs built in `ghist` (thread t's two bins
-// 2047 - 2t and 2046 - 2t read by the caller with the keys, as ga and gb;
-// zeroed here for the next call), bits 20..10 from a shared-memory histogram
-// of the keys with those top bits, bits 9..0 likewise; each level is one
-// prefix sum over the bins (two a thread) -- eight barriers in all, against
-// 32 counting barriers for a bit-by-bit search.  The ordered compaction then
-// writes the keys > T and the lowest-index keys == T, its output slots from
-// one prefix sum of both counts packed in a word.
+// The k-th largest key T is found in up to three histogram levels: its top
+// 11 bits from the histogram the scoring CTAs built in `ghist` (thread t's
+// two bins 2047 - 2t and 2046 - 2t read by the caller with the keys, as ga
+// and gb; zeroed here for the next call), bits 20..10 from a shared-memory
+// histogram of the keys with those top bits, bits 9..0 likewise; each level
+// is one prefix sum over the bins (two a thread) -- at most eight barriers,
+// against 32 counting barriers for a bit-by-bit search.  A level whose
+// chosen bin holds exactly the keys still to take ends the search: every
+// key of that bin is selected, so the compaction compares the keys' prefix
+// P = key >> s with the bin (s = 21 or 10) instead of the whole key with T,
+// and no tie is left to break.  (At the Llama shape the bins of the top 21
+// bits hold one key each almost always, so level 3 is rarely run.)  The
+// ordered compaction then writes the keys (prefixes) > P and the
+// lowest-index ones == P, its output slots from one prefix sum of both
+// counts packed in a word.
 template <int KPT>
 __device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int N, int k, int32_t* out,
                                            uint32_t* ghist, uint32_t ga, uint32_t gb,
                                            uint32_t* scan_sel) {
-  __shared__ uint32_t h2[kHistTop], h3[kHistTop / 2], pick[2];
+  __shared__ uint32_t h2[kHistTop], h3[kHistTop / 2], pick[3];
   const int tid = threadIdx.x;
   static_assert(kHistTop == 2 * kFusedThreads, "two top bins a thread");
   h2[2 * tid] = 0u;
@@ -659,41 +668,52 @@ __device__ __forceinline__ void fused_topk(const uint32_t (&key)[KPT], int N, in
   const uint32_t ba = kHistTop - 1 - 2 * tid, bb = ba - 1;
   ghist[ba] = 0u;
   ghist[bb] = 0u;
-  uint32_t rem = static_cast<uint32_t>(k), d;
-  hist_level(ga, ba, gb, bb, rem, d, scan_sel, pick);
-  uint32_t T = d << 21;
-  // level 2 (bits 20..10) among the keys with those top bits
+  uint32_t rem = static_cast<uint32_t>(k), d, cnt;
+  hist_level(ga, ba, gb, bb, rem, d, cnt, scan_sel, pick);
+  uint32_t P = d;  // the boundary keys' prefix key >> s
+  int s = 21;
+  if (cnt != rem) {  // rem and cnt came through shared memory: the branch is CTA-uniform
+    // level 2 (bits 20..10) among the keys with those top bits
 #pragma unroll
-  for (int e = 0; e < KPT; ++e)
-    if (tid * KPT + e < N && (key[e] >> 21) == (T >> 21)) atomicAdd(h2 + ((key[e] >> 10) & 2047u), 1u);
-  __syncthreads();
-  hist_level(h2[ba], ba, h2[bb], bb, rem, d, scan_sel, pick);
-  T |= d << 10;
-  // level 3 (bits 9..0): thread t takes bin 1023 - t
+    for (int e = 0; e < KPT; ++e)
+      if (tid * KPT + e < N && (key[e] >> 21) == P) atomicAdd(h2 + ((key[e] >> 10) & 2047u), 1u);
+    __syncthreads();
+    hist_level(h2[ba], ba, h2[bb], bb, rem, d, cnt, scan_sel, pick);
+    P = (P << 11) | d;
+    s = 10;
+    if (cnt != rem) {
+      // level 3 (bits 9..0): thread t takes bin 1023 - t
 #pragma unroll
-  for (int e = 0; e < KPT; ++e)
-    if (tid * KPT + e < N && (key[e] >> 10) == (T >> 10)) atomicAdd(h3 + (key[e] & 1023u), 1u);
-  __syncthreads();
-  const uint32_t bc = kHistTop / 2 - 1 - tid;
-  hist_level(h3[bc], bc, 0u, 0u, rem, d, scan_sel, pick);
-  T |= d;
-  const uint32_t need = rem;  // keys == T to keep, lowest index first (k - need keys are > T)
+      for (int e = 0; e < KPT; ++e)
+        if (tid * KPT + e < N && (key[e] >> 10) == P) atomicAdd(h3 + (key[e] & 1023u), 1u);
+      __syncthreads();
+      const uint32_t bc = kHistTop / 2 - 1 - tid;
+      hist_level(h3[bc], bc, 0u, 0u, rem, d, cnt, scan_sel, pick);
+      P = (P << 10) | d;  // T itself
+      s = 0;
+    }
+  }
+  // prefixes == P to keep, lowest index first (k - need keys have a larger
+  // prefix); with s > 0, need is the bin's whole count
+  const uint32_t need = rem;
   uint32_t n_gt = 0, n_eq = 0;
 #pragma unroll
   for (int e = 0; e < KPT; ++e) {
-    n_gt += key[e] > T ? 1u : 0u;
-    n_eq += key[e] == T ? 1u : 0u;
+    const uint32_t kp = key[e] >> s;
+    n_gt += kp > P ? 1u : 0u;
+    n_eq += kp == P ? 1u : 0u;
   }
-  // the keys > T and == T before this thread's, from one prefix sum: both
+  // the prefixes > P and == P before this thread's, from one prefix sum: both
   // counts total at most N <= 2048 < 2^16, so the low half never carries
   const uint32_t before = fused_scan(n_gt | (n_eq << 16), scan_sel);
   const uint32_t eq_before = before >> 16;
-  // the keys > T before this thread's, and the first `need` keys == T
+  // the keys > P before this thread's, and the first `need` keys == P
   uint32_t slot = (before & 0xFFFFu) + min(eq_before, need);
   uint32_t r = eq_before;
 #pragma unroll
   for (int e = 0; e < KPT; ++e) {
-    const bool sel = key[e] > T || (key[e] == T && r++ < need);
+    const uint32_t kp = key[e] >> s;
+    const bool sel = kp > P || (kp == P && r++ < need);
     if (sel && slot < static_cast<uint32_t>(k)) out[slot++] = tid * KPT + e;  // exactly k
   }
 }

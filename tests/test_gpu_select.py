@@ -164,6 +164,54 @@ def test_select_negative_and_signed_zero_scores(cuda_device):
     assert not np.signbit(scores[0, 3])
 
 
+def _bank_of_scores(s):
+    """Rows whose cosine with q = e_0 is s_j: m_j = (s_j, sqrt(1 - s_j^2), 0, ...)."""
+    N, D = len(s), 64
+    bank = np.zeros((1, N, D), dtype=np.float32)
+    bank[0, :, 0] = s
+    bank[0, :, 1] = np.sqrt(1.0 - np.asarray(s, dtype=np.float64) ** 2)
+    q = np.zeros((1, D), dtype=np.float32)
+    q[0, 0] = 1.0
+    return q, bank
+
+
+@pytest.mark.parametrize("case", ["level1_single", "level1_whole_bin", "level2", "level3_ties"])
+def test_select_search_levels(cuda_device, case):
+    """The one-launch selection's histogram search ends at the first level
+    whose chosen bin holds exactly the keys still to take; banks built so
+    that it ends at each level (top 11 key bits: the k-th score alone in
+    [0.5, 0.625), or that bin taken whole; top 21 bits: 0.56 among many
+    0.52; all 32: 0.56 three times, two of them taken, lowest indices
+    first).  N = 1,024, k = 100, against the oracle and the two-launch
+    path."""
+    N, k = 1024, 100
+    rng = np.random.default_rng(11)
+    s = np.full(N, 0.1)
+    s[rng.choice(N, 300, replace=False)] = 0.3
+    perm = rng.permutation(N)
+    if case == "level1_single":
+        s[perm[:k - 1]] = 0.9
+        s[perm[k - 1]] = 0.55
+    elif case == "level1_whole_bin":
+        s[perm[:k - 3]] = 0.9
+        s[perm[k - 3:k]] = 0.55
+    elif case == "level2":
+        s[perm[:k - 1]] = 0.9
+        s[perm[k - 1]] = 0.56
+        s[perm[k:k + 200]] = 0.52
+    else:
+        s[perm[:k - 2]] = 0.9
+        s[perm[k - 2:k + 1]] = 0.56
+        s[perm[k + 1:k + 200]] = 0.52
+    q, bank = _bank_of_scores(s)
+    idx, _ = _run(q, bank, k, cuda_device)
+    ref_idx, _ = oracle.score_select(q, bank, k)
+    np.testing.assert_array_equal(idx, ref_idx)
+    if case == "level3_ties":
+        tied = np.sort(perm[k - 2:k + 1])
+        assert set(tied[:2]) <= set(idx[0].tolist()) and tied[2] not in idx[0]
+
+
 @pytest.mark.parametrize("name,B", [("mistral_batched", 8), ("llama3_8b", 1), ("tiny", 2)])
 def test_one_launch_counters_reset_across_calls(cuda_device, name, B):
     """One workspace over calls on different banks (the one-launch path at the
