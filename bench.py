@@ -483,22 +483,29 @@ def run_gpu(args, w, world, rank, local):
             r.decode(0, mode=mode, rope=True)
     stream.synchronize()
 
-    # one graph = P rounds of R decode launches (forked over the S streams and
-    # joined again at its end); replayed T / P times per step
+    # one graph = GR rounds of R decode launches (forked over the S streams
+    # and joined again at its end; round p takes the pool's input p % P),
+    # replayed T / GR times per step; GR = P by default (8 rounds measured
+    # faster than 24 or 40 at the Llama shape)
+    GR = args.graph_rounds or P
+    if T % GR or GR % P:
+        raise SystemExit(f"--graph-rounds {GR} must divide --decode-steps {T} and be a "
+                         f"multiple of --pool {P}")
+
     def capture(m, rope=False):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             for st in streams[1:]:
                 st.wait_stream(stream)
-            for p in range(P):
+            for p in range(GR):
                 for ri, r in enumerate(reqs):
                     with torch.cuda.stream(streams[ri % S]):
-                        r.decode(p, mode=m, rope=rope)
+                        r.decode(p % P, mode=m, rope=rope)
             for st in streams[1:]:
                 stream.wait_stream(st)
         return g
     graph = capture(mode)
-    replays = T // P
+    replays = T // GR
 
     # the once-per-request kernels, also as graphs (so that their times are
     # GPU times, not Python launch rates)
@@ -575,7 +582,7 @@ def run_gpu(args, w, world, rank, local):
     select_us = 1000.0 * statistics.median(sel_ms) / R
     gather_us = 1000.0 * statistics.median(gat_ms) / R if mode == "dense" else 0.0
 
-    def time_graph(g):
+    def time_graph(g, launches):
         with torch.cuda.stream(stream):
             g.replay()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -584,21 +591,21 @@ def run_gpu(args, w, world, rank, local):
                 g.replay()
             e1.record(stream)
         stream.synchronize()
-        return 1000.0 * e0.elapsed_time(e1) / (args.variant_replays * P * R)
+        return 1000.0 * e0.elapsed_time(e1) / (args.variant_replays * launches)
 
     # the decode step with the other Tier-1 form, and the GQA-layer step with
     # rotary embedding (same state, same launch shape)
     variant = rope_variant = warm_l2 = None
     if not args.no_variant:
         g2 = capture(other)
-        v_us = time_graph(g2)
+        v_us = time_graph(g2, GR * R)
         v_bytes = decode_step_bytes(w.B, w.L, w.Hq, w.Hkv, w.d, w.k, w.W,
                                     gather=other == "gather")
         variant = {"tier1": other, "us_per_launch": v_us,
                    "achieved_gbs": v_bytes / (v_us * 1e-6) / 1e9}
         del g2
         g3 = capture(mode, rope=True)
-        r_us = time_graph(g3)
+        r_us = time_graph(g3, GR * R)
         rope_variant = {"step": "GQA layer: rotary embedding of q and k_new + append + attention",
                         "tier1": mode, "us_per_launch": r_us,
                         "achieved_gbs": nbytes / (r_us * 1e-6) / 1e9}
@@ -609,7 +616,7 @@ def run_gpu(args, w, world, rank, local):
         with torch.cuda.graph(gw, stream=stream):
             for p in range(P * R):
                 reqs[0].decode(p % P, mode=mode)
-        w_us = time_graph(gw)
+        w_us = time_graph(gw, P * R)
         warm_l2 = {"requests": 1, "us_per_launch": w_us,
                    "achieved_gbs": nbytes / (w_us * 1e-6) / 1e9,
                    "note": "one request's K/V re-read every launch (L2-resident when it "
@@ -858,8 +865,8 @@ def run_e2e(args, w, reqs, dev, stream, world, streams):
     before it (inputs double-buffered, outputs triple-buffered, so that decode
     never touches what it copies) and completes after it, so every decode
     launch keeps programmatic dependent launch and the copies overlap decode
-    work.  12 rounds (6 when T is not a multiple of 12) are captured in one
-    CUDA graph; the buffers rotate across replays, so a replay's first two
+    work.  60 rounds (12, 6 or 2 when T is not a multiple of 60) are captured
+    in one CUDA graph; the buffers rotate across replays, so a replay's first two
     copy launches carry the previous replay's last two rounds' outputs, and
     one copy launch after the step's last replay the step's last two.
     Selection and compaction run eagerly."""
@@ -874,8 +881,9 @@ def run_e2e(args, w, reqs, dev, stream, world, streams):
     # rounds per graph: a multiple of 6 super-rounds of spr rounds when T
     # allows, so that the double-buffered inputs and triple-buffered outputs
     # continue across replays and only the step's last two need a copy after
-    # the last replay
-    P = next((c for c in (12 * spr, 6 * spr, 2 * spr) if T % c == 0), None)
+    # the last replay; 60 rounds when T allows (74.1-74.2 k tokens/s at the
+    # Llama shape against 72.7 k with 12; 120 or 300: 74.4 k)
+    P = next((c for c in (60 * spr, 12 * spr, 6 * spr, 2 * spr) if T % c == 0), None)
     if P is None:  # one round per copy
         spr = 1
         P = next(c for c in (12, 6, P0, 2, T) if T % c == 0)
@@ -1081,6 +1089,9 @@ def main(argv=None):
     ap.add_argument("--requests", type=int, default=4)
     ap.add_argument("--decode-steps", type=int, default=None)
     ap.add_argument("--pool", type=int, default=8)
+    ap.add_argument("--graph-rounds", type=int, default=0,
+                    help="decode rounds per CUDA graph of the device loop (0: --pool); a "
+                         "multiple of --pool dividing the decode steps")
     ap.add_argument("--streams", type=int, default=4,
                     help="streams the independent requests' decode launches are spread over")
     ap.add_argument("--e2e-steps", type=int, default=2)
