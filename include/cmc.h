@@ -395,6 +395,17 @@ CMC_API int cmc_decode_step_rope(const void* q, const void* tier1_k, const void*
  * bits) into *flags, waiting for `stream`, and clears it when `clear` != 0. */
 CMC_API int cmc_read_status(void* workspace, int clear, uint32_t* flags, void* stream);
 
+/* Test hook for the failure path of the attention kernels (not part of the
+ * method; off unless called).  With on != 0, every pipeline stage of the
+ * attention launches made afterwards (cmc_two_tier_decode_attn,
+ * cmc_decode_step, cmc_decode_step_rope, from any thread) expects 16 bytes
+ * more than its loads deliver, so no stage ever completes: each CTA's first
+ * wait gives up after its 1 s limit, the CTA's other waits end at once, the
+ * launch returns and the workspace's status word gets CMC_DEVFLAG_TIMEOUT.
+ * Outputs, ring and pos of such a call are invalid, and its workspace must be
+ * zero-filled again.  on == 0 restores normal operation.  Always CMC_OK. */
+CMC_API int cmc_test_stall_attention_waits(int on);
+
 /* ------------------------------------------------------------------------ *
  * Staging copies for a serving loop (not a step of the paper's method: the  *
  * input and output traffic of the decode loop around it)                    *

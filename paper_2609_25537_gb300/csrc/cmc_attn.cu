@@ -119,6 +119,8 @@ struct AttnParams {
   unsigned long long rope_turns[64];  // theta^(-2i/d) / (2 pi) of the d/2 pairs as 0.64 fixed
                                       // point (turns per position), computed on the host
   int rope_slot;          // >= 0: the same table in g_rope_tables[rope_slot] (read from there)
+  uint32_t stall_tx;      // 0; the failure-path test hook: bytes every stage expects beyond
+                          // what its loads deliver, so that no stage ever completes
 };
 
 // Rotary frequency tables in device memory, one per (theta, d) a device has
@@ -664,7 +666,7 @@ __device__ __forceinline__ void finish_tile(const AttnParams& p, uint8_t* stage,
     hw[H_MASKED] = (n_rows < kTileKeys || (bad_lo | bad_hi)) ? 1 : 0;
     hw[H_BADLO] = static_cast<int>(bad_lo);
     hw[H_BADHI] = static_cast<int>(bad_hi);
-    uint32_t tx = 0;
+    uint32_t tx = p.stall_tx;   // 0 outside the failure-path test
     if (gath) tx += G * D * 2;  // query rows (box tiles: issued with the boxes)
     if (new_row >= 0) tx += 2 * D * 2;
     mbar_arrive_expect_tx(full, tx);  // releases the header
@@ -906,9 +908,11 @@ two_tier_attn_kernel(const __grid_constant__ AttnMaps maps, const AttnParams p) 
     uint8_t* stage = smem + s * S::kBytes;
     const uint8_t* aux = aux0 + s * S::kAuxBytes;
     // A stage whose wait gave up (this warp's or another's: the CTA's abort
-    // flag) is skipped: no key, no patch.  Barrier participation below does
-    // not depend on it.
-    const bool dead = attn_aborted() || !mbar_wait(&full_bar[s], static_cast<uint32_t>((i / NST) & 1));
+    // flag) is skipped: no key, no patch.  The vote makes that decision the
+    // same for every lane of the warp (the shuffles and votes below take the
+    // whole warp); barrier participation below does not depend on it.
+    const bool dead = __any_sync(0xffffffffu, attn_aborted() ||
+                                                  !mbar_wait(&full_bar[s], static_cast<uint32_t>((i / NST) & 1)));
     const int* hw = reinterpret_cast<const int*>(aux + S::kHdr);
     const int u = cc.u;
     const int n_rows = dead ? 0 : hw[H_NROWS];
@@ -1604,6 +1608,11 @@ static int dispatch_attn(const AttnMaps& maps, const AttnParams& p, int d, int G
   }
 }
 
+// The failure-path test hook (cmc_test_stall_attention_waits): bytes every
+// stage of the attention launches that follow expects beyond its loads; 0 in
+// normal use.
+static std::atomic<uint32_t> g_stall_tx{0};
+
 // theta^(-2i/d) / (2 pi) -- the pair's turns per position, below 1/6 -- as a
 // 64-bit binary fraction, rounded to nearest, computed in long double.
 static unsigned long long rope_turns_fixed(double theta, int i, int d) {
@@ -1718,6 +1727,7 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   p.scale_log2 = sc * 1.4426950408889634f;
   p.rope_offset = rope ? rope_offset : 0;
   p.l2_prefetch = kL2PrefetchTiles;
+  p.stall_tx = g_stall_tx.load(std::memory_order_relaxed);
   for (int i = 0; i < 64; ++i)
     p.rope_turns[i] = (rope && i < m.d / 2) ? rope_turns_fixed(rope_theta, i, m.d) : 0ull;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -1826,6 +1836,11 @@ int cmc_window_append(void* ring_k, void* ring_v, int64_t* pos, const void* k_ne
       static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new), m.L * m.Hkv, m.W,
       m.d);
   return check_launch();
+}
+
+int cmc_test_stall_attention_waits(int on) {
+  cmc::g_stall_tx.store(on ? 16u : 0u, std::memory_order_relaxed);
+  return CMC_OK;
 }
 
 }  // extern "C"
