@@ -114,6 +114,18 @@ def select_bytes(B, N, D, k) -> int:
     return 4 * B * N * D + 4 * B * D + 4 * B * k
 
 
+def select_launches(B, N, D, sms) -> int:
+    """Kernel launches of one cmc_score_select call with a workspace, as the
+    library chooses them: one when N <= 2,048, D <= 4,096 and CTAs of R <= 8
+    rows (R dividing N) cover the B N rows in one wave of one CTA per SM;
+    else two (scoring, then selection)."""
+    if N <= 2048 and D <= 4096:
+        for R in range(8, 0, -1):
+            if N % R == 0 and B * N // R <= sms:
+                return 1
+    return 2
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -844,7 +856,11 @@ def run_gpu(args, w, world, rank, local):
                             / 1e9, "unit": "GB/s"},
         "e2e": e2e,
         "cpu_baseline": cpu,
-        "gpu_launches": K * R * (T * step_launches + (3 if mode == "dense" else 2)),
+        # per request and step: the selection, the compaction (dense Tier-1)
+        # and T fused decode calls
+        "gpu_launches": K * R * (T * step_launches + (1 if mode == "dense" else 0)
+                                 + select_launches(w.B, w.N, w.D, torch.cuda.get_device_properties(
+                                     dev).multi_processor_count)),
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

@@ -38,3 +38,15 @@ def test_select_and_gather_bytes():
 def test_job_value_counts_every_rank():
     # tokens/s of the whole job: N ranks x steps x requests x batch x decode steps / time
     assert bench.job_tokens_per_s(2, 10, 4, 1, 3000, 1000.0) == 2 * 10 * 4 * 1 * 3000 / 1.0
+
+
+def test_select_launches_follow_the_one_launch_rule():
+    """One launch when CTAs of at most 8 rows (a divisor of N) cover the bank
+    in one wave of one CTA per SM and N <= 2,048, D <= 4,096; else two."""
+    assert bench.select_launches(1, 1024, 4096, 152) == 1      # Llama shape: 128 CTAs of 8
+    assert bench.select_launches(1, 1216, 64, 152) == 1        # 152 CTAs of 8
+    assert bench.select_launches(1, 1217, 64, 152) == 2        # prime: 1 row a CTA, 1,217 CTAs
+    assert bench.select_launches(32, 2048, 4096, 152) == 2     # Mistral batch: too many rows
+    assert bench.select_launches(1, 1024, 4100, 152) == 2      # D above 4,096
+    assert bench.select_launches(1, 4096, 64, 152) == 2        # N above 2,048
+    assert bench.select_launches(4, 256, 512, 152) == 1        # tiny batch of 4: 128 CTAs of 8
