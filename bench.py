@@ -80,6 +80,9 @@ NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 # machine-readable companion of profiles/decode_step_llama3_8b.md
 PROFILE_FILE = os.path.join(ROOT, "profiles", "decode_step_llama3_8b.json")
+# the attention launches' L2 prefetch depth for one stream of launches (the
+# library's default)
+SINGLE_STREAM_PREFETCH = 5
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2609_25537_gb300", "csrc", f)
                   for f in ("cmc_attn.cu", "cmc_internal.cuh")]
 
@@ -482,6 +485,12 @@ def run_gpu(args, w, world, rank, local):
     # concurrently; every request's steps stay in order on its stream
     S = max(1, min(args.streams, R))
     streams = [stream] + [torch.cuda.Stream(device=dev) for _ in range(S - 1)]
+    # the attention launches' L2 prefetch depth before their grid dependency
+    # wait: the library's default suits one stream of launches; with the
+    # requests on several streams (launches already overlapping) none
+    # measured best at the Llama shape (11.92 us per launch against 12.89)
+    pf = args.l2_prefetch if args.l2_prefetch >= 0 else (0 if S > 1 else SINGLE_STREAM_PREFETCH)
+    cmc.set_l2_prefetch_tiles(pf)
 
     mode = args.tier1
     other = "gather" if mode == "dense" else "dense"
@@ -624,10 +633,12 @@ def run_gpu(args, w, world, rank, local):
         del g3
         # warm-L2 companion: one request's launches back to back, so its K/V
         # (84.5 MB at the Llama shape) stays in the 129 MB L2 between launches
+        cmc.set_l2_prefetch_tiles(SINGLE_STREAM_PREFETCH)  # one stream of launches
         gw = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gw, stream=stream):
             for p in range(P * R):
                 reqs[0].decode(p % P, mode=mode)
+        cmc.set_l2_prefetch_tiles(pf)
         w_us = time_graph(gw, P * R)
         warm_l2 = {"requests": 1, "us_per_launch": w_us,
                    "achieved_gbs": nbytes / (w_us * 1e-6) / 1e9,
@@ -825,6 +836,7 @@ def run_gpu(args, w, world, rank, local):
         "config": dict(workload_config(w, R), tier1=mode),
         "tier1": mode,
         "decode_streams": S,
+        "l2_prefetch_tiles": pf,
         "decode_us_per_launch": launch_us,
         "hbm_pct_of_8tbs": 100.0 * achieved / NOMINAL_HBM_GBS,
         "select_us": select_us,
@@ -1108,6 +1120,9 @@ def main(argv=None):
     ap.add_argument("--graph-rounds", type=int, default=0,
                     help="decode rounds per CUDA graph of the device loop (0: --pool); a "
                          "multiple of --pool dividing the decode steps")
+    ap.add_argument("--l2-prefetch", type=int, default=-1,
+                    help="K/V tiles per CTA the attention launches prefetch into L2 before "
+                         "their grid dependency wait (-1: 0 with several streams, else 5)")
     ap.add_argument("--streams", type=int, default=4,
                     help="streams the independent requests' decode launches are spread over")
     ap.add_argument("--e2e-steps", type=int, default=2)

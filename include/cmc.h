@@ -395,6 +395,17 @@ CMC_API int cmc_decode_step_rope(const void* q, const void* tier1_k, const void*
  * bits) into *flags, waiting for `stream`, and clears it when `clear` != 0. */
 CMC_API int cmc_read_status(void* workspace, int clear, uint32_t* flags, void* stream);
 
+/* Tuning of the attention launches (cmc_two_tier_decode_attn,
+ * cmc_decode_step, cmc_decode_step_rope) made afterwards, from any thread:
+ * before its grid dependency wait every CTA asks L2 to prefetch the K/V boxes
+ * of its first `tiles` tiles (64 keys each), so that under programmatic
+ * dependent launch they stream in while the kernel before it on the stream
+ * drains.  A hint only: results do not depend on it.  Default 5, the best at
+ * the Llama-3-8B shape when one stream carries the launches; 0 was best when
+ * four independent requests' launches ran on four streams (their launches
+ * already overlap).  CMC_ERR_RANGE unless 0 <= tiles <= 64. */
+CMC_API int cmc_set_l2_prefetch_tiles(int tiles);
+
 /* Test hook for the failure path of the attention kernels (not part of the
  * method; off unless called).  With on != 0, every pipeline stage of the
  * attention launches made afterwards (cmc_two_tier_decode_attn,

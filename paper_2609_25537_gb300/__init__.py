@@ -20,6 +20,7 @@ from .cmc import (  # noqa: F401
     question_select,
     score_select,
     score_select_workspace_size,
+    set_l2_prefetch_tiles,
     stage_copies,
     tier1_gather,
     two_tier_decode_attn,

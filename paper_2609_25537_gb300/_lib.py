@@ -32,6 +32,7 @@ EXPORTS = (
     "cmc_tier1_gather",
     "cmc_decode_attn_plan",
     "cmc_read_status",
+    "cmc_set_l2_prefetch_tiles",
     "cmc_test_stall_attention_waits",
     "cmc_stage_copies",
     "cmc_score_select_static",
@@ -107,6 +108,7 @@ _SIGNATURES = {
     "cmc_tier1_gather": (_i, [_vp, _vp, _vp, _dims_p, _vp, _vp, _vp, _vp]),
     "cmc_decode_attn_plan": (_i, [_dims_p, _i, ctypes.POINTER(_i), ctypes.POINTER(_i)]),
     "cmc_read_status": (_i, [_vp, _i, ctypes.POINTER(ctypes.c_uint32), _vp]),
+    "cmc_set_l2_prefetch_tiles": (_i, [_i]),
     "cmc_test_stall_attention_waits": (_i, [_i]),
     "cmc_stage_copies": (_i, [_vp, _i, _i, _vp]),
     "cmc_score_select_static": (_i, [_vp, _vp, _i, _i, _i, _i, _vp, _vp]),

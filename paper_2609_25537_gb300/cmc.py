@@ -44,6 +44,7 @@ __all__ = [
     "tier1_gather",
     "decode_attn_workspace_size",
     "decode_attn_plan",
+    "set_l2_prefetch_tiles",
     "dims_of",
     "stage_copies",
     "DEVFLAG_BAD_INDEX",
@@ -394,6 +395,14 @@ def decode_step(q, tier1_k, tier1_v, idx, ring_k, ring_v, pos, k_new, v_new, *,
             int(rope_offset), _p(out), _p(ws.buf), ws.nbytes, _stream(dev))
         check(st, "cmc_decode_step_rope")
     return out
+
+
+def set_l2_prefetch_tiles(tiles: int) -> None:
+    """Box tiles per CTA the attention launches made afterwards prefetch into
+    L2 before their grid dependency wait (a hint); see
+    cmc_set_l2_prefetch_tiles.  Default 5 (one stream of launches); 0 suits
+    several streams of independent requests' launches."""
+    check(lib().cmc_set_l2_prefetch_tiles(int(tiles)), "cmc_set_l2_prefetch_tiles")
 
 
 @_ranged

@@ -1444,8 +1444,14 @@ constexpr int kStages = 3;
 // best at the Llama-3-8B shape (14.20 us against 14.34 for four, 14.30 for six,
 // 14.7 for three or eight); without the evict-first policy one tile was best.
 // A rolling prefetch a few tiles ahead of the TMA issue, on top, was slower at
-// every distance (16.2-16.9 us).
+// every distance (16.2-16.9 us).  That is for one stream of launches: with
+// independent requests' launches on four streams, whose launches already run
+// through each other's edges, no prefetch measured best (11.92 us against
+// 12.11 for one tile, 12.32 for two, 12.89 for five), so the depth is a
+// setting (cmc_set_l2_prefetch_tiles) with this default.
 constexpr int kL2PrefetchTiles = 5;
+constexpr int kMaxL2PrefetchTiles = 64;
+static std::atomic<int> g_l2_prefetch_tiles{kL2PrefetchTiles};
 
 // Launch plan of one attention call on the current device.
 struct AttnPlan {
@@ -1726,7 +1732,7 @@ static int run_attention(const void* q, const void* tier1_k, const void* tier1_v
   const float sc = scale > 0.f ? scale : 1.0f / sqrtf(static_cast<float>(m.d));
   p.scale_log2 = sc * 1.4426950408889634f;
   p.rope_offset = rope ? rope_offset : 0;
-  p.l2_prefetch = kL2PrefetchTiles;
+  p.l2_prefetch = g_l2_prefetch_tiles.load(std::memory_order_relaxed);
   p.stall_tx = g_stall_tx.load(std::memory_order_relaxed);
   for (int i = 0; i < 64; ++i)
     p.rope_turns[i] = (rope && i < m.d / 2) ? rope_turns_fixed(rope_theta, i, m.d) : 0ull;
@@ -1836,6 +1842,12 @@ int cmc_window_append(void* ring_k, void* ring_v, int64_t* pos, const void* k_ne
       static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new), m.L * m.Hkv, m.W,
       m.d);
   return check_launch();
+}
+
+int cmc_set_l2_prefetch_tiles(int tiles) {
+  if (tiles < 0 || tiles > cmc::kMaxL2PrefetchTiles) return CMC_ERR_RANGE;
+  cmc::g_l2_prefetch_tiles.store(tiles, std::memory_order_relaxed);
+  return CMC_OK;
 }
 
 int cmc_test_stall_attention_waits(int on) {

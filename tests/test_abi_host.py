@@ -298,3 +298,21 @@ def test_stage_copies_argument_checks(L):
     assert call([(FAKE + 8, FAKE, 64)], 1) == ALIGN
     assert call([(FAKE, FAKE + 4, 64)], 1) == ALIGN
     assert call([(FAKE, FAKE, 40)], 1) == ALIGN
+
+
+def test_l2_prefetch_setting_range(L):
+    """The attention launches' prefetch depth: 0 to 64 tiles, else
+    CMC_ERR_RANGE (host logic only; the default is put back)."""
+    assert L.cmc_set_l2_prefetch_tiles(-1) == 3
+    assert L.cmc_set_l2_prefetch_tiles(65) == 3
+    assert L.cmc_set_l2_prefetch_tiles(0) == 0
+    assert L.cmc_set_l2_prefetch_tiles(64) == 0
+    assert L.cmc_set_l2_prefetch_tiles(5) == 0
+
+
+def test_binding_sets_l2_prefetch():
+    """The package-level binding of the prefetch setting (host logic only)."""
+    cmc.set_l2_prefetch_tiles(0)
+    cmc.set_l2_prefetch_tiles(5)
+    with pytest.raises(cmc.CmcError):
+        cmc.set_l2_prefetch_tiles(65)

@@ -714,3 +714,28 @@ def test_rope_many_thetas(cuda_device):
     w = WORKLOADS["tiny"].with_(B=1, T=1)
     for j in range(20):
         _rope_run(w, cuda_device, "dense", theta=1000.0 + 97.5 * j, offset=w.k)
+
+
+@pytest.mark.parametrize("tiles", [0, 64])
+def test_l2_prefetch_depth_changes_no_result(cuda_device, tiles):
+    """The pre-wait L2 prefetch depth is a hint: at the 32-layer Llama shape
+    (dense Tier-1, one CTA per unit) steps with no prefetch or the deepest
+    one give the same bits as the default depth of 5, and match the oracle."""
+    w = WORKLOADS["llama3_8b"]
+    idx = random_tier1_indices(w)
+    outs = {}
+    try:
+        for depth in (5, tiles):
+            cmc.set_l2_prefetch_tiles(depth)
+            P = Problem(w, cuda_device, idx=idx, mode="dense")
+            got = []
+            for t in range(3):
+                out, ref = P.step(step_inputs(w, t))
+                assert_attn_close(to_f64(out), ref, f"prefetch {depth} step {t}")
+                got.append(host_bits(out))
+            P.check_state()
+            outs[depth] = got
+    finally:
+        cmc.set_l2_prefetch_tiles(5)
+    for a, b in zip(outs[5], outs[tiles]):
+        np.testing.assert_array_equal(a, b)
