@@ -150,17 +150,20 @@ def kernel_source_hash() -> str:
 def profiled_traffic(workload: str, tier1: str):
     """DRAM bytes per launch of the fused decode kernel from the committed ncu
     record, if it was taken on the current kernel source, for this workload
-    and Tier-1 form; else None."""
+    and Tier-1 form: (in the benchmark's request loop, with L2 carried over
+    between launches; one launch with L2 flushed before it), either None
+    when not recorded; (None, None) otherwise."""
     try:
         with open(PROFILE_FILE) as f:
             rec = json.load(f)
         if rec["kernel_source_sha256"] != kernel_source_hash():
-            return None
+            return None, None
         if (rec["workload"], rec["tier1"]) != (workload, tier1):
-            return None
-        return int(rec["dram_bytes_per_launch"])
-    except (OSError, ValueError, KeyError, TypeError):
-        return None
+            return None, None
+        loop = rec.get("in_loop", {}).get("dram_bytes_per_launch")
+        return (int(loop) if loop is not None else None), int(rec["dram_bytes_per_launch"])
+    except (OSError, ValueError, KeyError, TypeError, AttributeError):
+        return None, None
 
 
 # ----------------------------------------------------------------------------
@@ -828,6 +831,10 @@ def run_gpu(args, w, world, rank, local):
 
     if rank != 0:
         return 0
+    # DRAM bytes per launch from the committed ncu record: in the request loop
+    # (L2 carried over between launches: part of a request's K/V survives the
+    # other requests' traffic) and with L2 flushed
+    traffic_loop, traffic_cold = profiled_traffic(w.name, mode)
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": K, "warmup": args.warmup, "ms_per_step": max_ms / K,
@@ -861,7 +868,8 @@ def run_gpu(args, w, world, rank, local):
                      "frac": achieved / peak, "peak_kind": f"hbm copy, {peak_kind}",
                      "kernel": (f"fused decode step: two_tier_attn_kernel<{w.d},{w.Hq // w.Hkv},fused,3>"
                                 + plan_txt),
-                     "bytes_per_launch": nbytes, "traffic": profiled_traffic(w.name, mode),
+                     "bytes_per_launch": nbytes, "traffic": traffic_loop,
+                     "traffic_cold": traffic_cold,
                      "flops_per_launch": decode_step_flops(w.B, w.L, w.Hq, w.d, w.k, w.W)},
         "select_roofline": {"bound": "hbm", "bytes": select_bytes(w.B, w.N, w.D, w.k),
                             "achieved": select_bytes(w.B, w.N, w.D, w.k) / (select_us * 1e-6)
