@@ -50,3 +50,25 @@ def test_select_launches_follow_the_one_launch_rule():
     assert bench.select_launches(1, 1024, 4100, 152) == 2      # D above 4,096
     assert bench.select_launches(1, 4096, 64, 152) == 2        # N above 2,048
     assert bench.select_launches(4, 256, 512, 152) == 1        # tiny batch of 4: 128 CTAs of 8
+
+
+def test_profiled_traffic_reads_both_figures(tmp_path, monkeypatch):
+    """The traffic record: (request-loop bytes, flushed-cache bytes) while its
+    kernel hash and workload match the current source and run; (None, None)
+    otherwise; the loop figure None when the record has none."""
+    import json
+    rec = {"workload": "llama3_8b", "tier1": "dense", "dram_bytes_per_launch": 86,
+           "kernel_source_sha256": bench.kernel_source_hash(),
+           "in_loop": {"dram_bytes_per_launch": 77}}
+    f = tmp_path / "rec.json"
+    f.write_text(json.dumps(rec))
+    monkeypatch.setattr(bench, "PROFILE_FILE", str(f))
+    assert bench.profiled_traffic("llama3_8b", "dense") == (77, 86)
+    assert bench.profiled_traffic("llama3_8b", "gather") == (None, None)
+    assert bench.profiled_traffic("tiny", "dense") == (None, None)
+    del rec["in_loop"]
+    f.write_text(json.dumps(rec))
+    assert bench.profiled_traffic("llama3_8b", "dense") == (None, 86)
+    rec["kernel_source_sha256"] = "0" * 64
+    f.write_text(json.dumps(rec))
+    assert bench.profiled_traffic("llama3_8b", "dense") == (None, None)
