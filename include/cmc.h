@@ -20,7 +20,11 @@
  * ---------------------------------------
  *  - Every tensor argument is a DEVICE pointer to memory the caller owns.  The
  *    library allocates no memory and keeps no state between calls apart from
- *    the thread-local last CUDA error and a per-device SM-count cache.
+ *    the thread-local last CUDA error, a per-device SM-count cache, the
+ *    per-device rotary frequency tables of cmc_decode_step_rope (written once
+ *    per (theta, d)), the static score array of cmc_score_select_static and
+ *    two process-wide settings of the attention launches
+ *    (cmc_set_l2_prefetch_tiles, cmc_test_stall_attention_waits).
  *  - All work is enqueued on `stream` (a cudaStream_t passed as void*; NULL is
  *    the legacy default stream) and is asynchronous: a return of CMC_OK means
  *    the launch was accepted, not that it has finished.
